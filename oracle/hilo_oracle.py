@@ -1,0 +1,360 @@
+"""CPU oracle for the HiLo-Token hot path -- TEST INFRASTRUCTURE ONLY.
+
+Only the tests, the smoke check and the benchmark's CPU-baseline leg may
+import this module. The product path never calls it: it shares no code with
+the CUDA library (no kernels, headers, helpers, constants or tables) and
+imports nothing from the package.
+
+What it computes, step by step (paper: Sec. 2.3 "HiLo-Token Selection" and
+the DiT it feeds; the concrete variant -- token-space score, top-k split,
+2x2/4x4 pooling, MMDiT block -- is the one the hot path implements):
+
+  score   per-token high-frequency energy  s_i = sum_c (x_ic - m_w(i),c)^2,
+          m_w the mean of the aligned 2x2 window holding token i
+          (the token-space stand-in for the Sobel frequency map + 16x
+          regionalisation of Sec. 2.3).
+  split   keep = top-k tokens by (score desc, index asc) united with the edit
+          mask (Sec. 2.3: tokens inside the mask are always retained); the
+          rest is pooled 2x2, or for two-level pooling the next k_mid tokens
+          are pooled 2x2 and the remainder 4x4.
+  pack    the packed image sequence per image: kept tokens in raster order,
+          then one row per 2x2 window (mean of that window's 2x2-pooled
+          members), then one row per 4x4 window (Sec. 2.3: selected tokens
+          concatenated with the low-frequency tokens along the token axis).
+  block   an MMDiT-style block on the joint [text ; packed image] sequence:
+          pre-LayerNorm (no affine), two-stream QKV / out / MLP weights, joint
+          softmax attention, tanh-GELU 4x MLP, residual adds.
+  unpack  every grid token reads the output row of its kept token or of its
+          window (nearest broadcast).
+  update  x <- bf16(x - alpha * y) for the denoising loop.
+
+Precision. Where a float decides an integer or a stored bf16 code (the score
+decides the split; the pooled mean is stored as bf16; the loop update is
+stored as bf16) the oracle computes in fp32 with one fixed order of
+operations and no fused multiply-add, the precision the kernels use. The
+block is computed in fp64 from the exact bf16 inputs and weights.
+
+Fixed orders (readings where the paper is silent):
+  * window mean for the score: ((x_a + x_b) + (x_c + x_d)) * 0.25 with
+    members a,b,c,d in raster order;
+  * channel sum: channels are taken in groups of 8 consecutive channels;
+    group g is folded into partial sum p[g mod 32] (groups ascending, the 8
+    channels of a group ascending); the 32 partials are then combined by the
+    halving tree p[j] += p[j + h] for h = 16, 8, 4, 2, 1;
+  * pooled mean: fp32 sum of the class members in raster order starting from
+    the first member, one correctly rounded division by the member count,
+    then bf16 round-to-nearest-even.
+
+Bit patterns of bf16 arrays are carried as numpy uint16.
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+
+import numpy as np
+
+KEEP = 0
+POOL2 = 1
+POOL4 = 2
+
+# ---------------------------------------------------------------------------
+# bf16 conversion (own implementation; pinned against torch in the tests)
+# ---------------------------------------------------------------------------
+
+
+def bf16_to_f32(bits: np.ndarray) -> np.ndarray:
+    """Exact widening of bf16 bit patterns to fp32."""
+    return (np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)).view(np.float32)
+
+
+def f32_to_bf16(a: np.ndarray) -> np.ndarray:
+    """fp32 -> bf16 bit pattern, round to nearest, ties to even (finite inputs)."""
+    u = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    keep_lsb = (u >> np.uint64(16)) & np.uint64(1)
+    rounded = (u + np.uint64(0x7FFF) + keep_lsb) >> np.uint64(16)
+    return rounded.astype(np.uint16)
+
+
+# ---------------------------------------------------------------------------
+# Step 1: frequency score (fp32, fixed order)
+# ---------------------------------------------------------------------------
+
+
+def score(x_bits: np.ndarray) -> np.ndarray:
+    """Per-token energy of x minus its 2x2 average-pooled-then-upsampled value.
+
+    x_bits: uint16 [B,H,W,d] (bf16); H, W even; d a multiple of 8.
+    Returns fp32 [B, H*W].
+    """
+    B, H, W, d = x_bits.shape
+    assert H % 2 == 0 and W % 2 == 0 and d % 8 == 0
+    x = bf16_to_f32(x_bits)
+    a = x[:, 0::2, 0::2, :]
+    b = x[:, 0::2, 1::2, :]
+    c = x[:, 1::2, 0::2, :]
+    e = x[:, 1::2, 1::2, :]
+    m = ((a + b) + (c + e)) * np.float32(0.25)                 # [B,H/2,W/2,d]
+    up = np.repeat(np.repeat(m, 2, axis=1), 2, axis=2)          # nearest upsample
+    diff = x - up
+    sq = diff * diff                                            # fp32, no FMA
+    sq = sq.reshape(B, H * W, d)
+    partial = np.zeros((B, H * W, 32), dtype=np.float32)
+    for g in range(d // 8):
+        j = g % 32
+        for u in range(8):
+            partial[:, :, j] = partial[:, :, j] + sq[:, :, 8 * g + u]
+    for h in (16, 8, 4, 2, 1):
+        partial[:, :, :h] = partial[:, :, :h] + partial[:, :, h:2 * h]
+    return np.ascontiguousarray(partial[:, :, 0])
+
+
+def score_f64(x_bits: np.ndarray) -> np.ndarray:
+    """The same energy in fp64, summed plainly (a sanity reference)."""
+    B, H, W, d = x_bits.shape
+    x = bf16_to_f32(x_bits).astype(np.float64)
+    m = x.reshape(B, H // 2, 2, W // 2, 2, d).mean(axis=(2, 4))
+    up = np.repeat(np.repeat(m, 2, axis=1), 2, axis=2)
+    return ((x - up) ** 2).sum(axis=-1).reshape(B, H * W)
+
+
+# ---------------------------------------------------------------------------
+# Step 2: keep / pool split
+# ---------------------------------------------------------------------------
+
+
+@dataclasses.dataclass
+class Split:
+    labels: np.ndarray    # uint8 [B,N]   KEEP / POOL2 / POOL4
+    row_src: np.ndarray   # int32 [rows]  token id (kept rows) or window id (pooled rows)
+    counts: np.ndarray    # int32 [B,3]   kept tokens, 2x2 windows, 4x4 windows
+    cu_img: np.ndarray    # int32 [B+1]   packed image-row offsets
+    tok_row: np.ndarray   # int32 [B,N]   packed row each grid token reads back
+
+
+def ranking(s: np.ndarray) -> np.ndarray:
+    """Token ids ordered by (score descending, token index ascending)."""
+    idx = np.arange(s.shape[0])
+    return np.lexsort((idx, -s.astype(np.float64)))
+
+
+def split(s: np.ndarray, mask: np.ndarray, k_keep, k_mid, H: int, W: int, levels: int) -> Split:
+    """Deterministic keep/pool split of each image (see module docstring)."""
+    B, N = s.shape
+    assert N == H * W and levels in (1, 2)
+    labels = np.empty((B, N), dtype=np.uint8)
+    counts = np.zeros((B, 3), dtype=np.int32)
+    cu = np.zeros(B + 1, dtype=np.int32)
+    tok_row = np.empty((B, N), dtype=np.int32)
+    rows = []
+    p = np.arange(N) // W
+    q = np.arange(N) % W
+    win2_of = (p // 2) * (W // 2) + (q // 2)
+    win4_of = (p // 4) * (W // 4) + (q // 4) if levels == 2 else None
+    for b in range(B):
+        order = ranking(s[b])
+        keep = mask[b].astype(bool).copy()
+        keep[order[:int(k_keep[b])]] = True
+        lab = np.full(N, POOL2, dtype=np.uint8)
+        lab[keep] = KEEP
+        if levels == 2:
+            rest = order[~keep[order]]
+            lab[rest[int(k_mid[b]):]] = POOL4
+        labels[b] = lab
+        kept = np.nonzero(lab == KEEP)[0]
+        w2 = np.unique(win2_of[lab == POOL2])
+        w4 = np.unique(win4_of[lab == POOL4]) if levels == 2 else np.zeros(0, dtype=np.int64)
+        counts[b] = (len(kept), len(w2), len(w4))
+        cu[b + 1] = cu[b] + len(kept) + len(w2) + len(w4)
+        rows += [kept, w2, w4]
+        base = int(cu[b])
+        tok_row[b, kept] = base + np.arange(len(kept))
+        r2 = {int(w): base + len(kept) + i for i, w in enumerate(w2)}
+        r4 = {int(w): base + len(kept) + len(w2) + i for i, w in enumerate(w4)}
+        for i in np.nonzero(lab == POOL2)[0]:
+            tok_row[b, i] = r2[int(win2_of[i])]
+        for i in np.nonzero(lab == POOL4)[0]:
+            tok_row[b, i] = r4[int(win4_of[i])]
+    row_src = np.concatenate([np.asarray(r, dtype=np.int64) for r in rows]).astype(np.int32) \
+        if rows else np.zeros(0, np.int32)
+    return Split(labels, row_src, counts, cu, tok_row)
+
+
+# ---------------------------------------------------------------------------
+# Step 3: pack (gather + average pooling)
+# ---------------------------------------------------------------------------
+
+
+def window_members(w: int, size: int, W: int) -> list[int]:
+    """Token ids of aligned size x size window ``w`` in raster order."""
+    wp, wq = divmod(w, W // size)
+    return [(size * wp + i) * W + size * wq + j for i in range(size) for j in range(size)]
+
+
+def pack(x_bits: np.ndarray, sp: Split) -> np.ndarray:
+    """Packed image rows, uint16 [rows, d] (bf16)."""
+    B, H, W, d = x_bits.shape
+    x = bf16_to_f32(x_bits).reshape(B, H * W, d)
+    out = np.empty((int(sp.cu_img[-1]), d), dtype=np.uint16)
+    for b in range(B):
+        nk, n2, n4 = (int(c) for c in sp.counts[b])
+        base = int(sp.cu_img[b])
+        for r in range(nk + n2 + n4):
+            src = int(sp.row_src[base + r])
+            if r < nk:
+                out[base + r] = x_bits.reshape(B, H * W, d)[b, src]
+                continue
+            size, cls = (2, POOL2) if r < nk + n2 else (4, POOL4)
+            members = [t for t in window_members(src, size, W) if sp.labels[b, t] == cls]
+            acc = x[b, members[0]].copy()
+            for t in members[1:]:
+                acc = acc + x[b, t]
+            mean = acc / np.float32(len(members))
+            out[base + r] = f32_to_bf16(mean)
+    return out
+
+
+# ---------------------------------------------------------------------------
+# Step 4: MMDiT block (fp64)
+# ---------------------------------------------------------------------------
+
+
+def layer_norm(u: np.ndarray, eps: float = 1e-6) -> np.ndarray:
+    """LayerNorm over the last axis, no affine, biased variance."""
+    mu = u.mean(axis=-1, keepdims=True)
+    var = ((u - mu) ** 2).mean(axis=-1, keepdims=True)
+    return (u - mu) / np.sqrt(var + eps)
+
+
+def gelu_tanh(z: np.ndarray) -> np.ndarray:
+    """GELU, tanh approximation."""
+    return 0.5 * z * (1.0 + np.tanh(math.sqrt(2.0 / math.pi) * (z + 0.044715 * z ** 3)))
+
+
+def softmax_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray) -> np.ndarray:
+    """Non-causal softmax attention of one head, scale 1/sqrt(head_dim)."""
+    sc = (q @ k.T) / math.sqrt(q.shape[-1])
+    sc = sc - sc.max(axis=-1, keepdims=True)
+    p = np.exp(sc)
+    p = p / p.sum(axis=-1, keepdims=True)
+    return p @ v
+
+
+def _w(bits) -> np.ndarray:
+    return bf16_to_f32(bits).astype(np.float64)
+
+
+def _as_f64(u) -> np.ndarray:
+    return bf16_to_f32(u).astype(np.float64) if u.dtype == np.uint16 else np.asarray(u, np.float64)
+
+
+def block(u_txt, u_img, cu_img, T: int, weights, heads: int, mlp: bool):
+    """One MMDiT block on the joint sequence of each image.
+
+    u_txt: [B*T, d] text rows (image b owns rows b*T .. b*T+T-1);
+    u_img: [rows, d] packed image rows (image b owns cu_img[b] .. cu_img[b+1]-1).
+    Either may be bf16 bits (uint16) or floats. Returns fp64 (txt, img).
+    ``weights`` has ``.txt`` and ``.img`` with PyTorch-layout [out, in] arrays.
+    """
+    ut = _as_f64(u_txt)
+    ui = _as_f64(u_img)
+    d = ut.shape[1] if ut.size else ui.shape[1]
+    hd = d // heads
+    B = len(cu_img) - 1
+    streams = ((ut, weights.txt), (ui, weights.img))
+    qkv = [layer_norm(u) @ _w(w.w_qkv).T + _w(w.b_qkv) for u, w in streams]
+    att = [np.zeros_like(ut), np.zeros_like(ui)]
+    for b in range(B):
+        t0, t1 = b * T, (b + 1) * T
+        i0, i1 = int(cu_img[b]), int(cu_img[b + 1])
+        joint = np.concatenate([qkv[0][t0:t1], qkv[1][i0:i1]], axis=0)
+        o = np.empty((joint.shape[0], d))
+        for h in range(heads):
+            c = slice(h * hd, (h + 1) * hd)
+            o[:, c] = softmax_attention(joint[:, c], joint[:, d:][:, c], joint[:, 2 * d:][:, c])
+        att[0][t0:t1] = o[:T]
+        att[1][i0:i1] = o[T:]
+    out = []
+    for (u, w), a in zip(streams, att):
+        u = u + a @ _w(w.w_o).T + _w(w.b_o)
+        if mlp:
+            u = u + gelu_tanh(layer_norm(u) @ _w(w.w_1).T + _w(w.b_1)) @ _w(w.w_2).T + _w(w.b_2)
+        out.append(u)
+    return out[0], out[1]
+
+
+def block_rows(u_txt, u_img, cu_img, T: int, weights, heads: int, mlp: bool, b: int,
+               txt_rows, img_rows):
+    """The block's outputs for selected rows of image ``b`` only.
+
+    Same arithmetic as ``block``; keys and values of the whole joint sequence
+    of image b are projected, queries, attention and MLP only for the given
+    rows (absolute row ids in u_txt / u_img). Returns fp64 (txt_out, img_out).
+    """
+    ut = _as_f64(u_txt)
+    ui = _as_f64(u_img)
+    d = ut.shape[1]
+    hd = d // heads
+    t0, t1 = b * T, (b + 1) * T
+    i0, i1 = int(cu_img[b]), int(cu_img[b + 1])
+    wt, wi = weights.txt, weights.img
+    ln_t = layer_norm(ut[t0:t1])
+    ln_i = layer_norm(ui[i0:i1])
+    kv = np.concatenate([ln_t @ _w(wt.w_qkv[d:]).T + _w(wt.b_qkv[d:]),
+                         ln_i @ _w(wi.w_qkv[d:]).T + _w(wi.b_qkv[d:])], axis=0)
+    res = []
+    for rows, u_all, w in ((np.asarray(txt_rows, int), ut, wt), (np.asarray(img_rows, int), ui, wi)):
+        if rows.size == 0:
+            res.append(np.zeros((0, d)))
+            continue
+        u = u_all[rows]
+        q = layer_norm(u) @ _w(w.w_qkv[:d]).T + _w(w.b_qkv[:d])
+        o = np.empty((len(rows), d))
+        for h in range(heads):
+            c = slice(h * hd, (h + 1) * hd)
+            o[:, c] = softmax_attention(q[:, c], kv[:, :d][:, c], kv[:, d:][:, c])
+        u = u + o @ _w(w.w_o).T + _w(w.b_o)
+        if mlp:
+            u = u + gelu_tanh(layer_norm(u) @ _w(w.w_1).T + _w(w.b_1)) @ _w(w.w_2).T + _w(w.b_2)
+        res.append(u)
+    return res[0], res[1]
+
+
+def block_dense(x_bits, text_bits, weights, heads: int, mlp: bool):
+    """The uncompressed block: every grid token in raster order, no pooling."""
+    B, H, W, d = x_bits.shape
+    cu = np.arange(B + 1, dtype=np.int64) * (H * W)
+    return block(text_bits.reshape(B * text_bits.shape[1], d), x_bits.reshape(B * H * W, d),
+                 cu, text_bits.shape[1], weights, heads, mlp)
+
+
+# ---------------------------------------------------------------------------
+# Step 5: unpack, and the denoising-loop update
+# ---------------------------------------------------------------------------
+
+
+def unpack(out_img: np.ndarray, sp: Split) -> np.ndarray:
+    """y[b, i] = out_img[tok_row[b, i]]  ->  [B, N, d]."""
+    return out_img[sp.tok_row]
+
+
+def update(x_bits: np.ndarray, y: np.ndarray, alpha: float) -> np.ndarray:
+    """x <- bf16(x - alpha * y), fp32 multiply then subtract (no FMA)."""
+    x = bf16_to_f32(x_bits)
+    t = np.float32(alpha) * np.asarray(y, dtype=np.float32)
+    return f32_to_bf16(x - t)
+
+
+def hot_path(x_bits, text_bits, mask, k_keep, k_mid, levels, weights_list, heads, mlp):
+    """score -> split -> pack -> blocks -> unpack for one batch.
+
+    Returns (split, packed, (txt_out, img_out), y) with the block outputs in fp64.
+    """
+    B, H, W, d = x_bits.shape
+    T = text_bits.shape[1]
+    sp = split(score(x_bits), mask, k_keep, k_mid, H, W, levels)
+    packed = pack(x_bits, sp)
+    ut, ui = text_bits.reshape(B * T, d), packed
+    for wts in weights_list:
+        ut, ui = block(ut, ui, sp.cu_img, T, wts, heads, mlp)
+    return sp, packed, (ut, ui), unpack(ui, sp)

@@ -1,0 +1,418 @@
+"""Pins of the CPU oracle against facts that do not come from the oracle itself.
+
+Closed forms, hand-worked examples (tests/golden), special cases that reduce to
+a library routine, brute force on tiny inputs and invariants of the method
+(Sec. 2.3 of the paper: kept tokens stay at full resolution, low-frequency
+tokens are pooled, the sequence is concatenated along the token axis).
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import hilo_oracle as O
+from paper_2606_13898_gb300 import inputs as I
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def bits(a):
+    return I.f32_to_bf16_bits(np.asarray(a, dtype=np.float32))
+
+
+# ---------------------------------------------------------------- bf16 -----
+
+def test_bf16_rounding_matches_torch():
+    rng = np.random.default_rng(5)
+    v = np.concatenate([rng.standard_normal(20000).astype(np.float32) * 10,
+                        # exact ties between two bf16 neighbours (even and odd)
+                        np.array([1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, -1.0 - 2 ** -8, 0.0, -0.0,
+                                  3.0e38, 1e-40], dtype=np.float32)])
+    ref = torch.from_numpy(v).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(O.f32_to_bf16(v), ref)
+    assert np.array_equal(O.bf16_to_f32(ref), torch.from_numpy(ref.view(np.int16)).view(torch.bfloat16).float().numpy())
+
+
+# --------------------------------------------------------------- score -----
+
+def test_score_constant_field_is_zero():
+    x = np.full((1, 8, 8, 64), 1.75, dtype=np.float32)
+    x[..., 5] = -3.0
+    assert np.all(O.score(bits(x)) == 0.0)
+
+
+def test_score_checkerboard_closed_form():
+    # +-a alternating in both directions: every 2x2 window has mean 0, so each
+    # channel contributes a^2 and the score is d * a^2 for every token.
+    a, d = 0.75, 256
+    p = np.arange(8)[:, None]
+    q = np.arange(6)[None, :]
+    sign = np.where((p + q) % 2 == 0, 1.0, -1.0)
+    x = (a * sign)[None, :, :, None] * np.ones(d)[None, None, None, :]
+    s = O.score(bits(x))
+    assert np.all(s == np.float32(d * a * a))
+
+
+def test_score_linear_ramp_closed_form():
+    # x = alpha*p + beta*q (+ a per-channel constant): inside window (P,Q) the
+    # mean is alpha*(2P+1/2) + beta*(2Q+1/2), so token (2P+i, 2Q+j) has the
+    # residual alpha*(i-1/2) + beta*(j-1/2) in every channel.
+    alpha, beta, d = 0.5, 0.25, 64
+    H, W = 8, 8
+    p = np.arange(H)[:, None, None]
+    q = np.arange(W)[None, :, None]
+    off = (np.arange(d) % 4)[None, None, :] * 0.25
+    x = alpha * p + beta * q + off
+    s = O.score(bits(x[None]))[0].reshape(H, W)
+    for i in (0, 1):
+        for j in (0, 1):
+            e = alpha * (i - 0.5) + beta * (j - 0.5)
+            assert np.all(s[i::2, j::2] == np.float32(d * e * e)), (i, j)
+
+
+def test_score_agrees_with_fp64_sum():
+    wl = I.tiny_layer()
+    b = I.make_batch(wl)
+    s32 = O.score(b.x).astype(np.float64)
+    s64 = O.score_f64(b.x)
+    assert np.max(np.abs(s32 - s64) / np.maximum(s64, 1e-30)) < 1e-5
+
+
+def test_score_fixed_order_scalar_walkthrough():
+    # One token of a random field walked through the fixed order with scalar
+    # fp32 arithmetic: pins the vectorised grouping and the halving tree.
+    rng = np.random.default_rng(11)
+    d = 512
+    xb = bits(rng.standard_normal((1, 2, 2, d)))
+    x = O.bf16_to_f32(xb)[0]
+    f = np.float32
+    for t, (pi, qi) in enumerate(((0, 0), (0, 1), (1, 0), (1, 1))):
+        part = [f(0.0)] * 32
+        for c in range(d):
+            m = ((x[0, 0, c] + x[0, 1, c]) + (x[1, 0, c] + x[1, 1, c])) * f(0.25)
+            e = f(x[pi, qi, c] - m)
+            g = c // 8
+            part[g % 32] = f(part[g % 32] + f(e * e))
+        for h in (16, 8, 4, 2, 1):
+            for j in range(h):
+                part[j] = f(part[j] + part[j + h])
+        assert O.score(xb)[0, t] == part[0]
+
+
+# --------------------------------------------------------------- split -----
+
+def _golden_cases():
+    with open(os.path.join(GOLDEN, "split_worked_examples.json")) as fh:
+        return json.load(fh)["cases"]
+
+
+@pytest.mark.parametrize("case", _golden_cases(), ids=lambda c: c["name"])
+def test_split_hand_worked(case):
+    s = np.array([case["score"]], dtype=np.float32)
+    m = np.array([case["mask"]], dtype=np.uint8)
+    sp = O.split(s, m, [case["k_keep"]], [case["k_mid"]], case["H"], case["W"], case["levels"])
+    assert sp.labels[0].tolist() == case["labels"]
+    assert sp.row_src.tolist() == case["row_src"]
+    assert sp.counts[0].tolist() == case["counts"]
+    assert sp.cu_img.tolist() == case["cu_img"]
+    assert sp.tok_row[0].tolist() == case["tok_row"]
+
+
+def _brute_split(s, m, k, kmid, H, W, levels):
+    """Pure-Python split of one image from the rule, by full sort."""
+    N = H * W
+    order = sorted(range(N), key=lambda i: (-float(s[i]), i))
+    keep = set(order[:k]) | {i for i in range(N) if m[i]}
+    rest = [i for i in order if i not in keep]
+    pool2 = set(rest[:kmid]) if levels == 2 else set(rest)
+    pool4 = set(rest[kmid:]) if levels == 2 else set()
+    w2 = sorted({(i // W // 2) * (W // 2) + (i % W) // 2 for i in pool2})
+    w4 = sorted({(i // W // 4) * (W // 4) + (i % W) // 4 for i in pool4})
+    return sorted(keep), w2, w4, pool2, pool4
+
+
+@pytest.mark.parametrize("levels", [1, 2])
+@pytest.mark.parametrize("seed", range(6))
+def test_split_brute_force(seed, levels):
+    rng = np.random.default_rng(seed)
+    H, W = (8, 8) if seed % 2 else (4, 12)
+    N = H * W
+    B = 3
+    # coarse scores so that ties are common
+    s = (rng.integers(0, 6, size=(B, N)) * 0.5).astype(np.float32)
+    m = (rng.random((B, N)) < 0.15).astype(np.uint8)
+    kk = rng.integers(0, N + 1, size=B)
+    km = rng.integers(0, N + 1, size=B)
+    sp = O.split(s, m, kk, km, H, W, levels)
+    for b in range(B):
+        keep, w2, w4, pool2, pool4 = _brute_split(s[b], m[b], int(kk[b]), int(km[b]), H, W, levels)
+        base = int(sp.cu_img[b])
+        assert sp.counts[b].tolist() == [len(keep), len(w2), len(w4)]
+        rows = sp.row_src[base:int(sp.cu_img[b + 1])].tolist()
+        assert rows == keep + w2 + w4
+        assert {i for i in range(N) if sp.labels[b, i] == O.POOL2} == pool2
+        assert {i for i in range(N) if sp.labels[b, i] == O.POOL4} == pool4
+        # every token reads back the row that holds it
+        for i in range(N):
+            r = int(sp.tok_row[b, i]) - base
+            if i in keep:
+                assert rows[r] == i and r < len(keep)
+            elif i in pool2:
+                assert len(keep) <= r < len(keep) + len(w2)
+                assert rows[r] == (i // W // 2) * (W // 2) + (i % W) // 2
+            else:
+                assert r >= len(keep) + len(w2)
+                assert rows[r] == (i // W // 4) * (W // 4) + (i % W) // 4
+
+
+def test_split_ties_take_lowest_indices():
+    N = 64
+    s = np.ones((1, N), dtype=np.float32)
+    sp = O.split(s, np.zeros((1, N), np.uint8), [10], [0], 8, 8, 1)
+    assert np.nonzero(sp.labels[0] == O.KEEP)[0].tolist() == list(range(10))
+
+
+def test_split_extremes():
+    rng = np.random.default_rng(3)
+    N = 64
+    s = rng.random((1, N)).astype(np.float32)
+    m = (rng.random((1, N)) < 0.2).astype(np.uint8)
+    sp0 = O.split(s, m, [0], [0], 8, 8, 1)
+    assert np.array_equal(sp0.labels[0] == O.KEEP, m[0] == 1)
+    spN = O.split(s, m, [N], [0], 8, 8, 1)
+    assert np.all(spN.labels == O.KEEP) and spN.counts[0].tolist() == [N, 0, 0]
+    assert spN.row_src.tolist() == list(range(N))
+    spall = O.split(s, np.ones_like(m), [0], [0], 8, 8, 2)
+    assert np.all(spall.labels == O.KEEP)
+
+
+def test_split_count_law():
+    wl = I.tiny_layer()
+    b = I.make_batch(wl)
+    s = O.score(b.x)
+    sp = O.split(s, b.mask, b.k_keep, b.k_mid, wl.H, wl.W, 1)
+    top = set(O.ranking(s[0])[: int(b.k_keep[0])].tolist())
+    assert int(sp.counts[0, 0]) == len(top | set(np.nonzero(b.mask[0])[0].tolist()))
+
+
+# ---------------------------------------------------------- pack/unpack ----
+
+def test_pack_constant_windows_lossless():
+    rng = np.random.default_rng(4)
+    H, W, d = 8, 8, 32
+    # each 4x4 block constant (distinct per block and channel)
+    blk = rng.standard_normal((H // 4, W // 4, d)).astype(np.float32)
+    x = np.repeat(np.repeat(blk, 4, axis=0), 4, axis=1)[None]
+    xb = bits(x)
+    s = rng.random((1, H * W)).astype(np.float32)
+    for levels in (1, 2):
+        sp = O.split(s, np.zeros((1, H * W), np.uint8), [10], [20], H, W, levels)
+        packed = O.pack(xb, sp)
+        y = O.unpack(O.bf16_to_f32(packed), sp)
+        assert np.array_equal(y, O.bf16_to_f32(xb).reshape(1, H * W, d))
+
+
+def test_unpack_pack_identity_on_kept_rows_and_brute_mean():
+    wl = I.tiny_layer()
+    b = I.make_batch(wl)
+    s = O.score(b.x)
+    sp = O.split(s, b.mask, b.k_keep, b.k_mid, wl.H, wl.W, 1)
+    packed = O.pack(b.x, sp)
+    xf = O.bf16_to_f32(b.x).reshape(1, wl.N, wl.d)
+    y = O.unpack(O.bf16_to_f32(packed), sp)
+    kept = sp.labels[0] == O.KEEP
+    assert np.array_equal(y[0][kept], xf[0][kept])
+    # pooled rows: the mean of the 2x2 window's pooled members (fp64 mean,
+    # within one bf16 rounding)
+    nk, n2, _ = sp.counts[0]
+    W = wl.W
+    for r in range(nk, nk + n2):
+        w = int(sp.row_src[r])
+        wp, wq = divmod(w, W // 2)
+        mem = [(2 * wp + i) * W + 2 * wq + j for i in range(2) for j in range(2)]
+        mem = [t for t in mem if sp.labels[0, t] == O.POOL2]
+        assert 1 <= len(mem) <= 4
+        ref = xf[0, mem].astype(np.float64).mean(axis=0)
+        got = O.bf16_to_f32(packed[r]).astype(np.float64)
+        assert np.all(np.abs(got - ref) <= np.abs(ref) * 2 ** -8 + 1e-30)
+
+
+# --------------------------------------------------------------- block -----
+
+def test_layer_norm_and_gelu_closed_forms():
+    ln = O.layer_norm(np.array([[1.0, -1.0, 1.0, -1.0], [3.0, 3.0, 3.0, 3.0]]))
+    assert np.allclose(ln[0], np.array([1, -1, 1, -1]) / math.sqrt(1 + 1e-6), rtol=0, atol=1e-15)
+    assert np.all(ln[1] == 0.0)
+    z = np.linspace(-6, 6, 2001)
+    from scipy.special import erf
+    exact = 0.5 * z * (1 + erf(z / math.sqrt(2)))
+    assert np.max(np.abs(O.gelu_tanh(z) - exact)) < 1e-3
+    assert O.gelu_tanh(np.array([0.0]))[0] == 0.0
+
+
+def test_attention_two_token_closed_form():
+    # head_dim 1: logits 0 and ln 2 give weights 1/3 and 2/3
+    q = np.array([[1.0]])
+    k = np.array([[0.0], [math.log(2.0)]])
+    v = np.array([[3.0], [6.0]])
+    assert abs(O.softmax_attention(q, k, v)[0, 0] - 5.0) < 1e-12
+
+
+def _rand_weights(rng, d, mlp):
+    def one():
+        s = I.StreamWeights(w_qkv=bits(rng.normal(0, 0.2, (3 * d, d))), b_qkv=bits(rng.normal(0, 0.2, 3 * d)),
+                            w_o=bits(rng.normal(0, 0.2, (d, d))), b_o=bits(rng.normal(0, 0.2, d)))
+        if mlp:
+            s.w_1 = bits(rng.normal(0, 0.2, (4 * d, d)))
+            s.b_1 = bits(rng.normal(0, 0.2, 4 * d))
+            s.w_2 = bits(rng.normal(0, 0.2, (d, 4 * d)))
+            s.b_2 = bits(rng.normal(0, 0.2, d))
+        return s
+    return I.BlockWeights(txt=one(), img=one())
+
+
+def test_block_uniform_attention_closed_form():
+    # Constant rows -> LayerNorm output 0 -> q, k, v equal their biases for
+    # every token -> uniform attention returns b_v. With no MLP the block is
+    # u + b_v W_o^T + b_o for each stream.
+    rng = np.random.default_rng(2)
+    d, heads, T = 16, 2, 3
+    w = _rand_weights(rng, d, mlp=False)
+    ut = np.ones((T, d)) * 0.5
+    ui = np.ones((5, d)) * -2.0
+    ot, oi = O.block(ut, ui, [0, 5], T, w, heads, mlp=False)
+    f = lambda a: O.bf16_to_f32(a).astype(np.float64)
+    bv_t = f(w.txt.b_qkv)[2 * d:]
+    bv_i = f(w.img.b_qkv)[2 * d:]
+    # every query sees 3 text keys (b_k of text) and 5 image keys (b_k of
+    # image): two distinct logits per head, weighted by their multiplicity
+    hd = d // heads
+    o_ref = {}
+    for name, bq in (("t", f(w.txt.b_qkv)[:d]), ("i", f(w.img.b_qkv)[:d])):
+        o = np.empty(d)
+        for h in range(heads):
+            c = slice(h * hd, (h + 1) * hd)
+            lt = bq[c] @ f(w.txt.b_qkv)[d:2 * d][c] / math.sqrt(hd)
+            li = bq[c] @ f(w.img.b_qkv)[d:2 * d][c] / math.sqrt(hd)
+            wt = 3 * math.exp(lt) / (3 * math.exp(lt) + 5 * math.exp(li))
+            o[c] = wt * bv_t[c] + (1 - wt) * bv_i[c]
+        o_ref[name] = o
+    exp_t = ut + o_ref["t"] @ f(w.txt.w_o).T + f(w.txt.b_o)
+    exp_i = ui + o_ref["i"] @ f(w.img.w_o).T + f(w.img.b_o)
+    assert np.allclose(ot, exp_t, rtol=0, atol=1e-12)
+    assert np.allclose(oi, exp_i, rtol=0, atol=1e-12)
+
+
+def _brute_block(ut, ui, T, w, heads, mlp):
+    """Scalar pure-Python block on one image (tiny shapes only)."""
+    f = lambda a: O.bf16_to_f32(a).astype(np.float64).tolist()
+    d = len(ut[0])
+    hd = d // heads
+
+    def ln(row):
+        mu = sum(row) / d
+        var = sum((x - mu) ** 2 for x in row) / d
+        return [(x - mu) / math.sqrt(var + 1e-6) for x in row]
+
+    def lin(row, W_, b_):
+        return [sum(row[k] * W_[o][k] for k in range(len(row))) + b_[o] for o in range(len(W_))]
+
+    def gelu(z):
+        return 0.5 * z * (1 + math.tanh(math.sqrt(2 / math.pi) * (z + 0.044715 * z ** 3)))
+
+    rows = [(list(r), w.txt) for r in ut] + [(list(r), w.img) for r in ui]
+    qkv = [lin(ln(r), f(sw.w_qkv), f(sw.b_qkv)) for r, sw in rows]
+    out = []
+    for i, (r, sw) in enumerate(rows):
+        o = [0.0] * d
+        for h in range(heads):
+            lg = [sum(qkv[i][h * hd + c] * qkv[j][d + h * hd + c] for c in range(hd)) / math.sqrt(hd)
+                  for j in range(len(rows))]
+            mx = max(lg)
+            e = [math.exp(x - mx) for x in lg]
+            z = sum(e)
+            for c in range(hd):
+                o[h * hd + c] = sum(e[j] / z * qkv[j][2 * d + h * hd + c] for j in range(len(rows)))
+        u = [a + b for a, b in zip(r, lin(o, f(sw.w_o), f(sw.b_o)))]
+        if mlp:
+            hmid = [gelu(z) for z in lin(ln(u), f(sw.w_1), f(sw.b_1))]
+            u = [a + b for a, b in zip(u, lin(hmid, f(sw.w_2), f(sw.b_2)))]
+        out.append(u)
+    return np.array(out[:T]), np.array(out[T:])
+
+
+@pytest.mark.parametrize("grid,mlp", [((4, 4), True), ((8, 8), False)])
+def test_block_brute_force_tiny(grid, mlp):
+    rng = np.random.default_rng(7)
+    H, W = grid
+    d, heads, T = 16, 2, 3
+    w = _rand_weights(rng, d, mlp)
+    ut = bits(rng.standard_normal((T, d)))
+    ui = bits(rng.standard_normal((H * W, d)))
+    ot, oi = O.block(ut, ui, [0, H * W], T, w, heads, mlp)
+    bt, bi = _brute_block(O.bf16_to_f32(ut).astype(np.float64), O.bf16_to_f32(ui).astype(np.float64),
+                          T, w, heads, mlp)
+    assert np.max(np.abs(ot - bt)) < 1e-9 and np.max(np.abs(oi - bi)) < 1e-9
+
+
+def test_block_brute_force_d64_two_images():
+    # d=64, 2 heads of 32, two images of different lengths in one packed batch
+    rng = np.random.default_rng(8)
+    d, heads, T = 64, 2, 2
+    w = _rand_weights(rng, d, mlp=False)
+    ut = bits(rng.standard_normal((2 * T, d)))
+    ui = bits(rng.standard_normal((16 + 9, d)))
+    cu = [0, 16, 25]
+    ot, oi = O.block(ut, ui, cu, T, w, heads, mlp=False)
+    for b in range(2):
+        f = lambda a: O.bf16_to_f32(a).astype(np.float64)
+        bt, bi = _brute_block(f(ut[b * T:(b + 1) * T]), f(ui[cu[b]:cu[b + 1]]), T, w, heads, False)
+        assert np.max(np.abs(ot[b * T:(b + 1) * T] - bt)) < 1e-9
+        assert np.max(np.abs(oi[cu[b]:cu[b + 1]] - bi)) < 1e-9
+
+
+def test_block_rows_matches_block():
+    rng = np.random.default_rng(9)
+    d, heads, T = 32, 4, 5
+    w = _rand_weights(rng, d, mlp=True)
+    ut = bits(rng.standard_normal((2 * T, d)))
+    ui = bits(rng.standard_normal((30, d)))
+    cu = [0, 12, 30]
+    ot, oi = O.block(ut, ui, cu, T, w, heads, True)
+    rt, ri = O.block_rows(ut, ui, cu, T, w, heads, True, 1, [5, 8], [12, 20, 29])
+    assert np.allclose(rt, ot[[5, 8]], rtol=0, atol=1e-12)
+    assert np.allclose(ri, oi[[12, 20, 29]], rtol=0, atol=1e-12)
+
+
+def test_block_permutation_equivariance():
+    rng = np.random.default_rng(10)
+    d, heads, T = 32, 2, 4
+    w = _rand_weights(rng, d, mlp=True)
+    ut = bits(rng.standard_normal((T, d)))
+    ui = bits(rng.standard_normal((20, d)))
+    perm = rng.permutation(20)
+    _, oi = O.block(ut, ui, [0, 20], T, w, heads, True)
+    _, op = O.block(ut, ui[perm], [0, 20], T, w, heads, True)
+    assert np.allclose(op, oi[perm], rtol=0, atol=1e-10)
+
+
+def test_keep_ratio_one_is_dense_block():
+    wl = I.tiny_layer(keep_ratio=1024, H=16, W=16, d=64, heads=2, T=8)
+    b = I.make_batch(wl)
+    w = I.make_weights(wl.d, wl.mlp, seed=1)
+    sp, packed, (ot, oi), y = O.hot_path(b.x, b.text, b.mask, [wl.N], b.k_mid, 1, [w], wl.heads, wl.mlp)
+    assert np.array_equal(packed, b.x.reshape(wl.N, wl.d))
+    dt, di = O.block_dense(b.x, b.text, w, wl.heads, wl.mlp)
+    assert np.array_equal(oi, di) and np.array_equal(ot, dt)
+    assert np.array_equal(y[0], di)
+
+
+def test_update_closed_form():
+    x = bits(np.array([1.0, -2.0, 0.5]))
+    y = np.array([1.0, 0.0, -4.0])
+    got = O.bf16_to_f32(O.update(x, y, 0.035))
+    want = np.array([1.0 - np.float32(0.035), -2.0, 0.5 + 4 * np.float32(0.035)], dtype=np.float32)
+    assert np.array_equal(got, O.bf16_to_f32(I.f32_to_bf16_bits(want)))
