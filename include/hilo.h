@@ -1,0 +1,235 @@
+/*
+ * hilo.h -- C ABI of libhilo, the GB300 (sm_103a) hot path of HiLo-Token
+ * (input-adaptive high/low-frequency token compression around a diffusion
+ * transformer block; paper Sec. 2.3 "HiLo-Token Selection").
+ *
+ * The path, per batch of B images of H x W latent tokens with d channels and
+ * T text tokens each:
+ *
+ *   hilo_score          per-token high-frequency energy
+ *   hilo_split          keep / pool decision, packed offsets
+ *   hilo_pack           packed variable-length image sequence
+ *   hilo_block_forward  MMDiT block (joint attention + MLP) on the packed rows
+ *   hilo_unpack         back to the full token grid
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - All data pointers are DEVICE pointers owned by the caller; the library
+ *   allocates no device memory in any call. Scratch space is the
+ *   caller-provided workspace, sized by the *_workspace_bytes queries.
+ * - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *   Every call is asynchronous on that stream; no call synchronises with the
+ *   host, so a sequence of calls can be captured in a CUDA graph.
+ * - Argument and shape errors are detected on the host before any launch and
+ *   returned synchronously (HILO_ERR_ARG / HILO_ERR_SHAPE); a launch failure
+ *   returns HILO_ERR_CUDA. Device-side failures (a bounded wait that ran out)
+ *   are latched in a device word that hilo_sync_status() reads and clears.
+ *   hilo_last_error() gives a human-readable detail of the last error of the
+ *   calling thread.
+ * - bf16 tensors are passed as void* (IEEE bfloat16, 2 bytes per element).
+ * - Token index i of image b is p*W + q for grid position (p, q) (raster
+ *   order); latents are [B, H, W, d] row-major with d contiguous.
+ * - Packed rows ("row space"): the block works on R = B*T + cap rows of d
+ *   channels. Rows [0, B*T) are the text tokens (image b owns rows
+ *   b*T .. b*T+T-1); rows [B*T, B*T + cu_img[B]) are the packed image rows
+ *   (image b owns B*T + cu_img[b] .. B*T + cu_img[b+1] - 1). cap >= cu_img[B]
+ *   is the capacity the caller allocated (B*H*W always suffices), so no host
+ *   read-back of the data-dependent row counts is ever needed.
+ */
+#ifndef HILO_H
+#define HILO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes. */
+enum {
+  HILO_OK = 0,
+  HILO_ERR_ARG = -1,         /* null pointer or bad scalar argument */
+  HILO_ERR_SHAPE = -2,       /* shape outside the supported set (see hilo_shape) */
+  HILO_ERR_CUDA = -3,        /* a CUDA runtime/driver call failed */
+  HILO_ERR_WORKSPACE = -4,   /* workspace missing or smaller than required */
+  HILO_ERR_TIMEOUT = -5,     /* a device-side bounded wait ran out (see hilo_sync_status) */
+  HILO_ERR_UNSUPPORTED = -6  /* no sm_103a device, or a feature not built */
+};
+
+/* Per-token labels written by hilo_split. */
+enum { HILO_KEEP = 0, HILO_POOL2 = 1, HILO_POOL4 = 2 };
+
+/* Input dtypes of hilo_block_forward. */
+enum { HILO_BF16 = 0, HILO_F32 = 1 };
+
+/*
+ * Problem shape.
+ *   B       images in the batch (>= 1)
+ *   H, W    latent token grid (even; multiples of 4 when levels == 2)
+ *   d       channels (multiple of 128, <= 4096)
+ *   T       text tokens per image (>= 0)
+ *   heads   attention heads; head_dim = d / heads must be 64 or 128
+ *   mlp     1: attention + 4x GELU MLP (a full MMDiT block); 0: attention only
+ *   levels  1: every non-kept token is pooled 2x2; 2: 2x2 and 4x4 pooling
+ * Any other combination returns HILO_ERR_SHAPE.
+ */
+typedef struct {
+  int32_t B, H, W, d, T, heads, mlp, levels;
+} hilo_shape;
+
+/*
+ * Outputs of hilo_split (device pointers, caller-allocated), N = H*W:
+ *   labels   uint8 [B*N]  HILO_KEEP / HILO_POOL2 / HILO_POOL4 per token
+ *   row_src  int32 [B*N]  for packed image row r (0 <= r < cu_img[B]): the
+ *                         token id of a kept row, else the window id of a
+ *                         pooled row (2x2 window id (p/2)*(W/2) + q/2, 4x4
+ *                         window id (p/4)*(W/4) + q/4)
+ *   counts   int32 [B*3]  per image: kept tokens, 2x2 windows, 4x4 windows
+ *   cu_img   int32 [B+1]  packed image-row offsets, cu_img[0] = 0
+ *   tok_row  int32 [B*N]  the packed image row (0-based, without the B*T text
+ *                         offset) each grid token reads its output from
+ * Per image the packed rows are: kept tokens in raster order, then 2x2
+ * windows in window-raster order, then 4x4 windows in window-raster order.
+ */
+typedef struct {
+  uint8_t* labels;
+  int32_t* row_src;
+  int32_t* counts;
+  int32_t* cu_img;
+  int32_t* tok_row;
+} hilo_split_out;
+
+/*
+ * Weights of one stream (text or image) of the MMDiT block: bf16 device
+ * pointers in PyTorch nn.Linear layout, W[out, in] row-major, bias[out].
+ *   w_qkv [3d, d]  output columns: q (d) | k (d) | v (d); head h owns
+ *                  columns h*head_dim .. (h+1)*head_dim - 1 of each part
+ *   w_o   [d, d]
+ *   w_1   [4d, d], w_2 [d, 4d]   (ignored when shape.mlp == 0)
+ */
+typedef struct {
+  const void *w_qkv, *b_qkv, *w_o, *b_o, *w_1, *b_1, *w_2, *b_2;
+} hilo_stream_weights;
+
+typedef struct {
+  hilo_stream_weights txt, img;
+} hilo_block_weights;
+
+/* Readable name of a status code. */
+const char* hilo_status_string(int status);
+
+/* Detail of the last error returned to the calling thread ("" if none). */
+const char* hilo_last_error(void);
+
+/*
+ * Synchronises `stream`, then reads and clears the device error word.
+ * Returns HILO_OK, HILO_ERR_TIMEOUT if a device-side bounded wait ran out
+ * since the last call, or HILO_ERR_CUDA if the stream reported an error.
+ */
+int hilo_sync_status(void* stream);
+
+/* Number of SMs of the current device and whether it is sm_103 (1/0). */
+int hilo_device_info(int* num_sms, int* is_sm103);
+
+/*
+ * hilo_score -- per-token high-frequency energy (paper Sec. 2.3: the
+ * frequency map that decides which tokens keep full resolution; here the
+ * token-space form, the energy of a token minus its 2x2 average-pooled then
+ * nearest-upsampled value).
+ *   x      bf16 [B, H, W, d]
+ *   score  fp32 [B, H*W]   s_i = sum_c (x_ic - m_c)^2, m the mean of the
+ *                          aligned 2x2 window holding token i
+ * Arithmetic is fp32 in one fixed order: m = ((a + b) + (c + e)) * 0.25 over
+ * the window members in raster order; channels are summed in groups of 8
+ * consecutive channels, group g folded into partial g mod 32 (groups and
+ * channels ascending), partials combined by the halving tree j += j + h for
+ * h = 16, 8, 4, 2, 1; no fused multiply-add. The result is therefore
+ * bit-reproducible by any IEEE fp32 implementation of the same order.
+ */
+int hilo_score(const hilo_shape* shape, const void* x, float* score, void* stream);
+
+/* Workspace bytes hilo_split needs (currently 0: NULL is accepted). */
+size_t hilo_split_workspace_bytes(const hilo_shape* shape);
+
+/*
+ * hilo_split -- deterministic keep / pool split (paper Sec. 2.3: tokens
+ * inside the edit mask are always retained, high-frequency tokens are
+ * selected, the low-frequency rest is represented by pooled tokens).
+ *   score   fp32 [B, N]   from hilo_score (finite, >= 0)
+ *   mask    uint8 [B, N]  nonzero = edit-mask token (always kept)
+ *   k_keep  int32 [B]     device; top-k budget per image, 0 <= k <= N
+ *   k_mid   int32 [B]     device; levels == 2 only (else may be NULL):
+ *                         the next k_mid tokens are pooled 2x2, the rest 4x4
+ * Ranking is (score descending, token index ascending), so ties break by
+ * index and the result is unique. kept = top-k_keep ∪ mask.
+ * Values of k outside [0, N] are clamped on the device.
+ */
+int hilo_split(const hilo_shape* shape, const float* score, const uint8_t* mask,
+               const int32_t* k_keep, const int32_t* k_mid, const hilo_split_out* out,
+               void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * hilo_pack -- the packed image sequence (paper Sec. 2.3: selected tokens and
+ * low-frequency tokens concatenated along the token axis).
+ *   x       bf16 [B, H, W, d]
+ *   split   the outputs of hilo_split for the same x
+ *   packed  bf16 [cap, d]; rows [0, cu_img[B]) are written. A kept row is a
+ *           copy of its token; a pooled row is the mean of the window's
+ *           members of that class: fp32 sum in raster member order, one
+ *           correctly rounded division by the member count, bf16 round to
+ *           nearest even.
+ */
+int hilo_pack(const hilo_shape* shape, const void* x, const hilo_split_out* split,
+              void* packed, int32_t cap, void* stream);
+
+/* Workspace bytes hilo_block_forward needs for `cap` image-row capacity. */
+size_t hilo_block_workspace_bytes(const hilo_shape* shape, int32_t cap);
+
+/*
+ * hilo_block_forward -- one MMDiT block on the row space (the DiT the
+ * selected tokens feed, paper Sec. 2.1/2.3): for each stream s in {text,
+ * image} with its own weights
+ *     u += Attn(LN(u) W_qkv^s + b_qkv^s) W_o^s + b_o^s
+ *     u += GELU_tanh(LN(u) W_1^s + b_1^s) W_2^s + b_2^s        (mlp == 1)
+ * where LN has no affine parameters (eps 1e-6, biased variance) and the
+ * attention of image b is non-causal softmax attention over the joint
+ * sequence [its T text rows ; its packed image rows], scale 1/sqrt(head_dim).
+ *   in_txt   [B*T, d] text rows,  dtype in_dtype (HILO_BF16 or HILO_F32)
+ *   in_img   [cap, d] packed image rows, dtype in_dtype
+ *   cu_img   int32 [B+1] device, from hilo_split
+ *   out      fp32 [B*T + cap, d]: the residual stream after the block, text
+ *            rows first (row space). With in_dtype == HILO_F32, in-place use
+ *            (in_txt == out, in_img == out + B*T*d) is allowed.
+ * GEMM operands and attention inputs are bf16 with fp32 accumulation; the
+ * residual stream stays fp32.
+ */
+int hilo_block_forward(const hilo_shape* shape, const hilo_block_weights* weights,
+                       const int32_t* cu_img, int32_t cap, const void* in_txt,
+                       const void* in_img, int in_dtype, float* out, void* ws,
+                       size_t ws_bytes, void* stream);
+
+/*
+ * hilo_unpack -- back to the full grid (nearest broadcast): every token reads
+ * the block output of its kept row or of its window's row.
+ *   out_img  fp32 [cap, d]  image rows of the block output (out + B*T*d)
+ *   y        fp32 [B, H, W, d]   y[b, i] = out_img[tok_row[b, i]]
+ */
+int hilo_unpack(const hilo_shape* shape, const float* out_img, const hilo_split_out* split,
+                float* y, void* stream);
+
+/*
+ * hilo_unpack_update -- unpack fused with the denoising-loop update
+ *   x[b, i] <- bf16(x[b, i] - alpha * out_img[tok_row[b, i]])
+ * computed as an fp32 multiply, then an fp32 subtract (no fused
+ * multiply-add), then bf16 round to nearest even. x is bf16 [B, H, W, d],
+ * updated in place.
+ */
+int hilo_unpack_update(const hilo_shape* shape, const float* out_img,
+                       const hilo_split_out* split, void* x, float alpha, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HILO_H */

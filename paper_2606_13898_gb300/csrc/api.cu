@@ -1,0 +1,353 @@
+// extern "C" entry points of libhilo (declared in include/hilo.h): argument
+// and shape validation on the host, workspace layout, launch orchestration
+// of the kernels, device error reporting.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include "../../include/hilo.h"
+#include "internal.h"
+
+namespace {
+
+thread_local char g_last_error[512] = "";
+
+int fail(int status, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_last_error, sizeof(g_last_error), fmt, ap);
+  va_end(ap);
+  return status;
+}
+
+int cuda_fail(cudaError_t e, const char* where) {
+  return fail(HILO_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+struct DevInfo {
+  int num_sms = 0;
+  int major = 0, minor = 0;
+};
+
+// per-device cache (index = device ordinal)
+DevInfo g_dev[64];
+
+int current_device(DevInfo** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= 64) return fail(HILO_ERR_UNSUPPORTED, "device ordinal %d", dev);
+  DevInfo& d = g_dev[dev];
+  if (d.num_sms == 0) {
+    e = cudaDeviceGetAttribute(&d.major, cudaDevAttrComputeCapabilityMajor, dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&d.minor, cudaDevAttrComputeCapabilityMinor, dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) {
+      d.num_sms = 0;
+      return cuda_fail(e, "cudaDeviceGetAttribute");
+    }
+  }
+  if (d.major != 10 || d.minor != 3)
+    return fail(HILO_ERR_UNSUPPORTED, "libhilo is built for sm_103a; device is sm_%d%d", d.major,
+                d.minor);
+  *out = &d;
+  return HILO_OK;
+}
+
+int check_shape(const hilo_shape* s, bool need_block) {
+  if (!s) return fail(HILO_ERR_ARG, "shape is NULL");
+  if (s->B < 1) return fail(HILO_ERR_SHAPE, "B=%d must be >= 1", s->B);
+  if (s->H < 2 || s->W < 2 || (s->H & 1) || (s->W & 1))
+    return fail(HILO_ERR_SHAPE, "H=%d, W=%d must be even and >= 2", s->H, s->W);
+  if (s->levels != 1 && s->levels != 2) return fail(HILO_ERR_SHAPE, "levels=%d must be 1 or 2", s->levels);
+  if (s->levels == 2 && ((s->H & 3) || (s->W & 3)))
+    return fail(HILO_ERR_SHAPE, "H=%d, W=%d must be multiples of 4 for two-level pooling", s->H, s->W);
+  if (static_cast<long long>(s->H) * s->W > 32768)
+    return fail(HILO_ERR_SHAPE, "H*W=%lld exceeds 32768 tokens per image",
+                static_cast<long long>(s->H) * s->W);
+  if (s->d < 128 || s->d % 128 || s->d > 4096)
+    return fail(HILO_ERR_SHAPE, "d=%d must be a multiple of 128 in [128, 4096]", s->d);
+  if (need_block) {
+    if (s->T < 0) return fail(HILO_ERR_SHAPE, "T=%d must be >= 0", s->T);
+    if (s->heads < 1 || s->d % s->heads) return fail(HILO_ERR_SHAPE, "heads=%d must divide d=%d", s->heads, s->d);
+    const int hd = s->d / s->heads;
+    if (hd != 64 && hd != 128) return fail(HILO_ERR_SHAPE, "head_dim=%d must be 64 or 128", hd);
+    if (s->mlp != 0 && s->mlp != 1) return fail(HILO_ERR_SHAPE, "mlp=%d must be 0 or 1", s->mlp);
+  }
+  return HILO_OK;
+}
+
+int check_split(const hilo_split_out* sp) {
+  if (!sp || !sp->labels || !sp->row_src || !sp->counts || !sp->cu_img || !sp->tok_row)
+    return fail(HILO_ERR_ARG, "split output pointer is NULL");
+  return HILO_OK;
+}
+
+inline size_t align256(size_t v) { return (v + 255) & ~static_cast<size_t>(255); }
+
+struct BlockWs {
+  size_t ln, qkv, attn, hid, total;
+};
+
+BlockWs block_ws_layout(const hilo_shape* s, int32_t cap) {
+  const size_t R = static_cast<size_t>(s->B) * s->T + static_cast<size_t>(cap);
+  const size_t d = static_cast<size_t>(s->d);
+  BlockWs w;
+  w.ln = 0;
+  w.qkv = w.ln + align256(R * d * 2);
+  w.attn = w.qkv + align256(R * 3 * d * 2);
+  w.hid = w.attn + align256(R * d * 2);
+  w.total = w.hid + (s->mlp ? align256(R * 4 * d * 2) : 0);
+  return w;
+}
+
+}  // namespace
+
+namespace hilo {
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                    const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                    const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                    CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+// The driver's tensor-map encoder, resolved through the runtime so that the
+// library does not link libcuda (and loads on hosts without a driver).
+static EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+bool encode_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+                         uint64_t row_stride_elems, uint32_t box_inner, uint32_t box_outer) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {row_stride_elems * 2};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+                  estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+}  // namespace hilo
+
+extern "C" {
+
+const char* hilo_status_string(int status) {
+  switch (status) {
+    case HILO_OK: return "HILO_OK";
+    case HILO_ERR_ARG: return "HILO_ERR_ARG";
+    case HILO_ERR_SHAPE: return "HILO_ERR_SHAPE";
+    case HILO_ERR_CUDA: return "HILO_ERR_CUDA";
+    case HILO_ERR_WORKSPACE: return "HILO_ERR_WORKSPACE";
+    case HILO_ERR_TIMEOUT: return "HILO_ERR_TIMEOUT";
+    case HILO_ERR_UNSUPPORTED: return "HILO_ERR_UNSUPPORTED";
+    default: return "HILO_ERR_UNKNOWN";
+  }
+}
+
+const char* hilo_last_error(void) { return g_last_error; }
+
+int hilo_device_info(int* num_sms, int* is_sm103) {
+  int dev = 0, major = 0, minor = 0, n = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return cuda_fail(e, "hilo_device_info");
+  if (num_sms) *num_sms = n;
+  if (is_sm103) *is_sm103 = (major == 10 && minor == 3) ? 1 : 0;
+  return HILO_OK;
+}
+
+int hilo_sync_status(void* stream) {
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "hilo_sync_status: stream");
+  const int g = hilo::gemm_take_device_error();
+  const int a = hilo::attn_take_device_error();
+  if (g < 0 || a < 0) return fail(HILO_ERR_CUDA, "hilo_sync_status: reading the device error word failed");
+  if (g || a)
+    return fail(HILO_ERR_TIMEOUT, "device-side wait ran out (gemm=%d, attention=%d)", g, a);
+  return HILO_OK;
+}
+
+int hilo_score(const hilo_shape* shape, const void* x, float* score, void* stream) {
+  int st = check_shape(shape, false);
+  if (st) return st;
+  if (!x || !score) return fail(HILO_ERR_ARG, "hilo_score: NULL pointer");
+  DevInfo* dev;
+  if ((st = current_device(&dev))) return st;
+  cudaError_t e = hilo::launch_score(x, score, shape->B, shape->H, shape->W, shape->d, dev->num_sms,
+                                     static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_score");
+}
+
+size_t hilo_split_workspace_bytes(const hilo_shape* shape) {
+  (void)shape;
+  return 0;
+}
+
+int hilo_split(const hilo_shape* shape, const float* score, const uint8_t* mask,
+               const int32_t* k_keep, const int32_t* k_mid, const hilo_split_out* out, void* ws,
+               size_t ws_bytes, void* stream) {
+  (void)ws;
+  (void)ws_bytes;
+  int st = check_shape(shape, false);
+  if (st) return st;
+  if ((st = check_split(out))) return st;
+  if (!score || !mask || !k_keep) return fail(HILO_ERR_ARG, "hilo_split: NULL pointer");
+  if (shape->levels == 2 && !k_mid) return fail(HILO_ERR_ARG, "hilo_split: k_mid is NULL with levels=2");
+  DevInfo* dev;
+  if ((st = current_device(&dev))) return st;
+  cudaError_t e = hilo::launch_split(score, mask, k_keep, shape->levels == 2 ? k_mid : k_keep,
+                                     out->labels, out->row_src, out->counts, out->cu_img,
+                                     out->tok_row, shape->B, shape->H, shape->W, shape->levels,
+                                     static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_split");
+}
+
+int hilo_pack(const hilo_shape* shape, const void* x, const hilo_split_out* split, void* packed,
+              int32_t cap, void* stream) {
+  int st = check_shape(shape, false);
+  if (st) return st;
+  if ((st = check_split(split))) return st;
+  if (!x || !packed) return fail(HILO_ERR_ARG, "hilo_pack: NULL pointer");
+  if (cap < 0) return fail(HILO_ERR_ARG, "hilo_pack: cap=%d", cap);
+  DevInfo* dev;
+  if ((st = current_device(&dev))) return st;
+  cudaError_t e = hilo::launch_pack(x, split->labels, split->row_src, split->counts, split->cu_img,
+                                    packed, shape->B, shape->H, shape->W, shape->d, cap,
+                                    dev->num_sms, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_pack");
+}
+
+size_t hilo_block_workspace_bytes(const hilo_shape* shape, int32_t cap) {
+  if (!shape || cap < 0) return 0;
+  return block_ws_layout(shape, cap).total;
+}
+
+int hilo_block_forward(const hilo_shape* shape, const hilo_block_weights* w, const int32_t* cu_img,
+                       int32_t cap, const void* in_txt, const void* in_img, int in_dtype,
+                       float* out, void* ws, size_t ws_bytes, void* stream) {
+  int st = check_shape(shape, true);
+  if (st) return st;
+  if (!w || !cu_img || !in_img || !out) return fail(HILO_ERR_ARG, "hilo_block_forward: NULL pointer");
+  if (shape->T > 0 && !in_txt) return fail(HILO_ERR_ARG, "hilo_block_forward: in_txt is NULL with T>0");
+  if (in_dtype != HILO_BF16 && in_dtype != HILO_F32)
+    return fail(HILO_ERR_ARG, "hilo_block_forward: in_dtype=%d", in_dtype);
+  if (cap < 0) return fail(HILO_ERR_ARG, "hilo_block_forward: cap=%d", cap);
+  const hilo_stream_weights* sw[2] = {&w->txt, &w->img};
+  for (int i = 0; i < 2; ++i) {
+    if (i == 0 && shape->T == 0) continue;
+    if (!sw[i]->w_qkv || !sw[i]->b_qkv || !sw[i]->w_o || !sw[i]->b_o)
+      return fail(HILO_ERR_ARG, "hilo_block_forward: %s attention weight is NULL", i ? "image" : "text");
+    if (shape->mlp && (!sw[i]->w_1 || !sw[i]->b_1 || !sw[i]->w_2 || !sw[i]->b_2))
+      return fail(HILO_ERR_ARG, "hilo_block_forward: %s MLP weight is NULL", i ? "image" : "text");
+  }
+  const BlockWs L = block_ws_layout(shape, cap);
+  if (!ws || ws_bytes < L.total)
+    return fail(HILO_ERR_WORKSPACE, "hilo_block_forward: workspace %zu < %zu bytes", ws_bytes, L.total);
+  DevInfo* dev;
+  if ((st = current_device(&dev))) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int B = shape->B, T = shape->T, d = shape->d;
+  const int BT = B * T;
+  const int R = BT + cap;
+  char* base = static_cast<char*>(ws);
+  void* ln = base + L.ln;
+  void* qkv = base + L.qkv;
+  void* attn = base + L.attn;
+  void* hid = base + L.hid;
+  const int in_f32 = in_dtype == HILO_F32;
+  const bool in_place = in_f32 && in_txt == out && in_img == out + static_cast<size_t>(BT) * d;
+  const bool in_place_img = in_f32 && BT == 0 && in_img == out;
+
+  cudaError_t e = hilo::launch_layernorm(in_txt, in_img, in_f32, (in_place || in_place_img) ? nullptr : out,
+                                         ln, cu_img, B, BT, cap, d, dev->num_sms, s);
+  if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: layernorm 1");
+
+  auto gemm = [&](const void* A, int N, int K, int epi, void* o,
+                  const void* wt, const void* bt, const void* wi, const void* bi) {
+    hilo::GemmArgs g;
+    g.A = A;
+    g.R = R;
+    g.N = N;
+    g.K = K;
+    g.epilogue = epi;
+    g.out = o;
+    g.g[0] = {0, BT, nullptr, wt, bt, BT};
+    g.g[1] = {BT, 0, cu_img + B, wi, bi, cap};
+    return hilo::launch_gemm(g, dev->num_sms, s);
+  };
+  e = gemm(ln, 3 * d, d, hilo::EPI_BIAS_BF16, qkv, w->txt.w_qkv, w->txt.b_qkv, w->img.w_qkv, w->img.b_qkv);
+  if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: qkv gemm");
+
+  hilo::AttnArgs aa;
+  aa.qkv = qkv;
+  aa.out = attn;
+  aa.cu_img = cu_img;
+  aa.B = B;
+  aa.T = T;
+  aa.heads = shape->heads;
+  aa.head_dim = d / shape->heads;
+  aa.d = d;
+  aa.R = R;
+  aa.max_img_rows = shape->H * shape->W;
+  e = hilo::launch_attention(aa, dev->num_sms, s);
+  if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: attention");
+
+  e = gemm(attn, d, d, hilo::EPI_BIAS_RESID_F32, out, w->txt.w_o, w->txt.b_o, w->img.w_o, w->img.b_o);
+  if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: out-projection gemm");
+  if (shape->mlp) {
+    e = hilo::launch_layernorm(out, out + static_cast<size_t>(BT) * d, 1, nullptr, ln, cu_img, B, BT,
+                               cap, d, dev->num_sms, s);
+    if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: layernorm 2");
+    e = gemm(ln, 4 * d, d, hilo::EPI_BIAS_GELU_BF16, hid, w->txt.w_1, w->txt.b_1, w->img.w_1, w->img.b_1);
+    if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: mlp1 gemm");
+    e = gemm(hid, d, 4 * d, hilo::EPI_BIAS_RESID_F32, out, w->txt.w_2, w->txt.b_2, w->img.w_2, w->img.b_2);
+    if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: mlp2 gemm");
+  }
+  return HILO_OK;
+}
+
+int hilo_unpack(const hilo_shape* shape, const float* out_img, const hilo_split_out* split, float* y,
+                void* stream) {
+  int st = check_shape(shape, false);
+  if (st) return st;
+  if ((st = check_split(split))) return st;
+  if (!out_img || !y) return fail(HILO_ERR_ARG, "hilo_unpack: NULL pointer");
+  DevInfo* dev;
+  if ((st = current_device(&dev))) return st;
+  const long long ntok = static_cast<long long>(shape->B) * shape->H * shape->W;
+  cudaError_t e = hilo::launch_unpack(out_img, split->tok_row, y, ntok, shape->d, dev->num_sms,
+                                      static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_unpack");
+}
+
+int hilo_unpack_update(const hilo_shape* shape, const float* out_img, const hilo_split_out* split,
+                       void* x, float alpha, void* stream) {
+  int st = check_shape(shape, false);
+  if (st) return st;
+  if ((st = check_split(split))) return st;
+  if (!out_img || !x) return fail(HILO_ERR_ARG, "hilo_unpack_update: NULL pointer");
+  DevInfo* dev;
+  if ((st = current_device(&dev))) return st;
+  const long long ntok = static_cast<long long>(shape->B) * shape->H * shape->W;
+  cudaError_t e = hilo::launch_unpack_update(out_img, split->tok_row, x, ntok, shape->d, alpha,
+                                             dev->num_sms, static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_unpack_update");
+}
+
+}  // extern "C"

@@ -1,0 +1,676 @@
+// Bandwidth- and latency-bound kernels of the HiLo-Token hot path:
+//   score  (per-token high-frequency energy, Sec. 2.3 frequency map)
+//   split  (top-k select with index tie-break, mask union, compaction)
+//   pack / unpack / unpack_update (gather + pooling, scatter + broadcast)
+//   layernorm (the block's pre-norm, bf16 operand for the next GEMM)
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace hilo {
+
+// ============================================================== score =====
+//
+// One warp per aligned 2x2 window: the window mean is formed once per channel
+// and the four member energies are accumulated in the fixed order documented
+// in hilo.h (lane j owns channel groups j, j+32, ...; 8 channels per group;
+// halving tree over lanes). Every add/mul is an explicit round-to-nearest
+// intrinsic so the compiler cannot contract to FMA.
+
+__device__ __forceinline__ void bf16x8_to_f32(const uint4& v, float* f) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    f[2 * i] = __uint_as_float(w[i] << 16);
+    f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+  }
+}
+
+__global__ void __launch_bounds__(128) score_kernel(const __nv_bfloat16* __restrict__ x,
+                                                    float* __restrict__ s, int B, int H, int W,
+                                                    int d) {
+  const int lane = threadIdx.x & 31;
+  const int Hw = H >> 1, Ww = W >> 1;
+  const long long nwin = static_cast<long long>(B) * Hw * Ww;
+  const int G = d >> 3;
+  const long long wstep = static_cast<long long>(gridDim.x) * (blockDim.x >> 5);
+  for (long long w = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+       w < nwin; w += wstep) {
+    const int b = static_cast<int>(w / (Hw * Ww));
+    const int r = static_cast<int>(w % (Hw * Ww));
+    const int P = r / Ww, Q = r % Ww;
+    const long long t0 = (static_cast<long long>(b) * H + 2 * P) * W + 2 * Q;
+    const uint4* ra = reinterpret_cast<const uint4*>(x + t0 * d);
+    const uint4* rb = reinterpret_cast<const uint4*>(x + (t0 + 1) * d);
+    const uint4* rc = reinterpret_cast<const uint4*>(x + (t0 + W) * d);
+    const uint4* rd = reinterpret_cast<const uint4*>(x + (t0 + W + 1) * d);
+    float acc0 = 0.f, acc1 = 0.f, acc2 = 0.f, acc3 = 0.f;
+#pragma unroll 4
+    for (int g = lane; g < G; g += 32) {
+      const uint4 va = __ldg(ra + g), vb = __ldg(rb + g), vc = __ldg(rc + g), vd = __ldg(rd + g);
+      float fa[8], fb[8], fc[8], fd[8];
+      bf16x8_to_f32(va, fa);
+      bf16x8_to_f32(vb, fb);
+      bf16x8_to_f32(vc, fc);
+      bf16x8_to_f32(vd, fd);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const float m = __fmul_rn(__fadd_rn(__fadd_rn(fa[u], fb[u]), __fadd_rn(fc[u], fd[u])), 0.25f);
+        const float ea = __fsub_rn(fa[u], m), eb = __fsub_rn(fb[u], m);
+        const float ec = __fsub_rn(fc[u], m), ed = __fsub_rn(fd[u], m);
+        acc0 = __fadd_rn(acc0, __fmul_rn(ea, ea));
+        acc1 = __fadd_rn(acc1, __fmul_rn(eb, eb));
+        acc2 = __fadd_rn(acc2, __fmul_rn(ec, ec));
+        acc3 = __fadd_rn(acc3, __fmul_rn(ed, ed));
+      }
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) {
+      acc0 = __fadd_rn(acc0, __shfl_down_sync(0xffffffffu, acc0, off));
+      acc1 = __fadd_rn(acc1, __shfl_down_sync(0xffffffffu, acc1, off));
+      acc2 = __fadd_rn(acc2, __shfl_down_sync(0xffffffffu, acc2, off));
+      acc3 = __fadd_rn(acc3, __shfl_down_sync(0xffffffffu, acc3, off));
+    }
+    if (lane == 0) {
+      float* sb = s + t0;  // score index equals the token index (b*N + p*W + q)
+      *reinterpret_cast<float2*>(sb) = make_float2(acc0, acc1);
+      *reinterpret_cast<float2*>(sb + W) = make_float2(acc2, acc3);
+    }
+  }
+}
+
+// ============================================================== split =====
+
+constexpr int SPLIT_THREADS = 1024;
+
+// Exclusive scan of one int per thread over a 1024-thread block.
+__device__ __forceinline__ int block_excl_scan(int v, int* warp_tot, int* total) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  int incl = v;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int n = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += n;
+  }
+  if (lane == 31) warp_tot[wid] = incl;
+  __syncthreads();
+  if (wid == 0) {
+    int t = warp_tot[lane];
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int n = __shfl_up_sync(0xffffffffu, t, off);
+      if (lane >= off) t += n;
+    }
+    warp_tot[lane] = t;
+  }
+  __syncthreads();
+  const int res = incl - v + (wid > 0 ? warp_tot[wid - 1] : 0);
+  if (total) *total = warp_tot[31];
+  __syncthreads();
+  return res;
+}
+
+__device__ __forceinline__ int block_sum(int v, int* warp_tot) {
+  int tot;
+  block_excl_scan(v, warp_tot, &tot);
+  return tot;
+}
+
+struct SelectShared {
+  int hist[256];
+  int warp_tot[32];
+  int sel_digit;
+  int sel_k;
+};
+
+// MSB-first radix select over the candidates (cand[i] != 0): the key of the
+// k-th largest candidate (1 <= k <= #candidates) and how many candidates with
+// exactly that key belong to the top k (those with the lowest token ids).
+__device__ void radix_select(const uint32_t* keys, const uint8_t* cand, int N, int k,
+                             SelectShared& sh, uint32_t& thr, int& take) {
+  uint32_t prefix = 0, pmask = 0;
+  int kk = k;
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) sh.hist[i] = 0;
+    __syncthreads();
+    for (int i = threadIdx.x; i < N; i += blockDim.x) {
+      const uint32_t key = keys[i];
+      if (cand[i] && (key & pmask) == prefix) atomicAdd(&sh.hist[(key >> shift) & 255u], 1);
+    }
+    __syncthreads();
+    if (threadIdx.x < 32) {
+      const int lane = threadIdx.x;
+      // lane L covers digits 255-8L .. 248-8L (descending)
+      int cnt[8], lsum = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        cnt[j] = sh.hist[255 - 8 * lane - j];
+        lsum += cnt[j];
+      }
+      int incl = lsum;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int n = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off) incl += n;
+      }
+      const int excl = incl - lsum;
+      const bool here = excl < kk && kk <= incl;
+      if (here) {
+        int c = excl;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if (c + cnt[j] >= kk) {
+            sh.sel_digit = 255 - 8 * lane - j;
+            sh.sel_k = kk - c;
+            break;
+          }
+          c += cnt[j];
+        }
+      }
+    }
+    __syncthreads();
+    prefix |= static_cast<uint32_t>(sh.sel_digit) << shift;
+    pmask |= 255u << shift;
+    kk = sh.sel_k;
+    __syncthreads();
+  }
+  thr = prefix;
+  take = kk;
+}
+
+// Marks sel[i] = 1 for the top-k candidates under (key desc, index asc).
+__device__ void mark_topk(const uint32_t* keys, const uint8_t* cand, uint8_t* sel, int N, int k,
+                          SelectShared& sh) {
+  int ncand = 0;
+  {
+    int c = 0;
+    for (int i = threadIdx.x; i < N; i += blockDim.x) c += cand[i] ? 1 : 0;
+    ncand = block_sum(c, sh.warp_tot);
+  }
+  if (k <= 0) {
+    for (int i = threadIdx.x; i < N; i += blockDim.x) sel[i] = 0;
+    __syncthreads();
+    return;
+  }
+  if (k >= ncand) {
+    for (int i = threadIdx.x; i < N; i += blockDim.x) sel[i] = cand[i] ? 1 : 0;
+    __syncthreads();
+    return;
+  }
+  uint32_t thr;
+  int take;
+  radix_select(keys, cand, N, k, sh, thr, take);
+  // rank of equal-key candidates in index order: contiguous chunk per thread
+  const int chunk = (N + blockDim.x - 1) / blockDim.x;
+  const int i0 = threadIdx.x * chunk;
+  const int i1 = min(N, i0 + chunk);
+  int eq = 0;
+  for (int i = i0; i < i1; ++i) eq += (cand[i] && keys[i] == thr) ? 1 : 0;
+  int rank = block_excl_scan(eq, sh.warp_tot, nullptr);
+  for (int i = i0; i < i1; ++i) {
+    uint8_t v = 0;
+    if (cand[i]) {
+      const uint32_t key = keys[i];
+      if (key > thr) {
+        v = 1;
+      } else if (key == thr) {
+        v = rank < take ? 1 : 0;
+        ++rank;
+      }
+    }
+    sel[i] = v;
+  }
+  __syncthreads();
+}
+
+// Labels and per-image counts. One CTA per image.
+__global__ void __launch_bounds__(SPLIT_THREADS) split_select_kernel(
+    const float* __restrict__ score, const uint8_t* __restrict__ mask,
+    const int32_t* __restrict__ k_keep, const int32_t* __restrict__ k_mid, uint8_t* labels_out,
+    int32_t* counts, int H, int W, int levels) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  __shared__ SelectShared sh;
+  const int N = H * W;
+  const int b = blockIdx.x;
+  uint32_t* keys = reinterpret_cast<uint32_t*>(smem_raw);
+  uint8_t* lab = reinterpret_cast<uint8_t*>(keys + N);
+  uint8_t* cand = lab + N;
+  uint8_t* sel = cand + N;
+  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+    // scores are >= +0, so their IEEE bit patterns order like the values
+    keys[i] = __float_as_uint(score[static_cast<long long>(b) * N + i]);
+    cand[i] = 1;
+  }
+  __syncthreads();
+  const int k = min(max(k_keep[b], 0), N);
+  mark_topk(keys, cand, sel, N, k, sh);
+  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+    const bool keep = sel[i] || mask[static_cast<long long>(b) * N + i];
+    lab[i] = keep ? HILO_LABEL_KEEP : HILO_LABEL_POOL2;
+    cand[i] = keep ? 0 : 1;
+  }
+  __syncthreads();
+  if (levels == 2) {
+    const int km = min(max(k_mid[b], 0), N);
+    mark_topk(keys, cand, sel, N, km, sh);
+    for (int i = threadIdx.x; i < N; i += blockDim.x)
+      if (cand[i]) lab[i] = sel[i] ? HILO_LABEL_POOL2 : HILO_LABEL_POOL4;
+    __syncthreads();
+  }
+  int nk = 0;
+  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+    labels_out[static_cast<long long>(b) * N + i] = lab[i];
+    nk += lab[i] == HILO_LABEL_KEEP ? 1 : 0;
+  }
+  // windows that hold at least one member of their class
+  int n2 = 0, n4 = 0;
+  const int W2 = W >> 1, nw2 = (H >> 1) * W2;
+  for (int w = threadIdx.x; w < nw2; w += blockDim.x) {
+    const int t = (2 * (w / W2)) * W + 2 * (w % W2);
+    n2 += (lab[t] == HILO_LABEL_POOL2 || lab[t + 1] == HILO_LABEL_POOL2 ||
+           lab[t + W] == HILO_LABEL_POOL2 || lab[t + W + 1] == HILO_LABEL_POOL2)
+              ? 1
+              : 0;
+  }
+  if (levels == 2) {
+    const int W4 = W >> 2, nw4 = (H >> 2) * W4;
+    for (int w = threadIdx.x; w < nw4; w += blockDim.x) {
+      const int t = (4 * (w / W4)) * W + 4 * (w % W4);
+      bool any = false;
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) any |= lab[t + i * W + j] == HILO_LABEL_POOL4;
+      n4 += any ? 1 : 0;
+    }
+  }
+  nk = block_sum(nk, sh.warp_tot);
+  n2 = block_sum(n2, sh.warp_tot);
+  n4 = block_sum(n4, sh.warp_tot);
+  if (threadIdx.x == 0) {
+    counts[3 * b + 0] = nk;
+    counts[3 * b + 1] = n2;
+    counts[3 * b + 2] = n4;
+  }
+}
+
+// Packed offsets, row sources and token -> row map. One CTA per image.
+__global__ void __launch_bounds__(SPLIT_THREADS) split_compact_kernel(
+    const uint8_t* __restrict__ labels, const int32_t* __restrict__ counts, int32_t* cu_img,
+    int32_t* row_src, int32_t* tok_row, int H, int W, int levels) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  __shared__ int warp_tot[32];
+  const int N = H * W;
+  const int b = blockIdx.x;
+  uint8_t* lab = smem_raw;
+  for (int i = threadIdx.x; i < N; i += blockDim.x) lab[i] = labels[static_cast<long long>(b) * N + i];
+  int base = 0;
+  for (int j = 0; j < b; ++j) base += counts[3 * j] + counts[3 * j + 1] + counts[3 * j + 2];
+  const int nk = counts[3 * b], n2 = counts[3 * b + 1], n4 = counts[3 * b + 2];
+  if (threadIdx.x == 0) {
+    if (b == 0) cu_img[0] = 0;
+    cu_img[b + 1] = base + nk + n2 + n4;
+  }
+  __syncthreads();
+  int32_t* trow = tok_row + static_cast<long long>(b) * N;
+  // kept tokens in raster order
+  {
+    const int chunk = (N + blockDim.x - 1) / blockDim.x;
+    const int i0 = threadIdx.x * chunk, i1 = min(N, i0 + chunk);
+    int c = 0;
+    for (int i = i0; i < i1; ++i) c += lab[i] == HILO_LABEL_KEEP ? 1 : 0;
+    int r = base + block_excl_scan(c, warp_tot, nullptr);
+    for (int i = i0; i < i1; ++i)
+      if (lab[i] == HILO_LABEL_KEEP) {
+        row_src[r] = i;
+        trow[i] = r;
+        ++r;
+      }
+  }
+  // 2x2 windows in window-raster order
+  {
+    const int W2 = W >> 1, nw = (H >> 1) * W2;
+    const int chunk = (nw + blockDim.x - 1) / blockDim.x;
+    const int w0 = threadIdx.x * chunk, w1 = min(nw, w0 + chunk);
+    int c = 0;
+    for (int w = w0; w < w1; ++w) {
+      const int t = (2 * (w / W2)) * W + 2 * (w % W2);
+      c += (lab[t] == HILO_LABEL_POOL2 || lab[t + 1] == HILO_LABEL_POOL2 ||
+            lab[t + W] == HILO_LABEL_POOL2 || lab[t + W + 1] == HILO_LABEL_POOL2)
+               ? 1
+               : 0;
+    }
+    int r = base + nk + block_excl_scan(c, warp_tot, nullptr);
+    for (int w = w0; w < w1; ++w) {
+      const int t = (2 * (w / W2)) * W + 2 * (w % W2);
+      const int mem[4] = {t, t + 1, t + W, t + W + 1};
+      bool any = false;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) any |= lab[mem[j]] == HILO_LABEL_POOL2;
+      if (!any) continue;
+      row_src[r] = w;
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (lab[mem[j]] == HILO_LABEL_POOL2) trow[mem[j]] = r;
+      ++r;
+    }
+  }
+  if (levels == 2) {
+    const int W4 = W >> 2, nw = (H >> 2) * W4;
+    const int chunk = (nw + blockDim.x - 1) / blockDim.x;
+    const int w0 = threadIdx.x * chunk, w1 = min(nw, w0 + chunk);
+    int c = 0;
+    for (int w = w0; w < w1; ++w) {
+      const int t = (4 * (w / W4)) * W + 4 * (w % W4);
+      bool any = false;
+      for (int i = 0; i < 4; ++i)
+        for (int j = 0; j < 4; ++j) any |= lab[t + i * W + j] == HILO_LABEL_POOL4;
+      c += any ? 1 : 0;
+    }
+    int r = base + nk + n2 + block_excl_scan(c, warp_tot, nullptr);
+    for (int w = w0; w < w1; ++w) {
+      const int t = (4 * (w / W4)) * W + 4 * (w % W4);
+      bool any = false;
+      for (int i = 0; i < 4; ++i)
+        for (int j = 0; j < 4; ++j) any |= lab[t + i * W + j] == HILO_LABEL_POOL4;
+      if (!any) continue;
+      row_src[r] = w;
+      for (int i = 0; i < 4; ++i)
+        for (int j = 0; j < 4; ++j)
+          if (lab[t + i * W + j] == HILO_LABEL_POOL4) trow[t + i * W + j] = r;
+      ++r;
+    }
+  }
+  (void)n4;
+}
+
+// =============================================================== pack =====
+//
+// One warp per packed image row. A kept row is a 16-byte-vector copy; a
+// pooled row sums the window's members of its class in raster order (the
+// first member initialises the sum), divides once with correct rounding and
+// rounds to bf16 (nearest even).
+
+__global__ void __launch_bounds__(256) pack_kernel(const __nv_bfloat16* __restrict__ x,
+                                                   const uint8_t* __restrict__ labels,
+                                                   const int32_t* __restrict__ row_src,
+                                                   const int32_t* __restrict__ counts,
+                                                   const int32_t* __restrict__ cu_img,
+                                                   __nv_bfloat16* __restrict__ packed, int B,
+                                                   int H, int W, int d, int cap) {
+  const int lane = threadIdx.x & 31;
+  const int N = H * W;
+  const int total = min(cu_img[B], cap);
+  const int wstep = gridDim.x * (blockDim.x >> 5);
+  for (int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < total; r += wstep) {
+    int b = 0;
+    while (b + 1 < B && cu_img[b + 1] <= r) ++b;
+    const int local = r - cu_img[b];
+    const int nk = counts[3 * b], n2 = counts[3 * b + 1];
+    const int src = row_src[r];
+    const __nv_bfloat16* xb = x + static_cast<long long>(b) * N * d;
+    uint4* dst = reinterpret_cast<uint4*>(packed + static_cast<long long>(r) * d);
+    if (local < nk) {
+      const uint4* s = reinterpret_cast<const uint4*>(xb + static_cast<long long>(src) * d);
+      for (int c = lane; c < (d >> 3); c += 32) dst[c] = __ldg(s + c);
+      continue;
+    }
+    const int size = local < nk + n2 ? 2 : 4;
+    const uint8_t cls = size == 2 ? HILO_LABEL_POOL2 : HILO_LABEL_POOL4;
+    const int Wn = W / size;
+    const int t0 = (size * (src / Wn)) * W + size * (src % Wn);
+    // member m = i*size + j  <->  token t0 + i*W + j (raster order within the window)
+    bool is_member = false;
+    if (lane < size * size) {
+      const int t = t0 + (lane / size) * W + (lane % size);
+      is_member = labels[static_cast<long long>(b) * N + t] == cls;
+    }
+    const uint32_t mm = __ballot_sync(0xffffffffu, is_member);
+    const float cnt = static_cast<float>(__popc(mm));
+    for (int c = lane; c < (d >> 3); c += 32) {
+      float acc[8];
+      uint32_t rest = mm;
+      bool first = true;
+      while (rest) {
+        const int m = __ffs(rest) - 1;
+        rest &= rest - 1;
+        const int t = t0 + (m / size) * W + (m % size);
+        float f[8];
+        bf16x8_to_f32(__ldg(reinterpret_cast<const uint4*>(xb + static_cast<long long>(t) * d) + c), f);
+        if (first) {
+#pragma unroll
+          for (int u = 0; u < 8; ++u) acc[u] = f[u];
+          first = false;
+        } else {
+#pragma unroll
+          for (int u = 0; u < 8; ++u) acc[u] = __fadd_rn(acc[u], f[u]);
+        }
+      }
+      uint4 o;
+      o.x = pack_bf16x2(__fdiv_rn(acc[0], cnt), __fdiv_rn(acc[1], cnt));
+      o.y = pack_bf16x2(__fdiv_rn(acc[2], cnt), __fdiv_rn(acc[3], cnt));
+      o.z = pack_bf16x2(__fdiv_rn(acc[4], cnt), __fdiv_rn(acc[5], cnt));
+      o.w = pack_bf16x2(__fdiv_rn(acc[6], cnt), __fdiv_rn(acc[7], cnt));
+      dst[c] = o;
+    }
+  }
+}
+
+// ============================================================= unpack =====
+
+__global__ void __launch_bounds__(256) unpack_kernel(const float* __restrict__ out_img,
+                                                     const int32_t* __restrict__ tok_row,
+                                                     float* __restrict__ y, long long ntok,
+                                                     int d) {
+  const int lane = threadIdx.x & 31;
+  const long long wstep = static_cast<long long>(gridDim.x) * (blockDim.x >> 5);
+  for (long long t = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+       t < ntok; t += wstep) {
+    const int r = __ldg(tok_row + t);
+    const float4* s = reinterpret_cast<const float4*>(out_img + static_cast<long long>(r) * d);
+    float4* o = reinterpret_cast<float4*>(y + t * d);
+    for (int c = lane; c < (d >> 2); c += 32) __stcs(o + c, __ldg(s + c));
+  }
+}
+
+__global__ void __launch_bounds__(256) unpack_update_kernel(const float* __restrict__ out_img,
+                                                            const int32_t* __restrict__ tok_row,
+                                                            __nv_bfloat16* __restrict__ x,
+                                                            long long ntok, int d, float alpha) {
+  const int lane = threadIdx.x & 31;
+  const long long wstep = static_cast<long long>(gridDim.x) * (blockDim.x >> 5);
+  for (long long t = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+       t < ntok; t += wstep) {
+    const int r = __ldg(tok_row + t);
+    const float4* s = reinterpret_cast<const float4*>(out_img + static_cast<long long>(r) * d);
+    uint4* xr = reinterpret_cast<uint4*>(x + t * d);
+    for (int c = lane; c < (d >> 3); c += 32) {
+      float f[8];
+      bf16x8_to_f32(xr[c], f);
+      const float4 y0 = __ldg(s + 2 * c), y1 = __ldg(s + 2 * c + 1);
+      const float yv[8] = {y0.x, y0.y, y0.z, y0.w, y1.x, y1.y, y1.z, y1.w};
+      float o[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) o[u] = __fsub_rn(f[u], __fmul_rn(alpha, yv[u]));
+      uint4 v;
+      v.x = pack_bf16x2(o[0], o[1]);
+      v.y = pack_bf16x2(o[2], o[3]);
+      v.z = pack_bf16x2(o[4], o[5]);
+      v.w = pack_bf16x2(o[6], o[7]);
+      xr[c] = v;
+    }
+  }
+}
+
+// ========================================================== layernorm =====
+//
+// One warp per row of the row space. Rows [0, n_txt) come from in_txt, rows
+// [n_txt, n_txt + cu_img[B]) from in_img (bf16 or fp32). Writes the bf16
+// normalised row (no affine, eps 1e-6, biased variance) and, when `resid` is
+// not null, the fp32 copy of the input row (the residual stream).
+
+template <int NCH, bool IN_F32>
+__device__ __forceinline__ void ln_row(const void* src, float* resid_row,
+                                       __nv_bfloat16* ln_row_out, int d, float eps) {
+  const int lane = threadIdx.x & 31;
+  float v[NCH * 4];
+#pragma unroll
+  for (int t = 0; t < NCH; ++t) {
+    const int c = 128 * t + 4 * lane;
+    if (IN_F32) {
+      const float4 f = __ldg(reinterpret_cast<const float4*>(static_cast<const float*>(src) + c));
+      v[4 * t] = f.x; v[4 * t + 1] = f.y; v[4 * t + 2] = f.z; v[4 * t + 3] = f.w;
+    } else {
+      const uint2 u = __ldg(reinterpret_cast<const uint2*>(static_cast<const __nv_bfloat16*>(src) + c));
+      v[4 * t] = __uint_as_float(u.x << 16);
+      v[4 * t + 1] = __uint_as_float(u.x & 0xFFFF0000u);
+      v[4 * t + 2] = __uint_as_float(u.y << 16);
+      v[4 * t + 3] = __uint_as_float(u.y & 0xFFFF0000u);
+    }
+  }
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < NCH * 4; ++i) s += v[i];
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+  const float mean = s / static_cast<float>(d);
+  float q = 0.f;
+#pragma unroll
+  for (int i = 0; i < NCH * 4; ++i) {
+    const float e = v[i] - mean;
+    q += e * e;
+  }
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) q += __shfl_xor_sync(0xffffffffu, q, off);
+  const float rstd = rsqrtf(q / static_cast<float>(d) + eps);
+#pragma unroll
+  for (int t = 0; t < NCH; ++t) {
+    const int c = 128 * t + 4 * lane;
+    if (resid_row)
+      *reinterpret_cast<float4*>(resid_row + c) = make_float4(v[4 * t], v[4 * t + 1], v[4 * t + 2], v[4 * t + 3]);
+    uint2 o;
+    o.x = pack_bf16x2((v[4 * t] - mean) * rstd, (v[4 * t + 1] - mean) * rstd);
+    o.y = pack_bf16x2((v[4 * t + 2] - mean) * rstd, (v[4 * t + 3] - mean) * rstd);
+    *reinterpret_cast<uint2*>(ln_row_out + c) = o;
+  }
+}
+
+template <int NCH>
+__global__ void __launch_bounds__(256) layernorm_kernel(const void* __restrict__ in_txt,
+                                                        const void* __restrict__ in_img,
+                                                        int in_f32, float* resid,
+                                                        __nv_bfloat16* __restrict__ ln,
+                                                        const int32_t* __restrict__ cu_img, int B,
+                                                        int n_txt, int d) {
+  const int rows = n_txt + cu_img[B];
+  const int wstep = gridDim.x * (blockDim.x >> 5);
+  for (int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < rows; r += wstep) {
+    const long long off = static_cast<long long>(r < n_txt ? r : r - n_txt) * d;
+    const void* base = r < n_txt ? in_txt : in_img;
+    float* rr = resid ? resid + static_cast<long long>(r) * d : nullptr;
+    __nv_bfloat16* lo = ln + static_cast<long long>(r) * d;
+    if (in_f32)
+      ln_row<NCH, true>(static_cast<const float*>(base) + off, rr, lo, d, 1e-6f);
+    else
+      ln_row<NCH, false>(static_cast<const __nv_bfloat16*>(base) + off, rr, lo, d, 1e-6f);
+  }
+}
+
+// ============================================================ launchers ===
+
+static int grid_for(long long work_items, int per_block, int num_sms, int blocks_per_sm) {
+  long long g = (work_items + per_block - 1) / per_block;
+  const long long cap = static_cast<long long>(num_sms) * blocks_per_sm;
+  if (g > cap) g = cap;
+  if (g < 1) g = 1;
+  return static_cast<int>(g);
+}
+
+cudaError_t launch_score(const void* x, float* s, int B, int H, int W, int d, int num_sms,
+                         cudaStream_t st) {
+  const long long nwin = static_cast<long long>(B) * (H / 2) * (W / 2);
+  score_kernel<<<grid_for(nwin, 4, num_sms, 16), 128, 0, st>>>(
+      static_cast<const __nv_bfloat16*>(x), s, B, H, W, d);
+  return cudaGetLastError();
+}
+
+size_t split_select_smem(int N) { return static_cast<size_t>(N) * 7; }
+size_t split_compact_smem(int N) { return static_cast<size_t>(N); }
+
+cudaError_t launch_split(const float* score, const uint8_t* mask, const int32_t* k_keep,
+                         const int32_t* k_mid, uint8_t* labels, int32_t* row_src, int32_t* counts,
+                         int32_t* cu_img, int32_t* tok_row, int B, int H, int W, int levels,
+                         cudaStream_t st) {
+  const int N = H * W;
+  const size_t sm1 = split_select_smem(N), sm2 = split_compact_smem(N);
+  cudaError_t e = cudaFuncSetAttribute(split_select_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(sm1));
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(split_compact_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(sm2));
+  if (e != cudaSuccess) return e;
+  split_select_kernel<<<B, SPLIT_THREADS, sm1, st>>>(score, mask, k_keep, k_mid, labels, counts,
+                                                     H, W, levels);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  split_compact_kernel<<<B, SPLIT_THREADS, sm2, st>>>(labels, counts, cu_img, row_src, tok_row, H,
+                                                      W, levels);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pack(const void* x, const uint8_t* labels, const int32_t* row_src,
+                        const int32_t* counts, const int32_t* cu_img, void* packed, int B, int H,
+                        int W, int d, int cap, int num_sms, cudaStream_t st) {
+  pack_kernel<<<grid_for(cap, 8, num_sms, 8), 256, 0, st>>>(
+      static_cast<const __nv_bfloat16*>(x), labels, row_src, counts, cu_img,
+      static_cast<__nv_bfloat16*>(packed), B, H, W, d, cap);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_unpack(const float* out_img, const int32_t* tok_row, float* y, long long ntok,
+                          int d, int num_sms, cudaStream_t st) {
+  unpack_kernel<<<grid_for(ntok, 8, num_sms, 8), 256, 0, st>>>(out_img, tok_row, y, ntok, d);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_unpack_update(const float* out_img, const int32_t* tok_row, void* x,
+                                 long long ntok, int d, float alpha, int num_sms,
+                                 cudaStream_t st) {
+  unpack_update_kernel<<<grid_for(ntok, 8, num_sms, 8), 256, 0, st>>>(
+      out_img, tok_row, static_cast<__nv_bfloat16*>(x), ntok, d, alpha);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_layernorm(const void* in_txt, const void* in_img, int in_f32, float* resid,
+                             void* ln, const int32_t* cu_img, int B, int n_txt, int cap, int d,
+                             int num_sms, cudaStream_t st) {
+  const int grid = grid_for(static_cast<long long>(n_txt) + cap, 8, num_sms, 8);
+  __nv_bfloat16* lo = static_cast<__nv_bfloat16*>(ln);
+#define HILO_LN_CASE(NC)                                                                    \
+  case NC:                                                                                  \
+    layernorm_kernel<NC><<<grid, 256, 0, st>>>(in_txt, in_img, in_f32, resid, lo, cu_img, B, \
+                                               n_txt, d);                                   \
+    break;
+  switch (d / 128) {
+    HILO_LN_CASE(1)
+    HILO_LN_CASE(2)
+    HILO_LN_CASE(3)
+    HILO_LN_CASE(4)
+    HILO_LN_CASE(6)
+    HILO_LN_CASE(8)
+    HILO_LN_CASE(12)
+    HILO_LN_CASE(16)
+    HILO_LN_CASE(24)
+    HILO_LN_CASE(32)
+    default:
+      return cudaErrorInvalidValue;
+  }
+#undef HILO_LN_CASE
+  return cudaGetLastError();
+}
+
+}  // namespace hilo

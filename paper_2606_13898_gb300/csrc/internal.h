@@ -1,0 +1,81 @@
+// Internal launch interface between the C ABI (api.cu) and the kernel files.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#define HILO_LABEL_KEEP 0
+#define HILO_LABEL_POOL2 1
+#define HILO_LABEL_POOL4 2
+
+namespace hilo {
+
+// ---- bandwidth kernels (bw_kernels.cu)
+cudaError_t launch_score(const void* x, float* s, int B, int H, int W, int d, int num_sms,
+                         cudaStream_t st);
+size_t split_select_smem(int N);
+size_t split_compact_smem(int N);
+cudaError_t launch_split(const float* score, const uint8_t* mask, const int32_t* k_keep,
+                         const int32_t* k_mid, uint8_t* labels, int32_t* row_src, int32_t* counts,
+                         int32_t* cu_img, int32_t* tok_row, int B, int H, int W, int levels,
+                         cudaStream_t st);
+cudaError_t launch_pack(const void* x, const uint8_t* labels, const int32_t* row_src,
+                        const int32_t* counts, const int32_t* cu_img, void* packed, int B, int H,
+                        int W, int d, int cap, int num_sms, cudaStream_t st);
+cudaError_t launch_unpack(const float* out_img, const int32_t* tok_row, float* y, long long ntok,
+                          int d, int num_sms, cudaStream_t st);
+cudaError_t launch_unpack_update(const float* out_img, const int32_t* tok_row, void* x,
+                                 long long ntok, int d, float alpha, int num_sms,
+                                 cudaStream_t st);
+cudaError_t launch_layernorm(const void* in_txt, const void* in_img, int in_f32, float* resid,
+                             void* ln, const int32_t* cu_img, int B, int n_txt, int cap, int d,
+                             int num_sms, cudaStream_t st);
+
+// ---- tcgen05 grouped GEMM (gemm_tc.cu)
+enum GemmEpilogue : int {
+  EPI_BIAS_BF16 = 0,       // out_bf16 = acc + bias
+  EPI_BIAS_GELU_BF16 = 1,  // out_bf16 = gelu_tanh(acc + bias)
+  EPI_BIAS_RESID_F32 = 2,  // out_f32 += acc + bias
+};
+
+// Two row groups of the row space share the A operand (one tensor map over
+// all R rows) but use their own weights / bias. Group g covers rows
+// [row_base_g, row_base_g + rows_g); rows_g is rows_static_g, or, when
+// rows_dev_g is not null, read on the device from *rows_dev_g.
+struct GemmGroupArgs {
+  int row_base;
+  int rows_static;
+  const int32_t* rows_dev;
+  const void* weight;  // bf16 [N, K]
+  const void* bias;    // bf16 [N]
+  int rows_cap;        // upper bound of rows (grid sizing)
+};
+
+struct GemmArgs {
+  const void* A;  // bf16 [R, K] row space
+  int R, N, K;
+  GemmGroupArgs g[2];
+  int epilogue;
+  void* out;  // bf16 or f32 [R, N]
+};
+
+cudaError_t launch_gemm(const GemmArgs& a, int num_sms, cudaStream_t st);
+int gemm_take_device_error();
+
+// ---- tcgen05 joint varlen attention (attn_tc.cu)
+struct AttnArgs {
+  const void* qkv;  // bf16 [R, 3d]
+  void* out;        // bf16 [R, d]
+  const int32_t* cu_img;
+  int B, T, heads, head_dim, d, R, max_img_rows;
+};
+cudaError_t launch_attention(const AttnArgs& a, int num_sms, cudaStream_t st);
+int attn_take_device_error();
+
+// ---- tensor maps (api.cu)
+bool encode_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+                         uint64_t row_stride_elems, uint32_t box_inner, uint32_t box_outer);
+
+}  // namespace hilo

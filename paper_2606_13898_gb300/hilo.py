@@ -1,0 +1,308 @@
+"""Thin Python binding of libhilo's C ABI (include/hilo.h).
+
+Functions carry the C names and only marshal arguments: torch tensors are
+passed as device pointers, the shape as a ``hilo_shape`` struct, the stream
+as the current torch stream. Every step of the hot path runs in libhilo's
+CUDA kernels; there is no Python or CPU fallback. If the library has not been
+built, or the device is not an sm_103 GPU, the calls raise.
+
+PyTorch is used for device memory and streams only.
+"""
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import os
+
+import numpy as np
+import torch
+
+from . import build as _build
+
+HILO_OK = 0
+HILO_KEEP, HILO_POOL2, HILO_POOL4 = 0, 1, 2
+HILO_BF16, HILO_F32 = 0, 1
+
+
+class HiloError(RuntimeError):
+    def __init__(self, fn: str, status: int, detail: str):
+        super().__init__(f"{fn} failed: {status} ({detail})")
+        self.status = status
+
+
+class hilo_shape(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in ("B", "H", "W", "d", "T", "heads", "mlp", "levels")]
+
+
+class hilo_split_out(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in ("labels", "row_src", "counts", "cu_img", "tok_row")]
+
+
+class hilo_stream_weights(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in ("w_qkv", "b_qkv", "w_o", "b_o", "w_1", "b_1", "w_2", "b_2")]
+
+
+class hilo_block_weights(ctypes.Structure):
+    _fields_ = [("txt", hilo_stream_weights), ("img", hilo_stream_weights)]
+
+
+EXPORTS = ("hilo_status_string", "hilo_last_error", "hilo_sync_status", "hilo_device_info",
+           "hilo_score", "hilo_split_workspace_bytes", "hilo_split", "hilo_pack",
+           "hilo_block_workspace_bytes", "hilo_block_forward", "hilo_unpack", "hilo_unpack_update")
+
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def lib() -> ctypes.CDLL:
+    """Load libhilo.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = library_path()
+    if not os.path.exists(path):
+        raise RuntimeError(f"libhilo is not built ({path} missing); run paper_2606_13898_gb300.build.build()")
+    L = ctypes.CDLL(path)
+    P, I, S, F = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t, ctypes.c_float
+    shp = ctypes.POINTER(hilo_shape)
+    spo = ctypes.POINTER(hilo_split_out)
+    sig = {
+        "hilo_status_string": (ctypes.c_char_p, [I]),
+        "hilo_last_error": (ctypes.c_char_p, []),
+        "hilo_sync_status": (I, [P]),
+        "hilo_device_info": (I, [ctypes.POINTER(I), ctypes.POINTER(I)]),
+        "hilo_score": (I, [shp, P, P, P]),
+        "hilo_split_workspace_bytes": (S, [shp]),
+        "hilo_split": (I, [shp, P, P, P, P, spo, P, S, P]),
+        "hilo_pack": (I, [shp, P, spo, P, ctypes.c_int32, P]),
+        "hilo_block_workspace_bytes": (S, [shp, ctypes.c_int32]),
+        "hilo_block_forward": (I, [shp, ctypes.POINTER(hilo_block_weights), P, ctypes.c_int32, P, P, I,
+                                   P, P, S, P]),
+        "hilo_unpack": (I, [shp, P, spo, P, P]),
+        "hilo_unpack_update": (I, [shp, P, spo, P, F, P]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(L, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = L
+    return L
+
+
+def _ptr(t) -> int | None:
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(stream) -> int | None:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _check(fn: str, status: int) -> None:
+    if status != HILO_OK:
+        detail = lib().hilo_last_error().decode()
+        raise HiloError(fn, status, detail)
+
+
+@dataclasses.dataclass(frozen=True)
+class Shape:
+    B: int
+    H: int
+    W: int
+    d: int
+    T: int = 0
+    heads: int = 1
+    mlp: int = 1
+    levels: int = 1
+
+    @property
+    def N(self) -> int:
+        return self.H * self.W
+
+    def c(self) -> hilo_shape:
+        return hilo_shape(self.B, self.H, self.W, self.d, self.T, self.heads, int(self.mlp), self.levels)
+
+
+@dataclasses.dataclass
+class SplitBuffers:
+    """Device outputs of hilo_split for one shape (allocated with torch)."""
+
+    labels: torch.Tensor
+    row_src: torch.Tensor
+    counts: torch.Tensor
+    cu_img: torch.Tensor
+    tok_row: torch.Tensor
+
+    @staticmethod
+    def alloc(shape: Shape, device="cuda") -> "SplitBuffers":
+        n = shape.B * shape.N
+        return SplitBuffers(
+            labels=torch.empty(n, dtype=torch.uint8, device=device),
+            row_src=torch.empty(n, dtype=torch.int32, device=device),
+            counts=torch.empty(3 * shape.B, dtype=torch.int32, device=device),
+            cu_img=torch.empty(shape.B + 1, dtype=torch.int32, device=device),
+            tok_row=torch.empty(n, dtype=torch.int32, device=device))
+
+    def c(self) -> hilo_split_out:
+        return hilo_split_out(*(t.data_ptr() for t in (self.labels, self.row_src, self.counts, self.cu_img,
+                                                      self.tok_row)))
+
+
+def bf16_from_bits(a: np.ndarray, device="cuda") -> torch.Tensor:
+    """uint16 bf16 bit patterns (numpy) -> bf16 torch tensor on ``device``."""
+    return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(device)
+
+
+def bits_from_bf16(t: torch.Tensor) -> np.ndarray:
+    return t.detach().contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+@dataclasses.dataclass
+class DeviceWeights:
+    """bf16 device copies of one block's weights (both streams)."""
+
+    tensors: dict
+
+    @staticmethod
+    def from_host(w, device="cuda") -> "DeviceWeights":
+        t = {}
+        for sname in ("txt", "img"):
+            sw = getattr(w, sname)
+            for f in ("w_qkv", "b_qkv", "w_o", "b_o", "w_1", "b_1", "w_2", "b_2"):
+                v = getattr(sw, f)
+                t[(sname, f)] = None if v is None else bf16_from_bits(v, device)
+        return DeviceWeights(t)
+
+    def c(self) -> hilo_block_weights:
+        def sw(s):
+            return hilo_stream_weights(*(_ptr(self.tensors[(s, f)]) for f in
+                                         ("w_qkv", "b_qkv", "w_o", "b_o", "w_1", "b_1", "w_2", "b_2")))
+        return hilo_block_weights(sw("txt"), sw("img"))
+
+
+# ---------------------------------------------------------------------------
+# The C entry points
+# ---------------------------------------------------------------------------
+
+
+def hilo_device_info() -> tuple[int, int]:
+    n, s = ctypes.c_int(), ctypes.c_int()
+    _check("hilo_device_info", lib().hilo_device_info(ctypes.byref(n), ctypes.byref(s)))
+    return n.value, s.value
+
+
+def hilo_sync_status(stream=None) -> None:
+    _check("hilo_sync_status", lib().hilo_sync_status(_stream(stream)))
+
+
+def hilo_score(shape: Shape, x, score, stream=None) -> None:
+    s = shape.c()
+    _check("hilo_score", lib().hilo_score(ctypes.byref(s), _ptr(x), _ptr(score), _stream(stream)))
+
+
+def hilo_split_workspace_bytes(shape: Shape) -> int:
+    s = shape.c()
+    return lib().hilo_split_workspace_bytes(ctypes.byref(s))
+
+
+def hilo_split(shape: Shape, score, mask, k_keep, k_mid, out: SplitBuffers, ws=None, ws_bytes=0,
+               stream=None) -> None:
+    s = shape.c()
+    o = out.c()
+    _check("hilo_split", lib().hilo_split(ctypes.byref(s), _ptr(score), _ptr(mask), _ptr(k_keep), _ptr(k_mid),
+                                          ctypes.byref(o), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def hilo_pack(shape: Shape, x, split: SplitBuffers, packed, cap: int, stream=None) -> None:
+    s = shape.c()
+    o = split.c()
+    _check("hilo_pack", lib().hilo_pack(ctypes.byref(s), _ptr(x), ctypes.byref(o), _ptr(packed), cap,
+                                        _stream(stream)))
+
+
+def hilo_block_workspace_bytes(shape: Shape, cap: int) -> int:
+    s = shape.c()
+    return lib().hilo_block_workspace_bytes(ctypes.byref(s), cap)
+
+
+def hilo_block_forward(shape: Shape, weights: DeviceWeights, cu_img, cap: int, in_txt, in_img, in_dtype: int,
+                       out, ws, ws_bytes: int, stream=None) -> None:
+    s = shape.c()
+    w = weights.c()
+    _check("hilo_block_forward", lib().hilo_block_forward(
+        ctypes.byref(s), ctypes.byref(w), _ptr(cu_img), cap, _ptr(in_txt), _ptr(in_img), in_dtype, _ptr(out),
+        _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def hilo_unpack(shape: Shape, out_img, split: SplitBuffers, y, stream=None) -> None:
+    s = shape.c()
+    o = split.c()
+    _check("hilo_unpack", lib().hilo_unpack(ctypes.byref(s), _ptr(out_img), ctypes.byref(o), _ptr(y),
+                                            _stream(stream)))
+
+
+def hilo_unpack_update(shape: Shape, out_img, split: SplitBuffers, x, alpha: float, stream=None) -> None:
+    s = shape.c()
+    o = split.c()
+    _check("hilo_unpack_update", lib().hilo_unpack_update(ctypes.byref(s), _ptr(out_img), ctypes.byref(o),
+                                                          _ptr(x), ctypes.c_float(alpha), _stream(stream)))
+
+
+# ---------------------------------------------------------------------------
+# One pass of the hot path with every buffer resident on the device
+# ---------------------------------------------------------------------------
+
+
+class HotPath:
+    """Device buffers and the five C calls of one hot-path pass.
+
+    score -> split -> pack -> n_layers x block_forward -> unpack. All buffers
+    are sized to the upper bound cap = B*H*W image rows, so no call needs the
+    data-dependent row counts on the host.
+    """
+
+    def __init__(self, shape: Shape, weights: list, device="cuda"):
+        self.shape = shape
+        self.cap = shape.B * shape.N
+        self.weights = weights
+        B, N, d, T = shape.B, shape.N, shape.d, shape.T
+        self.score = torch.empty(B * N, dtype=torch.float32, device=device)
+        self.split = SplitBuffers.alloc(shape, device)
+        self.packed = torch.empty(self.cap, d, dtype=torch.bfloat16, device=device)
+        self.out = torch.empty(B * T + self.cap, d, dtype=torch.float32, device=device)
+        self.y = torch.empty(B, shape.H, shape.W, d, dtype=torch.float32, device=device)
+        self.ws_bytes = hilo_block_workspace_bytes(shape, self.cap)
+        self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=device)
+
+    @property
+    def out_img(self) -> torch.Tensor:
+        return self.out[self.shape.B * self.shape.T:]
+
+    def run(self, x, text, mask, k_keep, k_mid, stream=None, unpack: bool = True) -> None:
+        sh = self.shape
+        hilo_score(sh, x, self.score, stream)
+        hilo_split(sh, self.score, mask, k_keep, k_mid, self.split, None, 0, stream)
+        hilo_pack(sh, x, self.split, self.packed, self.cap, stream)
+        self.blocks(text, self.packed, HILO_BF16, stream)
+        if unpack:
+            hilo_unpack(sh, self.out_img, self.split, self.y, stream)
+
+    def blocks(self, in_txt, in_img, in_dtype, stream=None) -> None:
+        sh = self.shape
+        for i, w in enumerate(self.weights):
+            if i == 0:
+                hilo_block_forward(sh, w, self.split.cu_img, self.cap, in_txt, in_img, in_dtype, self.out,
+                                   self.ws, self.ws_bytes, stream)
+            else:
+                hilo_block_forward(sh, w, self.split.cu_img, self.cap, self.out, self.out_img, HILO_F32,
+                                   self.out, self.ws, self.ws_bytes, stream)

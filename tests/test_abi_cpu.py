@@ -1,0 +1,99 @@
+"""The C-ABI library builds, loads and exports every symbol of include/hilo.h.
+
+No test here needs a GPU: calls are limited to pure host queries and to
+argument/shape errors that the library rejects before touching the device.
+"""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def H():
+    from paper_2606_13898_gb300 import build
+    from paper_2606_13898_gb300 import hilo
+
+    build.build()
+    hilo.lib()
+    return hilo
+
+
+def declared_functions():
+    names = []
+    for f in os.listdir(os.path.join(ROOT, "include")):
+        if f.endswith(".h"):
+            txt = open(os.path.join(ROOT, "include", f)).read()
+            txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+            names += re.findall(r"\b(hilo_[a-z0-9_]+)\s*\(", txt)
+    return sorted(set(names))
+
+
+def test_exports_every_declared_symbol(H):
+    L = H.lib()
+    names = declared_functions()
+    assert len(names) >= 12
+    for n in names:
+        assert hasattr(L, n), n
+    assert set(H.EXPORTS) <= set(names)
+
+
+def test_status_strings(H):
+    L = H.lib()
+    assert L.hilo_status_string(0) == b"HILO_OK"
+    assert L.hilo_status_string(-5) == b"HILO_ERR_TIMEOUT"
+    assert L.hilo_status_string(123) == b"HILO_ERR_UNKNOWN"
+
+
+@pytest.mark.parametrize("bad,code", [
+    (dict(H=7), -2), (dict(W=0), -2), (dict(d=100), -2), (dict(d=8192), -2), (dict(B=0), -2),
+    (dict(levels=3), -2), (dict(levels=2, H=6), -2), (dict(H=256, W=256), -2),
+])
+def test_shape_rejected_before_launch(H, bad, code):
+    kw = dict(B=1, H=8, W=8, d=128, T=4, heads=1, mlp=0, levels=1)
+    kw.update(bad)
+    s = H.hilo_shape(*(kw[k] for k in ("B", "H", "W", "d", "T", "heads", "mlp", "levels")))
+    L = H.lib()
+    assert L.hilo_score(ctypes.byref(s), 1, 1, None) == code
+    assert L.hilo_last_error() != b""
+
+
+@pytest.mark.parametrize("bad", [dict(heads=3), dict(heads=4, d=128), dict(mlp=2), dict(T=-1)])
+def test_block_shape_rejected(H, bad):
+    kw = dict(B=1, H=8, W=8, d=256, T=4, heads=2, mlp=1, levels=1)
+    kw.update(bad)
+    s = H.hilo_shape(*(kw[k] for k in ("B", "H", "W", "d", "T", "heads", "mlp", "levels")))
+    w = H.hilo_block_weights()
+    rc = H.lib().hilo_block_forward(ctypes.byref(s), ctypes.byref(w), 1, 64, 1, 1, 0, 1, 1, 1 << 30, None)
+    assert rc == -2
+
+
+def test_null_pointers_rejected(H):
+    s = H.hilo_shape(1, 8, 8, 128, 4, 1, 1, 1)
+    L = H.lib()
+    assert L.hilo_score(ctypes.byref(s), None, 1, None) == -1
+    assert L.hilo_score(None, 1, 1, None) == -1
+    sp = H.hilo_split_out()
+    assert L.hilo_split(ctypes.byref(s), 1, 1, 1, 1, ctypes.byref(sp), None, 0, None) == -1
+    w = H.hilo_block_weights()
+    assert L.hilo_block_forward(ctypes.byref(s), ctypes.byref(w), 1, 64, 1, 1, 0, 1, 1, 1 << 30, None) == -1
+
+
+def test_workspace_size_and_check(H):
+    s = H.hilo_shape(2, 64, 64, 3072, 512, 24, 1, 1)
+    cap = 2 * 4096
+    nb = H.lib().hilo_block_workspace_bytes(ctypes.byref(s), cap)
+    R = 2 * 512 + cap
+    assert nb >= R * 3072 * 2 * (1 + 3 + 1 + 4)
+    s0 = H.hilo_shape(2, 64, 64, 3072, 512, 24, 0, 1)
+    assert H.lib().hilo_block_workspace_bytes(ctypes.byref(s0), cap) < nb
+    w = H.hilo_block_weights()
+    for f in ("txt", "img"):
+        sw = getattr(w, f)
+        for n in ("w_qkv", "b_qkv", "w_o", "b_o", "w_1", "b_1", "w_2", "b_2"):
+            setattr(sw, n, 1)
+    rc = H.lib().hilo_block_forward(ctypes.byref(s), ctypes.byref(w), 1, cap, 1, 1, 0, 1, 1, nb - 1, None)
+    assert rc == -4

@@ -1,0 +1,249 @@
+"""GPU-vs-oracle parity of each C entry point on small shapes.
+
+Sizes span several tiles (128-row GEMM / attention tiles, 256-column GEMM
+tiles) and ragged tails, with the oracle finishing in seconds. Integer and
+bf16-coded outputs (scores, labels, offsets, packed rows, unpacked rows) must
+match bit for bit; block outputs within max-abs 2e-2 and rel-L2 1e-2.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import hilo_oracle as O
+from paper_2606_13898_gb300 import inputs as I
+
+from .gpu_helpers import assert_block_close, lib_ready, to_dev_f32, to_dev_i32, to_dev_u8
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def H():
+    return lib_ready()
+
+
+def bits(a):
+    return I.f32_to_bf16_bits(np.asarray(a, dtype=np.float32))
+
+
+# ------------------------------------------------------------------ score --
+
+@pytest.mark.parametrize("B,Hh,W,d", [(1, 32, 32, 512), (2, 6, 10, 128), (1, 2, 2, 3072), (3, 8, 4, 384)])
+def test_score_bitexact(H, B, Hh, W, d):
+    rng = np.random.default_rng(B * 100 + Hh + d)
+    x = bits(rng.standard_normal((B, Hh, W, d)) * rng.uniform(0.1, 10, size=(B, Hh, W, 1)))
+    sh = H.Shape(B=B, H=Hh, W=W, d=d)
+    s = torch.empty(B * Hh * W, dtype=torch.float32, device="cuda")
+    H.hilo_score(sh, H.bf16_from_bits(x), s)
+    torch.cuda.synchronize()
+    ref = O.score(x)
+    got = s.cpu().numpy().reshape(ref.shape)
+    assert np.array_equal(got.view(np.uint32), ref.view(np.uint32))
+
+
+def test_score_closed_forms_on_gpu(H):
+    # checkerboard +-a -> d*a^2 everywhere; constant -> 0
+    d = 256
+    p = np.arange(8)[:, None]
+    q = np.arange(8)[None, :]
+    cb = np.where((p + q) % 2 == 0, 0.75, -0.75)[None, :, :, None] * np.ones(d)
+    x = np.concatenate([cb, np.full((1, 8, 8, d), 3.0)], axis=0)
+    sh = H.Shape(B=2, H=8, W=8, d=d)
+    s = torch.empty(2 * 64, dtype=torch.float32, device="cuda")
+    H.hilo_score(sh, H.bf16_from_bits(bits(x)), s)
+    got = s.cpu().numpy().reshape(2, 64)
+    assert np.all(got[0] == np.float32(d * 0.5625)) and np.all(got[1] == 0.0)
+
+
+# ------------------------------------------------------------------ split --
+
+def run_split(H, s, mask, kk, km, Hh, W, levels):
+    B = s.shape[0]
+    sh = H.Shape(B=B, H=Hh, W=W, d=128, levels=levels)
+    sp = H.SplitBuffers.alloc(sh)
+    H.hilo_split(sh, to_dev_f32(s), to_dev_u8(mask), to_dev_i32(kk), to_dev_i32(km), sp)
+    torch.cuda.synchronize()
+    return sp
+
+
+def check_split(sp, ref, B, N):
+    cu = sp.cu_img.cpu().numpy()
+    assert np.array_equal(cu, ref.cu_img)
+    rows = int(cu[-1])
+    assert np.array_equal(sp.labels.cpu().numpy().reshape(B, N), ref.labels)
+    assert np.array_equal(sp.counts.cpu().numpy().reshape(B, 3), ref.counts)
+    assert np.array_equal(sp.row_src.cpu().numpy()[:rows], ref.row_src)
+    assert np.array_equal(sp.tok_row.cpu().numpy().reshape(B, N), ref.tok_row)
+
+
+@pytest.mark.parametrize("levels", [1, 2])
+@pytest.mark.parametrize("seed", range(4))
+def test_split_bitexact_random_ties(H, seed, levels):
+    rng = np.random.default_rng(seed)
+    Hh, W = [(8, 8), (16, 12), (64, 64), (128, 128)][seed]
+    N = Hh * W
+    B = 3
+    # coarse scores: many exact ties decided by the token index
+    s = (rng.integers(0, 7, size=(B, N)) * 0.25).astype(np.float32)
+    mask = (rng.random((B, N)) < 0.2).astype(np.uint8)
+    kk = rng.integers(0, N + 1, size=B).astype(np.int32)
+    km = rng.integers(0, N + 1, size=B).astype(np.int32)
+    sp = run_split(H, s, mask, kk, km, Hh, W, levels)
+    check_split(sp, O.split(s, mask, kk, km, Hh, W, levels), B, N)
+
+
+@pytest.mark.parametrize("case", ["k0", "kN", "all_mask", "no_mask", "all_equal", "wide_range"])
+def test_split_edge_cases(H, case):
+    rng = np.random.default_rng(7)
+    Hh, W, B = 32, 32, 2
+    N = Hh * W
+    s = rng.random((B, N)).astype(np.float32)
+    mask = (rng.random((B, N)) < 0.15).astype(np.uint8)
+    kk = np.array([N // 4, 3], dtype=np.int32)
+    km = np.array([N // 3, 0], dtype=np.int32)
+    if case == "k0":
+        kk[:] = 0
+    elif case == "kN":
+        kk[:] = N
+    elif case == "all_mask":
+        mask[:] = 1
+    elif case == "no_mask":
+        mask[:] = 0
+    elif case == "all_equal":
+        s[:] = 1.5
+    elif case == "wide_range":
+        s = (rng.random((B, N)) * 1e30).astype(np.float32)
+        s[:, ::7] = 0.0
+        s[:, 3::11] = 1e-40   # subnormal scores order correctly by their bits
+    for levels in (1, 2):
+        sp = run_split(H, s, mask, kk, km, Hh, W, levels)
+        check_split(sp, O.split(s, mask, kk, km, Hh, W, levels), B, N)
+
+
+# ------------------------------------------------------------ pack/unpack --
+
+@pytest.mark.parametrize("levels", [1, 2])
+def test_pack_unpack_bitexact(H, levels):
+    rng = np.random.default_rng(20 + levels)
+    B, Hh, W, d = 3, 16, 24, 256
+    N = Hh * W
+    x = bits(rng.standard_normal((B, Hh, W, d)))
+    s = O.score(x)
+    mask = (rng.random((B, N)) < 0.1).astype(np.uint8)
+    kk = np.array([0, N // 5, N], dtype=np.int32)
+    km = np.array([N // 2, N // 3, 0], dtype=np.int32)
+    ref = O.split(s, mask, kk, km, Hh, W, levels)
+    sh = H.Shape(B=B, H=Hh, W=W, d=d, levels=levels)
+    sp = H.SplitBuffers.alloc(sh)
+    H.hilo_split(sh, to_dev_f32(s), to_dev_u8(mask), to_dev_i32(kk), to_dev_i32(km), sp)
+    cap = B * N
+    packed = torch.full((cap, d), float("nan"), dtype=torch.bfloat16, device="cuda")
+    xd = H.bf16_from_bits(x)
+    H.hilo_pack(sh, xd, sp, packed, cap)
+    torch.cuda.synchronize()
+    rows = int(ref.cu_img[-1])
+    assert np.array_equal(H.bits_from_bf16(packed[:rows]), O.pack(x, ref))
+    # unpack of an arbitrary fp32 block output
+    out = torch.from_numpy(rng.standard_normal((cap, d)).astype(np.float32)).cuda()
+    y = torch.empty(B, Hh, W, d, dtype=torch.float32, device="cuda")
+    H.hilo_unpack(sh, out, sp, y)
+    torch.cuda.synchronize()
+    assert np.array_equal(y.cpu().numpy().reshape(B, N, d), O.unpack(out.cpu().numpy(), ref))
+    # fused update x <- bf16(x - alpha * y)
+    H.hilo_unpack_update(sh, out, sp, xd, 0.035)
+    torch.cuda.synchronize()
+    yref = O.unpack(out.cpu().numpy(), ref).reshape(B, Hh, W, d)
+    assert np.array_equal(H.bits_from_bf16(xd), O.update(x, yref, 0.035))
+
+
+# ------------------------------------------------------------------ block --
+
+def scaled_weights(rng, d, mlp, std):
+    def one():
+        s = I.StreamWeights(w_qkv=bits(rng.normal(0, std, (3 * d, d))), b_qkv=bits(rng.normal(0, std, 3 * d)),
+                            w_o=bits(rng.normal(0, std, (d, d))), b_o=bits(rng.normal(0, std, d)))
+        if mlp:
+            s.w_1 = bits(rng.normal(0, std, (4 * d, d)))
+            s.b_1 = bits(rng.normal(0, std, 4 * d))
+            s.w_2 = bits(rng.normal(0, std / 2, (d, 4 * d)))
+            s.b_2 = bits(rng.normal(0, std, d))
+        return s
+    return I.BlockWeights(txt=one(), img=one())
+
+
+@pytest.mark.parametrize("d,heads,T,lens,mlp", [
+    (128, 1, 64, [200], 0),          # head_dim 128, ragged text and image tiles
+    (128, 2, 64, [256, 77], 1),      # head_dim 64, two images of different length
+    (256, 2, 0, [130, 300, 5], 1),   # no text, three images
+    (512, 8, 200, [384], 1),         # several 256-wide GEMM column tiles
+])
+def test_block_forward_matches_oracle(H, d, heads, T, lens, mlp):
+    rng = np.random.default_rng(d + T + len(lens))
+    B = len(lens)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    rows = int(cu[-1])
+    cap = rows + 37   # capacity above the used rows: the tail must not matter
+    ut = bits(rng.standard_normal((B * T, d)))
+    ui = bits(rng.standard_normal((rows, d)))
+    w = scaled_weights(rng, d, mlp, std=1.0 / np.sqrt(d))
+    grid = int(np.ceil(np.sqrt(cap)))
+    sh = H.Shape(B=B, H=2 * grid, W=2 * grid, d=d, T=T, heads=heads, mlp=mlp)
+    dw = H.DeviceWeights.from_host(w)
+    in_txt = H.bf16_from_bits(ut) if T else torch.empty(0, dtype=torch.bfloat16, device="cuda")
+    in_img = torch.full((cap, d), float("nan"), dtype=torch.bfloat16, device="cuda")
+    in_img[:rows] = H.bf16_from_bits(ui)
+    out = torch.empty(B * T + cap, d, dtype=torch.float32, device="cuda")
+    wsb = H.hilo_block_workspace_bytes(sh, cap)
+    ws = torch.full((wsb,), 0xFF, dtype=torch.uint8, device="cuda")   # NaN-filled scratch
+    H.hilo_block_forward(sh, dw, to_dev_i32(cu), cap, in_txt if T else None, in_img, H.HILO_BF16, out, ws, wsb)
+    H.hilo_sync_status()
+    ot, oi = O.block(ut, ui, cu, T, w, heads, bool(mlp))
+    got = out.cpu().numpy()
+    assert_block_close(got[:B * T], ot, "text rows")
+    assert_block_close(got[B * T:B * T + rows], oi, "image rows")
+
+
+def test_block_forward_fp32_in_place_chain(H):
+    # two blocks chained on the fp32 residual stream, in place
+    rng = np.random.default_rng(99)
+    d, heads, T = 256, 2, 32
+    lens = [150, 64]
+    B = len(lens)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    rows = int(cu[-1])
+    cap = rows
+    ut = bits(rng.standard_normal((B * T, d)))
+    ui = bits(rng.standard_normal((rows, d)))
+    ws_ = [scaled_weights(rng, d, True, 1.0 / np.sqrt(d)) for _ in range(2)]
+    sh = H.Shape(B=B, H=16, W=16, d=d, T=T, heads=heads, mlp=1)
+    out = torch.empty(B * T + cap, d, dtype=torch.float32, device="cuda")
+    wsb = H.hilo_block_workspace_bytes(sh, cap)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    cud = to_dev_i32(cu)
+    H.hilo_block_forward(sh, H.DeviceWeights.from_host(ws_[0]), cud, cap, H.bf16_from_bits(ut),
+                         H.bf16_from_bits(ui), H.HILO_BF16, out, ws, wsb)
+    H.hilo_block_forward(sh, H.DeviceWeights.from_host(ws_[1]), cud, cap, out, out[B * T:], H.HILO_F32, out,
+                         ws, wsb)
+    H.hilo_sync_status()
+    t1, i1 = O.block(ut, ui, cu, T, ws_[0], heads, True)
+    t2, i2 = O.block(t1, i1, cu, T, ws_[1], heads, True)
+    got = out.cpu().numpy()
+    assert_block_close(got[:B * T], t2, "text rows")
+    assert_block_close(got[B * T:], i2, "image rows")
+
+
+def test_host_argument_errors(H):
+    sh = H.Shape(B=1, H=8, W=8, d=128, T=0, heads=1, mlp=0)
+    s = torch.empty(64, dtype=torch.float32, device="cuda")
+    with pytest.raises(H.HiloError) as e:
+        H.hilo_score(H.Shape(B=1, H=7, W=8, d=128), torch.empty(1, device="cuda"), s)
+    assert e.value.status == -2
+    with pytest.raises(H.HiloError) as e:
+        H.hilo_score(sh, None, s)
+    assert e.value.status == -1
+    with pytest.raises(H.HiloError) as e:
+        H.hilo_block_forward(sh, H.DeviceWeights.from_host(scaled_weights(np.random.default_rng(0), 128, False, 0.1)),
+                             torch.zeros(2, dtype=torch.int32, device="cuda"), 64, None,
+                             torch.empty(64, 128, dtype=torch.bfloat16, device="cuda"), H.HILO_BF16,
+                             torch.empty(64, 128, device="cuda"), torch.empty(16, dtype=torch.uint8, device="cuda"), 16)
+    assert e.value.status == -4
