@@ -1,0 +1,483 @@
+#!/usr/bin/env python
+"""Benchmark of the HiLo-Token hot path on GB300.
+
+One step = one pass of the whole hot path -- hilo_score -> hilo_split ->
+hilo_pack -> hilo_block_forward -> hilo_unpack -- over one batch of the
+64x64-token workload (4096 image tokens + 512 text tokens, d=3072, 24 heads of
+128, 4x GELU MLP, keep ratio 1/4, edit mask 10-40% of the grid), inputs
+resident in HBM. The headline value is image-tokens/s over the full grid
+(B*H*W per step / step time), so the compression gain is visible.
+
+Prints one JSON line. Extra keys: the keep-ratio sweep (0.1, 0.25, 0.5, 1.0),
+the uncompressed dense block on the same kernels, per-kernel times, the GEMM
+roofline (dominant kernel), the oracle on the host cores (cpu_baseline), the
+end-to-end number with host buffers (e2e) and the SM clocks seen meanwhile.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl hilo|reference]
+
+Under torchrun (N > 1) every rank runs its own replica of the workload on its
+own GPU (weak scaling, no collective in the data path); rank 0 prints.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "compressed DiT block ms & image-tokens/sec at 4096 tokens; % of bf16/HBM roofline"
+UNIT = "image-tokens/s"
+FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["hilo", "reference"], default="hilo")
+    ap.add_argument("--ratio", default="1/4", help="keep ratio of the timed workload")
+    ap.add_argument("--no-extras", action="store_true", help="skip sweep / dense / e2e / cpu_baseline")
+    return ap.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as fh:
+            p = json.load(fh)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, "fallback"
+
+
+# ------------------------------------------------------------------ clocks --
+
+class ClockSampler:
+    """nvidia-smi SM clock / throttle-reason samples while the timed region runs."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{gpu_index}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": float(max(mx)), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# -------------------------------------------------------------- workloads --
+
+def workload(ratio: str):
+    from paper_2606_13898_gb300 import inputs as I
+    return I.block_64(keep_ratio=ratio)
+
+
+def source_sha(files) -> str:
+    h = hashlib.sha256()
+    for f in files:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def gemm_traffic_per_launch():
+    """DRAM bytes per GEMM launch from the committed ncu summary, if still current."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as fh:
+            t = json.load(fh)
+        g = t["gemm_kernel"]
+        if g["source_sha"] != source_sha(g["sources"]):
+            return None
+        return float(g["bytes_per_launch_mean"])
+    except Exception:
+        return None
+
+
+# ------------------------------------------------------------ oracle arm --
+
+def oracle_sample(ratio: str, crop: int, seed_offset: int = 0):
+    """Inputs of the oracle's bounded sample: a crop x crop window of the workload.
+
+    The crop keeps the workload's channel width, heads, MLP and keep ratio; the
+    text length is scaled with the crop area (at least 8 tokens).
+    """
+    from oracle import hilo_oracle as O
+    from paper_2606_13898_gb300 import inputs as I
+    wl = workload(ratio)
+    b = I.make_batch(wl, seed_offset)
+    # weights widened to fp64 once, outside the timed steps (a model load)
+    w = O.weights_f64(I.make_weights(wl.d, wl.mlp, seed=I.weight_seed(wl)))
+    if crop >= wl.H:
+        return wl, b.x, b.text, b.mask, b.k_keep, b.k_mid, w, wl.T
+    o = (wl.H - crop) // 2
+    x = np.ascontiguousarray(b.x[:, o:o + crop, o:o + crop])
+    m = np.ascontiguousarray(b.mask.reshape(wl.B, wl.H, wl.W)[:, o:o + crop, o:o + crop].reshape(wl.B, -1))
+    T = max(8, wl.T * crop * crop // wl.N)
+    text = np.ascontiguousarray(b.text[:, :T])
+    kk = np.array([I.ceil_ratio(ratio, crop * crop)] * wl.B, dtype=np.int32)
+    return wl, x, text, m, kk, b.k_mid, w, T
+
+
+def oracle_step(sample):
+    from oracle import hilo_oracle as O
+    wl, x, text, m, kk, km, w, T = sample
+    O.hot_path(x, text, m, kk, km, wl.levels, [w], wl.heads, wl.mlp)
+
+
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(ratio: str, min_seconds: float = 10.0):
+    """The oracle, as it stands, on this host's cores: full workload, >= 1 run."""
+    sample = oracle_sample(ratio, crop=64)
+    wl = sample[0]
+    runs, t0 = 0, time.perf_counter()
+    while True:
+        oracle_step(sample)
+        runs += 1
+        el = time.perf_counter() - t0
+        if el >= min_seconds or runs >= 4:
+            break
+    return {"value": wl.B * wl.N * runs / el, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
+            "sample": f"{runs} full hot-path pass(es) of the timed workload (64x64 grid, 512 text, d=3072) "
+                      f"in {el:.1f} s; numpy fp64 block, fp32 score/split/pack"}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    budget = 150.0
+    per_step = budget / max(1, args.steps + args.warmup)
+    # calibrate on an 8x8 crop, then take the largest crop that fits the per-step budget
+    cal = oracle_sample(args.ratio, crop=8)
+    t0 = time.perf_counter()
+    oracle_step(cal)
+    t8 = time.perf_counter() - t0
+    crop = 2
+    for c in (64, 32, 16, 8, 4):
+        if t8 * (c * c) / 64.0 <= per_step:
+            crop = c
+            break
+    sample = oracle_sample(args.ratio, crop=crop)
+    for _ in range(args.warmup):
+        oracle_step(sample)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle_step(sample)
+    el = time.perf_counter() - t0
+    toks = sample[1].shape[0] * crop * crop
+    value = toks * args.steps / el
+    desc = (f"each step: the oracle hot path on a {crop}x{crop} crop ({toks} image tokens, {sample[7]} text "
+            f"tokens, d=3072, keep ratio {args.ratio}) of the 64x64 workload; value = crop tokens / step time")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": workload(args.ratio).name, "B": 1, "H": 64, "W": 64,
+                                            "T": 512, "d": 3072, "heads": 24, "keep_ratio": args.ratio},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
+                             "sample": desc},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------- GPU arm --
+
+def run_hilo(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2606_13898_gb300 import build
+    from paper_2606_13898_gb300 import hilo as H
+    from paper_2606_13898_gb300 import inputs as I
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    build.build()
+    H.lib()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    def max_over_ranks(v: float) -> float:
+        if world == 1:
+            return v
+        t = torch.tensor([v], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    hbm_peak, bf16_peak, peak_src = peaks()
+    stream = torch.cuda.current_stream()
+
+    def setup(ratio: str):
+        wl = workload(ratio)
+        b = I.make_batch(wl, seed_offset=17 * rank)
+        return wl, b
+
+    wl, batch = setup(args.ratio)
+    w = I.make_weights(wl.d, wl.mlp, seed=I.weight_seed(wl))
+    dw = H.DeviceWeights.from_host(w)
+    sh = H.Shape(B=wl.B, H=wl.H, W=wl.W, d=wl.d, T=wl.T, heads=wl.heads, mlp=int(wl.mlp), levels=wl.levels)
+    hp = H.HotPath(sh, [dw])
+
+    def dev_inputs(b):
+        return (H.bf16_from_bits(b.x), H.bf16_from_bits(b.text), torch.from_numpy(b.mask).cuda(),
+                torch.from_numpy(b.k_keep).cuda(), torch.from_numpy(b.k_mid).cuda())
+
+    x, text, mask, kk, km = dev_inputs(batch)
+    for _ in range(max(3, args.warmup)):
+        hp.run(x, text, mask, kk, km)
+    H.hilo_sync_status()
+    cu = hp.split.cu_img.cpu().numpy()
+    L = int(cu[-1])
+    M = wl.B * wl.T + L
+
+    # ---- timed region: K steps, per-kernel events on the launching stream
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(13)] for _ in range(K)]
+    for e in ev[0]:
+        e.record(stream)
+    for row in ev[1:]:
+        for e in row:
+            e.record(stream)
+    torch.cuda.synchronize()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    n0 = H.hilo_launch_count()
+    clocks = ClockSampler(local)
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    start.record(stream)
+    for i in range(K):
+        e = ev[i]
+        H.hilo_set_stage_events(e[3:11])
+        e[0].record(stream)
+        H.hilo_score(sh, x, hp.score)
+        e[1].record(stream)
+        H.hilo_split(sh, hp.score, mask, kk, km, hp.split)
+        e[2].record(stream)
+        H.hilo_pack(sh, x, hp.split, hp.packed, hp.cap)
+        hp.blocks(text, hp.packed, H.HILO_BF16)
+        e[11].record(stream)
+        H.hilo_unpack(sh, hp.out_img, hp.split, hp.y)
+        e[12].record(stream)
+    end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    barrier()
+    H.hilo_set_stage_events([])
+    launches = H.hilo_launch_count() - n0
+    H.hilo_sync_status()
+    ms_total = max_over_ranks(start.elapsed_time(end))
+    ms_step = ms_total / K
+
+    def span(a, b):
+        return sum(ev[i][a].elapsed_time(ev[i][b]) for i in range(K)) / K
+
+    t_score = span(0, 1)
+    t_split = span(1, 2)
+    t_pack = span(2, 3)
+    t_ln1 = span(3, 4)
+    t_qkv = span(4, 5)
+    t_attn = span(5, 6)
+    t_o = span(6, 7)
+    t_ln2 = span(7, 8)
+    t_mlp1 = span(8, 9)
+    t_mlp2 = span(9, 10)
+    t_block = span(3, 11)
+    t_unpack = span(11, 12)
+    d = wl.d
+    gemm_flops = 2.0 * M * d * (3 * d + d + 4 * d + 4 * d)
+    gemm_ms = t_qkv + t_o + t_mlp1 + t_mlp2
+    gemm_tflops = gemm_flops / (gemm_ms * 1e-3) / 1e12
+    # attention: QK^T and PV over each image's joint sequence (T + L_b)
+    S = [wl.T + int(cu[b + 1] - cu[b]) for b in range(wl.B)]
+    attn_flops = sum(4.0 * s * s * d for s in S)
+    attn_tflops = attn_flops / (t_attn * 1e-3) / 1e12
+    N = wl.N * wl.B
+    bytes_score = N * d * 2 + N * 4
+    bytes_pack = N * d * 2 + L * d * 2
+    bytes_unpack = L * d * 4 + N * d * 4
+    bw = lambda by, ms: by / (ms * 1e-3) / 1e9
+    kernels = {
+        "score": {"ms": t_score, "GB/s": bw(bytes_score, t_score), "frac_hbm": bw(bytes_score, t_score) / hbm_peak},
+        "split": {"ms": t_split},
+        "pack": {"ms": t_pack, "GB/s": bw(bytes_pack, t_pack), "frac_hbm": bw(bytes_pack, t_pack) / hbm_peak},
+        "layernorm": {"ms": t_ln1 + t_ln2},
+        "gemm": {"ms": gemm_ms, "TFLOP/s": gemm_tflops, "frac_bf16": gemm_tflops / bf16_peak,
+                 "qkv_ms": t_qkv, "o_ms": t_o, "mlp1_ms": t_mlp1, "mlp2_ms": t_mlp2},
+        "attention": {"ms": t_attn, "TFLOP/s": attn_tflops, "frac_bf16": attn_tflops / bf16_peak},
+        "unpack": {"ms": t_unpack, "GB/s": bw(bytes_unpack, t_unpack),
+                   "frac_hbm": bw(bytes_unpack, t_unpack) / hbm_peak},
+    }
+    block_tflops = (gemm_flops + attn_flops) / (t_block * 1e-3) / 1e12
+    value = N * K * world / (ms_total * 1e-3)
+    traffic = gemm_traffic_per_launch()
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
+        "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": wl.name, "B": wl.B, "H": wl.H, "W": wl.W, "T": wl.T, "d": wl.d,
+                   "heads": wl.heads, "mlp": "4x GELU", "keep_ratio": args.ratio, "mask": "rect 10-40%",
+                   "packed_image_rows": L, "block_rows": M, "parallelism": f"replicas x{world}",
+                   "l2": "no flush: per-step working set 0.53 GB (bf16 weights 453 MB) > 129 MB L2"},
+        "block_ms": t_block, "block_tflops": block_tflops,
+        "roofline": {"bound": "tensor", "kernel": "gemm_kernel (tcgen05)", "achieved": gemm_tflops,
+                     "peak": bf16_peak, "unit": "TFLOP/s", "frac": gemm_tflops / bf16_peak,
+                     "traffic": traffic, "peak_source": f"{peak_src} bf16 dense (burst)",
+                     "algorithmic": f"24*M*d^2 FLOP per step over 4 launches, M={M} rows"},
+        "kernels": kernels,
+        "gpu_launches": int(launches),
+        "clocks": clk,
+    }
+    if not args.no_extras:
+        extras = {}
+        # keep-ratio sweep and the dense uncompressed block on the same kernels
+        Ks = max(5, min(K, 200))
+        sweep = {}
+        for r in ("1/10", "1/4", "1/2", "1"):
+            wl_r, b_r = setup(r)
+            xr, tr, mr, kr, kmr = dev_inputs(b_r)
+            for _ in range(3):
+                hp.run(xr, tr, mr, kr, kmr)
+            torch.cuda.synchronize()
+            s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            s0.record(stream)
+            for _ in range(Ks):
+                hp.run(xr, tr, mr, kr, kmr)
+            s1.record(stream)
+            torch.cuda.synchronize()
+            ms_r = s0.elapsed_time(s1) / Ks
+            Lr = int(hp.split.cu_img[-1].item())
+            sweep[r] = {"hot_path_ms": ms_r, "image_tokens_per_s": N / (ms_r * 1e-3), "packed_image_rows": Lr}
+        extras["sweep"] = sweep
+        # dense block: every grid token is its own row, no score/split/pack/unpack
+        cu_dense = torch.arange(wl.B + 1, dtype=torch.int32, device="cuda") * wl.N
+        x_rows = x.view(wl.B * wl.N, d)
+        for _ in range(3):
+            H.hilo_block_forward(sh, dw, cu_dense, hp.cap, text, x_rows, H.HILO_BF16, hp.out, hp.ws, hp.ws_bytes)
+        torch.cuda.synchronize()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for _ in range(Ks):
+            H.hilo_block_forward(sh, dw, cu_dense, hp.cap, text, x_rows, H.HILO_BF16, hp.out, hp.ws, hp.ws_bytes)
+        s1.record(stream)
+        torch.cuda.synchronize()
+        dense_ms = s0.elapsed_time(s1) / Ks
+        Md = wl.B * (wl.T + wl.N)
+        dense_flops = 24.0 * Md * d * d + wl.B * 4.0 * (wl.T + wl.N) ** 2 * d
+        extras["dense_block"] = {"ms": dense_ms, "image_tokens_per_s": N / (dense_ms * 1e-3),
+                                 "tflops": dense_flops / (dense_ms * 1e-3) / 1e12,
+                                 "speedup_of_compressed_block": dense_ms / t_block,
+                                 "speedup_of_compressed_hot_path": dense_ms / ms_step}
+        # end to end with host buffers: pinned H2D of the step's inputs, D2H of y
+        xh = torch.from_numpy(batch.x.view(np.int16)).view(torch.bfloat16).pin_memory()
+        th = torch.from_numpy(batch.text.view(np.int16)).view(torch.bfloat16).pin_memory()
+        mh = torch.from_numpy(batch.mask).pin_memory()
+        kh = torch.from_numpy(batch.k_keep).pin_memory()
+        kmh = torch.from_numpy(batch.k_mid).pin_memory()
+        yh = torch.empty(hp.y.shape, dtype=torch.float32).pin_memory()
+        xd, td, md, kd, kmd = (torch.empty_like(t, device="cuda") for t in (xh, th, mh, kh, kmh))
+
+        def e2e_step():
+            for dd, hh in ((xd, xh), (td, th), (md, mh), (kd, kh), (kmd, kmh)):
+                dd.copy_(hh, non_blocking=True)
+            hp.run(xd, td, md, kd, kmd)
+            yh.copy_(hp.y, non_blocking=True)
+
+        for _ in range(3):
+            e2e_step()
+        torch.cuda.synchronize()
+        barrier()
+        Ke = max(5, min(K, 200))
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for _ in range(Ke):
+            e2e_step()
+        s1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = max_over_ranks(s0.elapsed_time(s1) / Ke)
+        h2d = sum(t.numel() * t.element_size() for t in (xh, th, mh, kh, kmh))
+        d2h = yh.numel() * yh.element_size()
+        line["e2e"] = {"value": N * world / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+                       "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms, "steps": Ke}
+        line.update(extras)
+        if rank == 0 and world == 1:
+            line["cpu_baseline"] = cpu_baseline(args.ratio)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_hilo(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -101,12 +101,18 @@ typedef struct {
 } hilo_split_out;
 
 /*
- * Weights of one stream (text or image) of the MMDiT block: bf16 device
- * pointers in PyTorch nn.Linear layout, W[out, in] row-major, bias[out].
- *   w_qkv [3d, d]  output columns: q (d) | k (d) | v (d); head h owns
+ * Weights of one stream (text or image) of the MMDiT block: device pointers
+ * in PyTorch nn.Linear layout, W[out, in] row-major, bias[out]. Attention
+ * weights and all biases are bf16; the MLP matrices w_1 and w_2 are IEEE fp16
+ * (convert a bf16 checkpoint once with hilo_convert_bf16_to_f16: exact for
+ * every bf16 value in the fp16 normal range). The MLP runs with fp16
+ * tensor-core operands (11-bit mantissa) because its two activation roundings
+ * (LayerNorm output, GELU output) dominate the block's error budget; the
+ * tensor-core rate is the same as for bf16.
+ *   w_qkv [3d, d]  bf16; output columns: q (d) | k (d) | v (d); head h owns
  *                  columns h*head_dim .. (h+1)*head_dim - 1 of each part
- *   w_o   [d, d]
- *   w_1   [4d, d], w_2 [d, 4d]   (ignored when shape.mlp == 0)
+ *   w_o   [d, d]   bf16
+ *   w_1   [4d, d], w_2 [d, 4d]   fp16 (ignored when shape.mlp == 0)
  */
 typedef struct {
   const void *w_qkv, *b_qkv, *w_o, *b_o, *w_1, *b_1, *w_2, *b_2;
@@ -201,7 +207,8 @@ size_t hilo_block_workspace_bytes(const hilo_shape* shape, int32_t cap);
  *   out      fp32 [B*T + cap, d]: the residual stream after the block, text
  *            rows first (row space). With in_dtype == HILO_F32, in-place use
  *            (in_txt == out, in_img == out + B*T*d) is allowed.
- * GEMM operands and attention inputs are bf16 with fp32 accumulation; the
+ * QKV / out-projection GEMM operands and attention inputs are bf16, the MLP
+ * GEMM operands fp16 (saturating conversion), all with fp32 accumulation; the
  * residual stream stays fp32.
  */
 int hilo_block_forward(const hilo_shape* shape, const hilo_block_weights* weights,
@@ -227,6 +234,30 @@ int hilo_unpack(const hilo_shape* shape, const float* out_img, const hilo_split_
  */
 int hilo_unpack_update(const hilo_shape* shape, const float* out_img,
                        const hilo_split_out* split, void* x, float alpha, void* stream);
+
+/*
+ * hilo_convert_bf16_to_f16 -- dst[i] = fp16(src[i]) for n elements (n a
+ * multiple of 8, both pointers 16-byte aligned, device memory), round to
+ * nearest even, saturating at +-65504. For preparing the fp16 MLP weights
+ * once at load time (no counterpart in the paper).
+ */
+int hilo_convert_bf16_to_f16(const void* src, void* dst, size_t n, void* stream);
+
+/*
+ * Instrumentation (no counterpart in the paper; used by the benchmark).
+ *
+ * hilo_set_stage_events -- register up to 16 CUDA events (cudaEvent_t as
+ * void*) for the calling thread. While registered, hilo_block_forward records
+ * events[k] on its stream at the stage boundaries k = 0..7: before the first
+ * LayerNorm, after it, after the QKV GEMM, after attention, after the
+ * out-projection GEMM, after the second LayerNorm, after the MLP1 GEMM and
+ * after the MLP2 GEMM (k = 5..7 only when mlp == 1). The caller owns the
+ * events; n = 0 unregisters them. Returns HILO_ERR_ARG for n outside [0, 16].
+ *
+ * hilo_launch_count -- number of kernels libhilo has launched in this process.
+ */
+int hilo_set_stage_events(void* const* events, int n);
+unsigned long long hilo_launch_count(void);
 
 #ifdef __cplusplus
 }

@@ -241,7 +241,25 @@ def softmax_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray) -> np.ndarray
 
 
 def _w(bits) -> np.ndarray:
-    return bf16_to_f32(bits).astype(np.float64)
+    """Weights as fp64: bf16 bit patterns are widened, float arrays pass through."""
+    if bits.dtype == np.uint16:
+        return bf16_to_f32(bits).astype(np.float64)
+    return bits
+
+
+def weights_f64(w):
+    """A copy of block weights widened to fp64 once (same values as _w gives
+    per call), for callers that run the block many times."""
+    import copy
+    out = copy.copy(w)
+    for sname in ("txt", "img"):
+        sw = copy.copy(getattr(w, sname))
+        for f in ("w_qkv", "b_qkv", "w_o", "b_o", "w_1", "b_1", "w_2", "b_2"):
+            v = getattr(sw, f, None)
+            if v is not None:
+                setattr(sw, f, _w(v))
+        setattr(out, sname, sw)
+    return out
 
 
 def _as_f64(u) -> np.ndarray:

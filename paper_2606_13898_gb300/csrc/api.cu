@@ -3,6 +3,7 @@
 // of the kernels, device error reporting.
 #include <cuda.h>
 #include <cuda_runtime.h>
+#include <atomic>
 #include <stdarg.h>
 #include <stdio.h>
 #include <string.h>
@@ -13,6 +14,15 @@
 namespace {
 
 thread_local char g_last_error[512] = "";
+thread_local cudaEvent_t g_stage_ev[16];
+thread_local int g_stage_n = 0;
+std::atomic<unsigned long long> g_launches{0};
+
+void stage_mark(int k, cudaStream_t s) {
+  if (k < g_stage_n && g_stage_ev[k]) cudaEventRecord(g_stage_ev[k], s);
+}
+
+void count(int n) { g_launches.fetch_add(static_cast<unsigned long long>(n), std::memory_order_relaxed); }
 
 int fail(int status, const char* fmt, ...) {
   va_list ap;
@@ -191,6 +201,7 @@ int hilo_score(const hilo_shape* shape, const void* x, float* score, void* strea
   if ((st = current_device(&dev))) return st;
   cudaError_t e = hilo::launch_score(x, score, shape->B, shape->H, shape->W, shape->d, dev->num_sms,
                                      static_cast<cudaStream_t>(stream));
+  if (e == cudaSuccess) count(1);
   return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_score");
 }
 
@@ -215,6 +226,7 @@ int hilo_split(const hilo_shape* shape, const float* score, const uint8_t* mask,
                                      out->labels, out->row_src, out->counts, out->cu_img,
                                      out->tok_row, shape->B, shape->H, shape->W, shape->levels,
                                      static_cast<cudaStream_t>(stream));
+  if (e == cudaSuccess) count(2);
   return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_split");
 }
 
@@ -230,6 +242,7 @@ int hilo_pack(const hilo_shape* shape, const void* x, const hilo_split_out* spli
   cudaError_t e = hilo::launch_pack(x, split->labels, split->row_src, split->counts, split->cu_img,
                                     packed, shape->B, shape->H, shape->W, shape->d, cap,
                                     dev->num_sms, static_cast<cudaStream_t>(stream));
+  if (e == cudaSuccess) count(1);
   return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_pack");
 }
 
@@ -274,14 +287,18 @@ int hilo_block_forward(const hilo_shape* shape, const hilo_block_weights* w, con
   const bool in_place = in_f32 && in_txt == out && in_img == out + static_cast<size_t>(BT) * d;
   const bool in_place_img = in_f32 && BT == 0 && in_img == out;
 
+  stage_mark(0, s);
   cudaError_t e = hilo::launch_layernorm(in_txt, in_img, in_f32, (in_place || in_place_img) ? nullptr : out,
-                                         ln, cu_img, B, BT, cap, d, dev->num_sms, s);
+                                         ln, 0, cu_img, B, BT, cap, d, dev->num_sms, s);
   if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: layernorm 1");
+  count(1);
+  stage_mark(1, s);
 
-  auto gemm = [&](const void* A, int N, int K, int epi, void* o,
+  auto gemm = [&](const void* A, int op_f16, int N, int K, int epi, void* o,
                   const void* wt, const void* bt, const void* wi, const void* bi) {
     hilo::GemmArgs g;
     g.A = A;
+    g.op_f16 = op_f16;
     g.R = R;
     g.N = N;
     g.K = K;
@@ -289,10 +306,13 @@ int hilo_block_forward(const hilo_shape* shape, const hilo_block_weights* w, con
     g.out = o;
     g.g[0] = {0, BT, nullptr, wt, bt, BT};
     g.g[1] = {BT, 0, cu_img + B, wi, bi, cap};
-    return hilo::launch_gemm(g, dev->num_sms, s);
+    cudaError_t ge = hilo::launch_gemm(g, dev->num_sms, s);
+    if (ge == cudaSuccess) count(1);
+    return ge;
   };
-  e = gemm(ln, 3 * d, d, hilo::EPI_BIAS_BF16, qkv, w->txt.w_qkv, w->txt.b_qkv, w->img.w_qkv, w->img.b_qkv);
+  e = gemm(ln, 0, 3 * d, d, hilo::EPI_BIAS_BF16, qkv, w->txt.w_qkv, w->txt.b_qkv, w->img.w_qkv, w->img.b_qkv);
   if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: qkv gemm");
+  stage_mark(2, s);
 
   hilo::AttnArgs aa;
   aa.qkv = qkv;
@@ -307,17 +327,24 @@ int hilo_block_forward(const hilo_shape* shape, const hilo_block_weights* w, con
   aa.max_img_rows = shape->H * shape->W;
   e = hilo::launch_attention(aa, dev->num_sms, s);
   if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: attention");
+  count(1);
+  stage_mark(3, s);
 
-  e = gemm(attn, d, d, hilo::EPI_BIAS_RESID_F32, out, w->txt.w_o, w->txt.b_o, w->img.w_o, w->img.b_o);
+  e = gemm(attn, 0, d, d, hilo::EPI_BIAS_RESID_F32, out, w->txt.w_o, w->txt.b_o, w->img.w_o, w->img.b_o);
   if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: out-projection gemm");
+  stage_mark(4, s);
   if (shape->mlp) {
-    e = hilo::launch_layernorm(out, out + static_cast<size_t>(BT) * d, 1, nullptr, ln, cu_img, B, BT,
+    e = hilo::launch_layernorm(out, out + static_cast<size_t>(BT) * d, 1, nullptr, ln, 1, cu_img, B, BT,
                                cap, d, dev->num_sms, s);
     if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: layernorm 2");
-    e = gemm(ln, 4 * d, d, hilo::EPI_BIAS_GELU_BF16, hid, w->txt.w_1, w->txt.b_1, w->img.w_1, w->img.b_1);
+    count(1);
+    stage_mark(5, s);
+    e = gemm(ln, 1, 4 * d, d, hilo::EPI_BIAS_GELU_F16, hid, w->txt.w_1, w->txt.b_1, w->img.w_1, w->img.b_1);
     if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: mlp1 gemm");
-    e = gemm(hid, d, 4 * d, hilo::EPI_BIAS_RESID_F32, out, w->txt.w_2, w->txt.b_2, w->img.w_2, w->img.b_2);
+    stage_mark(6, s);
+    e = gemm(hid, 1, d, 4 * d, hilo::EPI_BIAS_RESID_F32, out, w->txt.w_2, w->txt.b_2, w->img.w_2, w->img.b_2);
     if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: mlp2 gemm");
+    stage_mark(7, s);
   }
   return HILO_OK;
 }
@@ -333,6 +360,7 @@ int hilo_unpack(const hilo_shape* shape, const float* out_img, const hilo_split_
   const long long ntok = static_cast<long long>(shape->B) * shape->H * shape->W;
   cudaError_t e = hilo::launch_unpack(out_img, split->tok_row, y, ntok, shape->d, dev->num_sms,
                                       static_cast<cudaStream_t>(stream));
+  if (e == cudaSuccess) count(1);
   return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_unpack");
 }
 
@@ -347,7 +375,32 @@ int hilo_unpack_update(const hilo_shape* shape, const float* out_img, const hilo
   const long long ntok = static_cast<long long>(shape->B) * shape->H * shape->W;
   cudaError_t e = hilo::launch_unpack_update(out_img, split->tok_row, x, ntok, shape->d, alpha,
                                              dev->num_sms, static_cast<cudaStream_t>(stream));
+  if (e == cudaSuccess) count(1);
   return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_unpack_update");
 }
+
+int hilo_convert_bf16_to_f16(const void* src, void* dst, size_t n, void* stream) {
+  if (!src || !dst) return fail(HILO_ERR_ARG, "hilo_convert_bf16_to_f16: NULL pointer");
+  if (n % 8) return fail(HILO_ERR_ARG, "hilo_convert_bf16_to_f16: n=%zu is not a multiple of 8", n);
+  if ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15)
+    return fail(HILO_ERR_ARG, "hilo_convert_bf16_to_f16: pointers must be 16-byte aligned");
+  DevInfo* dev;
+  int st;
+  if ((st = current_device(&dev))) return st;
+  if (n == 0) return HILO_OK;
+  cudaError_t e = hilo::launch_bf16_to_f16(src, dst, static_cast<long long>(n), dev->num_sms,
+                                           static_cast<cudaStream_t>(stream));
+  if (e == cudaSuccess) count(1);
+  return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_convert_bf16_to_f16");
+}
+
+int hilo_set_stage_events(void* const* events, int n) {
+  if (n < 0 || n > 16 || (n > 0 && !events)) return fail(HILO_ERR_ARG, "hilo_set_stage_events: n=%d", n);
+  for (int i = 0; i < n; ++i) g_stage_ev[i] = static_cast<cudaEvent_t>(events[i]);
+  g_stage_n = n;
+  return HILO_OK;
+}
+
+unsigned long long hilo_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
 }  // extern "C"

@@ -2,7 +2,7 @@
 //   score  (per-token high-frequency energy, Sec. 2.3 frequency map)
 //   split  (top-k select with index tie-break, mask union, compaction)
 //   pack / unpack / unpack_update (gather + pooling, scatter + broadcast)
-//   layernorm (the block's pre-norm, bf16 operand for the next GEMM)
+//   layernorm (the block's pre-norm: bf16 or fp16 operand for the next GEMM)
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -512,9 +512,9 @@ __global__ void __launch_bounds__(256) unpack_update_kernel(const float* __restr
 // normalised row (no affine, eps 1e-6, biased variance) and, when `resid` is
 // not null, the fp32 copy of the input row (the residual stream).
 
-template <int NCH, bool IN_F32>
-__device__ __forceinline__ void ln_row(const void* src, float* resid_row,
-                                       __nv_bfloat16* ln_row_out, int d, float eps) {
+template <int NCH, bool IN_F32, bool OUT_F16>
+__device__ __forceinline__ void ln_row(const void* src, float* resid_row, uint16_t* ln_row_out,
+                                       int d, float eps) {
   const int lane = threadIdx.x & 31;
   float v[NCH * 4];
 #pragma unroll
@@ -552,8 +552,13 @@ __device__ __forceinline__ void ln_row(const void* src, float* resid_row,
     if (resid_row)
       *reinterpret_cast<float4*>(resid_row + c) = make_float4(v[4 * t], v[4 * t + 1], v[4 * t + 2], v[4 * t + 3]);
     uint2 o;
-    o.x = pack_bf16x2((v[4 * t] - mean) * rstd, (v[4 * t + 1] - mean) * rstd);
-    o.y = pack_bf16x2((v[4 * t + 2] - mean) * rstd, (v[4 * t + 3] - mean) * rstd);
+    if (OUT_F16) {
+      o.x = pack_f16x2_sat((v[4 * t] - mean) * rstd, (v[4 * t + 1] - mean) * rstd);
+      o.y = pack_f16x2_sat((v[4 * t + 2] - mean) * rstd, (v[4 * t + 3] - mean) * rstd);
+    } else {
+      o.x = pack_bf16x2((v[4 * t] - mean) * rstd, (v[4 * t + 1] - mean) * rstd);
+      o.y = pack_bf16x2((v[4 * t + 2] - mean) * rstd, (v[4 * t + 3] - mean) * rstd);
+    }
     *reinterpret_cast<uint2*>(ln_row_out + c) = o;
   }
 }
@@ -562,7 +567,7 @@ template <int NCH>
 __global__ void __launch_bounds__(256) layernorm_kernel(const void* __restrict__ in_txt,
                                                         const void* __restrict__ in_img,
                                                         int in_f32, float* resid,
-                                                        __nv_bfloat16* __restrict__ ln,
+                                                        uint16_t* __restrict__ ln, int ln_f16,
                                                         const int32_t* __restrict__ cu_img, int B,
                                                         int n_txt, int d) {
   const int rows = n_txt + cu_img[B];
@@ -571,11 +576,37 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const void* __restrict__
     const long long off = static_cast<long long>(r < n_txt ? r : r - n_txt) * d;
     const void* base = r < n_txt ? in_txt : in_img;
     float* rr = resid ? resid + static_cast<long long>(r) * d : nullptr;
-    __nv_bfloat16* lo = ln + static_cast<long long>(r) * d;
-    if (in_f32)
-      ln_row<NCH, true>(static_cast<const float*>(base) + off, rr, lo, d, 1e-6f);
-    else
-      ln_row<NCH, false>(static_cast<const __nv_bfloat16*>(base) + off, rr, lo, d, 1e-6f);
+    uint16_t* lo = ln + static_cast<long long>(r) * d;
+    if (in_f32) {
+      if (ln_f16)
+        ln_row<NCH, true, true>(static_cast<const float*>(base) + off, rr, lo, d, 1e-6f);
+      else
+        ln_row<NCH, true, false>(static_cast<const float*>(base) + off, rr, lo, d, 1e-6f);
+    } else {
+      if (ln_f16)
+        ln_row<NCH, false, true>(static_cast<const __nv_bfloat16*>(base) + off, rr, lo, d, 1e-6f);
+      else
+        ln_row<NCH, false, false>(static_cast<const __nv_bfloat16*>(base) + off, rr, lo, d, 1e-6f);
+    }
+  }
+}
+
+// ===================================================== bf16 -> fp16 =====
+// Weight conversion at load time (exact for bf16 values in the fp16 normal
+// range; saturating at +-65504).
+
+__global__ void __launch_bounds__(256) bf16_to_f16_kernel(const uint4* __restrict__ src,
+                                                          uint4* __restrict__ dst, long long n8) {
+  for (long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; i < n8;
+       i += static_cast<long long>(gridDim.x) * blockDim.x) {
+    float f[8];
+    bf16x8_to_f32(__ldg(src + i), f);
+    uint4 o;
+    o.x = pack_f16x2_sat(f[0], f[1]);
+    o.y = pack_f16x2_sat(f[2], f[3]);
+    o.z = pack_f16x2_sat(f[4], f[5]);
+    o.w = pack_f16x2_sat(f[6], f[7]);
+    dst[i] = o;
   }
 }
 
@@ -645,15 +676,24 @@ cudaError_t launch_unpack_update(const float* out_img, const int32_t* tok_row, v
   return cudaGetLastError();
 }
 
+cudaError_t launch_bf16_to_f16(const void* src, void* dst, long long n, int num_sms,
+                               cudaStream_t st) {
+  if (n % 8) return cudaErrorInvalidValue;
+  const long long n8 = n / 8;
+  bf16_to_f16_kernel<<<grid_for(n8, 256, num_sms, 8), 256, 0, st>>>(
+      static_cast<const uint4*>(src), static_cast<uint4*>(dst), n8);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_layernorm(const void* in_txt, const void* in_img, int in_f32, float* resid,
-                             void* ln, const int32_t* cu_img, int B, int n_txt, int cap, int d,
-                             int num_sms, cudaStream_t st) {
+                             void* ln, int ln_f16, const int32_t* cu_img, int B, int n_txt,
+                             int cap, int d, int num_sms, cudaStream_t st) {
   const int grid = grid_for(static_cast<long long>(n_txt) + cap, 8, num_sms, 8);
-  __nv_bfloat16* lo = static_cast<__nv_bfloat16*>(ln);
+  uint16_t* lo = static_cast<uint16_t*>(ln);
 #define HILO_LN_CASE(NC)                                                                    \
   case NC:                                                                                  \
-    layernorm_kernel<NC><<<grid, 256, 0, st>>>(in_txt, in_img, in_f32, resid, lo, cu_img, B, \
-                                               n_txt, d);                                   \
+    layernorm_kernel<NC><<<grid, 256, 0, st>>>(in_txt, in_img, in_f32, resid, lo, ln_f16, cu_img, \
+                                               B, n_txt, d);                                \
     break;
   switch (d / 128) {
     HILO_LN_CASE(1)

@@ -195,14 +195,20 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t smem_addr, uint32_t lbo,
   return d;
 }
 
-// Instruction descriptor of kind::f16 with bf16 A/B and fp32 D.
-//   D format f32: bit 4; A bf16: bits 7..9 = 1; B bf16: bits 10..12 = 1;
+// Instruction descriptor of kind::f16 with fp32 D; A and B share one format
+// (fmt 0 = fp16, 1 = bf16).
+//   D format f32: bit 4; A format: bits 7..9; B format: bits 10..12;
 //   A major (0 K, 1 MN): bit 15; B major: bit 16; N >> 3: bits 17..22;
 //   M >> 4: bits 24..28.
+__host__ __device__ constexpr uint32_t idesc_kind_f16(int M, int N, int a_mn_major, int b_mn_major,
+                                                      int fmt) {
+  return (1u << 4) | (static_cast<uint32_t>(fmt) << 7) | (static_cast<uint32_t>(fmt) << 10) |
+         (static_cast<uint32_t>(a_mn_major) << 15) | (static_cast<uint32_t>(b_mn_major) << 16) |
+         (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
+}
+
 __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, int a_mn_major, int b_mn_major) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(a_mn_major) << 15) |
-         (static_cast<uint32_t>(b_mn_major) << 16) | (static_cast<uint32_t>(N >> 3) << 17) |
-         (static_cast<uint32_t>(M >> 4) << 24);
+  return idesc_kind_f16(M, N, a_mn_major, b_mn_major, 1);
 }
 
 __device__ __forceinline__ int warp_id() { return threadIdx.x >> 5; }
@@ -211,6 +217,13 @@ __device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// Two fp32 -> fp16x2, round to nearest even, saturating to +-65504 (no inf).
+__device__ __forceinline__ uint32_t pack_f16x2_sat(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.satfinite.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
 }
 
 }  // namespace hilo

@@ -36,6 +36,7 @@ constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
 
 struct GemmParams {
   int N, K;
+  uint32_t idesc;
   int row_base[2];
   int rows_static[2];
   const int32_t* rows_dev[2];
@@ -176,7 +177,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       // ---------------- MMA issuer
-      const uint32_t idesc = idesc_bf16(BM, BN, 0, 0);
+      const uint32_t idesc = p.idesc;
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
@@ -265,20 +266,30 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         } else {
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] += bv[i];
-          if (p.epilogue == EPI_BIAS_GELU_BF16) {
+          uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(p.out) +
+                                                static_cast<long long>(grow) * p.N + col0);
+          if (p.epilogue == EPI_BIAS_GELU_F16) {
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = gelu_tanh(v[i]);
-          }
-          uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(p.out) +
-                                                static_cast<long long>(grow) * p.N + col0);
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            uint4 o;
-            o.x = pack_bf16x2(v[8 * j], v[8 * j + 1]);
-            o.y = pack_bf16x2(v[8 * j + 2], v[8 * j + 3]);
-            o.z = pack_bf16x2(v[8 * j + 4], v[8 * j + 5]);
-            o.w = pack_bf16x2(v[8 * j + 6], v[8 * j + 7]);
-            dst[j] = o;
+            for (int j = 0; j < 4; ++j) {
+              uint4 o;
+              o.x = pack_f16x2_sat(v[8 * j], v[8 * j + 1]);
+              o.y = pack_f16x2_sat(v[8 * j + 2], v[8 * j + 3]);
+              o.z = pack_f16x2_sat(v[8 * j + 4], v[8 * j + 5]);
+              o.w = pack_f16x2_sat(v[8 * j + 6], v[8 * j + 7]);
+              dst[j] = o;
+            }
+          } else {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              uint4 o;
+              o.x = pack_bf16x2(v[8 * j], v[8 * j + 1]);
+              o.y = pack_bf16x2(v[8 * j + 2], v[8 * j + 3]);
+              o.z = pack_bf16x2(v[8 * j + 4], v[8 * j + 5]);
+              o.w = pack_bf16x2(v[8 * j + 6], v[8 * j + 7]);
+              dst[j] = o;
+            }
           }
         }
       }
@@ -310,6 +321,7 @@ cudaError_t launch_gemm(const GemmArgs& a, int num_sms, cudaStream_t st) {
   GemmParams p;
   p.N = a.N;
   p.K = a.K;
+  p.idesc = idesc_kind_f16(BM, BN, 0, 0, a.op_f16 ? 0 : 1);
   long long upper = 0;
   for (int g = 0; g < 2; ++g) {
     p.row_base[g] = a.g[g].row_base;

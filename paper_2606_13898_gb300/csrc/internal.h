@@ -30,14 +30,16 @@ cudaError_t launch_unpack_update(const float* out_img, const int32_t* tok_row, v
                                  long long ntok, int d, float alpha, int num_sms,
                                  cudaStream_t st);
 cudaError_t launch_layernorm(const void* in_txt, const void* in_img, int in_f32, float* resid,
-                             void* ln, const int32_t* cu_img, int B, int n_txt, int cap, int d,
-                             int num_sms, cudaStream_t st);
+                             void* ln, int ln_f16, const int32_t* cu_img, int B, int n_txt, int cap,
+                             int d, int num_sms, cudaStream_t st);
+cudaError_t launch_bf16_to_f16(const void* src, void* dst, long long n, int num_sms,
+                               cudaStream_t st);
 
 // ---- tcgen05 grouped GEMM (gemm_tc.cu)
 enum GemmEpilogue : int {
-  EPI_BIAS_BF16 = 0,       // out_bf16 = acc + bias
-  EPI_BIAS_GELU_BF16 = 1,  // out_bf16 = gelu_tanh(acc + bias)
-  EPI_BIAS_RESID_F32 = 2,  // out_f32 += acc + bias
+  EPI_BIAS_BF16 = 0,      // out_bf16 = acc + bias
+  EPI_BIAS_GELU_F16 = 1,  // out_f16 = gelu_tanh(acc + bias)   (saturating)
+  EPI_BIAS_RESID_F32 = 2, // out_f32 += acc + bias
 };
 
 // Two row groups of the row space share the A operand (one tensor map over
@@ -54,8 +56,9 @@ struct GemmGroupArgs {
 };
 
 struct GemmArgs {
-  const void* A;  // bf16 [R, K] row space
+  const void* A;  // [R, K] row space, bf16 (op_f16 = 0) or fp16 (op_f16 = 1); W_g the same type
   int R, N, K;
+  int op_f16;
   GemmGroupArgs g[2];
   int epilogue;
   void* out;  // bf16 or f32 [R, N]

@@ -48,7 +48,8 @@ class hilo_block_weights(ctypes.Structure):
 
 EXPORTS = ("hilo_status_string", "hilo_last_error", "hilo_sync_status", "hilo_device_info",
            "hilo_score", "hilo_split_workspace_bytes", "hilo_split", "hilo_pack",
-           "hilo_block_workspace_bytes", "hilo_block_forward", "hilo_unpack", "hilo_unpack_update")
+           "hilo_block_workspace_bytes", "hilo_block_forward", "hilo_unpack", "hilo_unpack_update",
+           "hilo_convert_bf16_to_f16", "hilo_set_stage_events", "hilo_launch_count")
 
 _lib = None
 
@@ -83,6 +84,9 @@ def lib() -> ctypes.CDLL:
                                    P, P, S, P]),
         "hilo_unpack": (I, [shp, P, spo, P, P]),
         "hilo_unpack_update": (I, [shp, P, spo, P, F, P]),
+        "hilo_convert_bf16_to_f16": (I, [P, P, S, P]),
+        "hilo_set_stage_events": (I, [ctypes.POINTER(ctypes.c_void_p), I]),
+        "hilo_launch_count": (ctypes.c_ulonglong, []),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -169,7 +173,9 @@ def bits_from_bf16(t: torch.Tensor) -> np.ndarray:
 
 @dataclasses.dataclass
 class DeviceWeights:
-    """bf16 device copies of one block's weights (both streams)."""
+    """Device copies of one block's weights (both streams): bf16, except the
+    MLP matrices w_1 / w_2, which are converted once to fp16 on the device
+    (hilo_convert_bf16_to_f16)."""
 
     tensors: dict
 
@@ -180,7 +186,16 @@ class DeviceWeights:
             sw = getattr(w, sname)
             for f in ("w_qkv", "b_qkv", "w_o", "b_o", "w_1", "b_1", "w_2", "b_2"):
                 v = getattr(sw, f)
-                t[(sname, f)] = None if v is None else bf16_from_bits(v, device)
+                if v is None:
+                    t[(sname, f)] = None
+                elif f in ("w_1", "w_2"):
+                    src = bf16_from_bits(v, device)
+                    dst = torch.empty(src.shape, dtype=torch.float16, device=device)
+                    hilo_convert_bf16_to_f16(src, dst, src.numel())
+                    t[(sname, f)] = dst
+                else:
+                    t[(sname, f)] = bf16_from_bits(v, device)
+        torch.cuda.synchronize()
         return DeviceWeights(t)
 
     def c(self) -> hilo_block_weights:
@@ -256,6 +271,21 @@ def hilo_unpack_update(shape: Shape, out_img, split: SplitBuffers, x, alpha: flo
     o = split.c()
     _check("hilo_unpack_update", lib().hilo_unpack_update(ctypes.byref(s), _ptr(out_img), ctypes.byref(o),
                                                           _ptr(x), ctypes.c_float(alpha), _stream(stream)))
+
+
+def hilo_convert_bf16_to_f16(src, dst, n: int, stream=None) -> None:
+    _check("hilo_convert_bf16_to_f16", lib().hilo_convert_bf16_to_f16(_ptr(src), _ptr(dst), n, _stream(stream)))
+
+
+def hilo_set_stage_events(events) -> None:
+    """Register torch.cuda.Event objects (already recorded once) as block stage markers."""
+    n = len(events)
+    arr = (ctypes.c_void_p * max(n, 1))(*[e.cuda_event for e in events])
+    _check("hilo_set_stage_events", lib().hilo_set_stage_events(arr, n))
+
+
+def hilo_launch_count() -> int:
+    return int(lib().hilo_launch_count())
 
 
 # ---------------------------------------------------------------------------

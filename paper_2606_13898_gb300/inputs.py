@@ -19,7 +19,9 @@ below stand in for them:
 * all linear weights and biases are N(0, 0.02^2).
 
 Every floating value is drawn in fp32 and rounded to bf16 (round to nearest
-even); arrays of bf16 are carried as numpy ``uint16`` bit patterns.
+even); arrays of bf16 are carried as numpy ``uint16`` bit patterns. Small
+draws (field parameters, masks, keep ratios) use numpy's default_rng; the
+bulk normal draws use seeded torch CPU generators (faster).
 """
 from __future__ import annotations
 
@@ -28,18 +30,17 @@ import math
 from fractions import Fraction
 
 import numpy as np
+import torch
 
 # ---------------------------------------------------------------------------
 # bf16 bit helpers (storage format only)
 # ---------------------------------------------------------------------------
 
 
-def f32_to_bf16_bits(a: np.ndarray) -> np.ndarray:
+def f32_to_bf16_bits(a) -> np.ndarray:
     """Round fp32 values to bf16 (nearest even) and return the uint16 patterns."""
-    u = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32)
-    lsb = (u >> np.uint32(16)) & np.uint32(1)
-    r = (u + np.uint32(0x7FFF) + lsb) >> np.uint32(16)
-    return r.astype(np.uint16)
+    t = a if isinstance(a, torch.Tensor) else torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32))
+    return t.to(torch.float32).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
 
 
 def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
@@ -140,19 +141,28 @@ def denoise_loop(**kw) -> Workload:
 # ---------------------------------------------------------------------------
 
 
-def _field(rng: np.random.Generator, H: int, W: int, d: int) -> np.ndarray:
-    """Sum of 4 random 2-D sinusoids per channel, wavelength U[8,32] tokens."""
-    p = np.arange(H, dtype=np.float64)[:, None]
-    q = np.arange(W, dtype=np.float64)[None, :]
-    out = np.zeros((H, W, d), dtype=np.float64)
+def _field(rng: np.random.Generator, H: int, W: int, d: int) -> torch.Tensor:
+    """Sum of 4 random 2-D sinusoids per channel, wavelength U[8,32] tokens (fp32)."""
+    p = torch.arange(H, dtype=torch.float64)[:, None]
+    q = torch.arange(W, dtype=torch.float64)[None, :]
+    out = torch.zeros((H, W, d), dtype=torch.float64)
     for _ in range(4):
         lam = rng.uniform(8.0, 32.0)
         theta = rng.uniform(0.0, math.pi)
-        amp = rng.normal(0.0, 0.5, size=d)
-        phase = rng.uniform(0.0, 2.0 * math.pi, size=d)
+        amp = torch.from_numpy(rng.normal(0.0, 0.5, size=d))
+        phase = torch.from_numpy(rng.uniform(0.0, 2.0 * math.pi, size=d))
         arg = 2.0 * math.pi * (p * math.cos(theta) + q * math.sin(theta)) / lam   # [H,W]
-        out += amp[None, None, :] * np.sin(arg[:, :, None] + phase[None, None, :])
-    return out.astype(np.float32)
+        out += amp[None, None, :] * torch.sin(arg[:, :, None] + phase[None, None, :])
+    return out.to(torch.float32)
+
+
+def _normal(seed: int, shape, std: float = 1.0) -> torch.Tensor:
+    """Seeded N(0, std^2) fp32 draws (torch CPU generator)."""
+    g = torch.Generator().manual_seed(int(seed))
+    t = torch.randn(shape, generator=g, dtype=torch.float32)
+    if std != 1.0:
+        t.mul_(std)
+    return t
 
 
 def _rect_mask(rng: np.random.Generator, H: int, W: int, lo: float, hi: float) -> np.ndarray:
@@ -215,10 +225,11 @@ def make_batch(wl: Workload, seed_offset: int = 0) -> Batch:
             m = _ellipse_mask(rng, H, W, wl.mask_lo, wl.mask_hi)
         else:
             m = _rect_mask(rng, H, W, wl.mask_lo, wl.mask_hi)
-        noise = rng.standard_normal((H, W, d), dtype=np.float32)
-        f = np.where(m[:, :, None] == 1, noise, f)
+        noise_seed, text_seed = (int(v) for v in rng.integers(0, 2 ** 62, size=2))
+        noise = _normal(noise_seed, (H, W, d))
+        f = torch.where(torch.from_numpy(m)[:, :, None] == 1, noise, f)
         xs[b] = f32_to_bf16_bits(f)
-        ts[b] = f32_to_bf16_bits(rng.standard_normal((T, d), dtype=np.float32))
+        ts[b] = f32_to_bf16_bits(_normal(text_seed, (T, d)))
         ms[b] = m.reshape(N)
         if wl.keep_ratio is None:
             r = rng.uniform(wl.ratio_lo, wl.ratio_hi)
@@ -252,25 +263,21 @@ class BlockWeights:
     img: StreamWeights
 
 
-def _normal_bf16(rng: np.random.Generator, shape) -> np.ndarray:
-    a = rng.standard_normal(shape, dtype=np.float32)
-    a *= np.float32(0.02)
-    return f32_to_bf16_bits(a)
-
-
 def make_weights(d: int, mlp: bool, seed: int, mlp_ratio: int = 4) -> BlockWeights:
     """N(0, 0.02^2) weights and biases for both streams of one block."""
-    rng = np.random.default_rng(seed)
+    counter = [0]
+
+    def draw(shape) -> np.ndarray:
+        counter[0] += 1
+        return f32_to_bf16_bits(_normal(seed * 1000 + counter[0], shape, 0.02))
 
     def stream() -> StreamWeights:
-        s = StreamWeights(
-            w_qkv=_normal_bf16(rng, (3 * d, d)), b_qkv=_normal_bf16(rng, (3 * d,)),
-            w_o=_normal_bf16(rng, (d, d)), b_o=_normal_bf16(rng, (d,)))
+        s = StreamWeights(w_qkv=draw((3 * d, d)), b_qkv=draw((3 * d,)), w_o=draw((d, d)), b_o=draw((d,)))
         if mlp:
-            s.w_1 = _normal_bf16(rng, (mlp_ratio * d, d))
-            s.b_1 = _normal_bf16(rng, (mlp_ratio * d,))
-            s.w_2 = _normal_bf16(rng, (d, mlp_ratio * d))
-            s.b_2 = _normal_bf16(rng, (d,))
+            s.w_1 = draw((mlp_ratio * d, d))
+            s.b_1 = draw((mlp_ratio * d,))
+            s.w_2 = draw((d, mlp_ratio * d))
+            s.b_2 = draw((d,))
         return s
 
     return BlockWeights(txt=stream(), img=stream())

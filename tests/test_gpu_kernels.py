@@ -247,3 +247,18 @@ def test_host_argument_errors(H):
                              torch.empty(64, 128, dtype=torch.bfloat16, device="cuda"), H.HILO_BF16,
                              torch.empty(64, 128, device="cuda"), torch.empty(16, dtype=torch.uint8, device="cuda"), 16)
     assert e.value.status == -4
+
+
+def test_convert_bf16_to_f16(H):
+    rng = np.random.default_rng(31)
+    v = np.concatenate([rng.standard_normal(4096) * 0.02, rng.standard_normal(4096) * 100,
+                        [1e5, -1e6, 65504.0, 65520.0, 3e-5, 1e-9, 0.0, -0.0]]).astype(np.float32)
+    v = np.concatenate([v, np.zeros((-len(v)) % 8, np.float32)])
+    b = bits(v)
+    src = H.bf16_from_bits(b)
+    dst = torch.empty(len(v), dtype=torch.float16, device="cuda")
+    H.hilo_convert_bf16_to_f16(src, dst, len(v))
+    torch.cuda.synchronize()
+    exact = I.bf16_bits_to_f32(b)
+    ref = np.clip(exact, -65504, 65504).astype(np.float16)   # round to nearest even, saturate
+    assert np.array_equal(dst.cpu().numpy().view(np.uint16), ref.view(np.uint16))

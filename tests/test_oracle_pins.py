@@ -416,3 +416,14 @@ def test_update_closed_form():
     got = O.bf16_to_f32(O.update(x, y, 0.035))
     want = np.array([1.0 - np.float32(0.035), -2.0, 0.5 + 4 * np.float32(0.035)], dtype=np.float32)
     assert np.array_equal(got, O.bf16_to_f32(I.f32_to_bf16_bits(want)))
+
+
+def test_weights_f64_same_block():
+    rng = np.random.default_rng(12)
+    d, heads, T = 32, 2, 3
+    w = _rand_weights(rng, d, mlp=True)
+    ut = bits(rng.standard_normal((T, d)))
+    ui = bits(rng.standard_normal((7, d)))
+    a = O.block(ut, ui, [0, 7], T, w, heads, True)
+    b = O.block(ut, ui, [0, 7], T, O.weights_f64(w), heads, True)
+    assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
