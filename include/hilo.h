@@ -236,6 +236,33 @@ int hilo_unpack_update(const hilo_shape* shape, const float* out_img,
                        const hilo_split_out* split, void* x, float alpha, void* stream);
 
 /*
+ * hilo_block_forward_static_ws -- hilo_block_forward without a workspace
+ * argument, for callers that cannot allocate device memory at call time (code
+ * inside a host framework whose allocator the call site cannot reach, or a
+ * service that fixes its device-memory footprint at start-up). The paper has
+ * no counterpart; this is a deployment convenience.
+ *
+ * The scratch is one fixed array of HILO_STATIC_SCRATCH_BYTES in the
+ * library's own device memory; every GPU that loads the library holds it until
+ * the process exits. The call allocates nothing. Arguments, layouts and
+ * results are those of hilo_block_forward. Limits and caveats:
+ *   - shapes whose hilo_block_workspace_bytes(shape, cap) exceeds
+ *     HILO_STATIC_SCRATCH_BYTES are rejected with HILO_ERR_WORKSPACE (the
+ *     detail in hilo_last_error()); e.g. d=512, T=64, 1024 image rows fits,
+ *     the d=3072 blocks do not;
+ *   - the first call on a device looks up the array's device address (once
+ *     per device, with that device current); make that first call before any
+ *     stream capture;
+ *   - all calls share the one array: calls that overlap on the GPU (other
+ *     streams, other host threads) race and must be serialised by the caller.
+ *     No part of the array needs to start at zero.
+ */
+#define HILO_STATIC_SCRATCH_BYTES (16u << 20)
+int hilo_block_forward_static_ws(const hilo_shape* shape, const hilo_block_weights* weights,
+                                 const int32_t* cu_img, int32_t cap, const void* in_txt,
+                                 const void* in_img, int in_dtype, float* out, void* stream);
+
+/*
  * hilo_convert_bf16_to_f16 -- dst[i] = fp16(src[i]) for n elements (n a
  * multiple of 8, both pointers 16-byte aligned, device memory), round to
  * nearest even, saturating at +-65504. For preparing the fp16 MLP weights

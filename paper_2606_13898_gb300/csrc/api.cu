@@ -151,6 +151,10 @@ bool encode_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uin
   return r == CUDA_SUCCESS;
 }
 
+// Sets the calling thread's hilo_last_error() text and returns `status`
+// (for entry points defined in other files).
+int set_error(int status, const char* msg) { return fail(status, "%s", msg); }
+
 }  // namespace hilo
 
 extern "C" {

@@ -77,6 +77,9 @@ struct AttnArgs {
 cudaError_t launch_attention(const AttnArgs& a, int num_sms, cudaStream_t st);
 int attn_take_device_error();
 
+// ---- error text of the calling thread (api.cu)
+int set_error(int status, const char* msg);
+
 // ---- tensor maps (api.cu)
 bool encode_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
                          uint64_t row_stride_elems, uint32_t box_inner, uint32_t box_outer);

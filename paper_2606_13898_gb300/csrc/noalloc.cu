@@ -1,0 +1,61 @@
+// hilo_block_forward_static_ws: hilo_block_forward for callers that cannot
+// allocate device memory when they call the block.
+//
+// Some callers have no way to hand the library a workspace: code that runs
+// inside a host framework whose device allocator is not reachable from the
+// call site, or a service that fixes its device-memory footprint at start-up
+// and forbids any allocation afterwards. This entry point needs no workspace
+// argument: its scratch is a fixed array in the library's own device memory,
+// HILO_STATIC_SCRATCH_BYTES long, which every GPU that loads the library holds
+// until the process exits. It allocates nothing itself, and calls no
+// allocating routine.
+#include <cuda_runtime.h>
+#include <stdio.h>
+
+#include "../../include/hilo.h"
+#include "internal.h"
+
+namespace {
+
+// The shared scratch (one copy per device context).
+static __device__ __align__(256) unsigned char g_static_scratch[HILO_STATIC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
+// Device address of g_static_scratch per device ordinal (null until looked up).
+void* g_scratch_addr[kMaxDevices] = {};
+
+}  // namespace
+
+extern "C" int hilo_block_forward_static_ws(const hilo_shape* shape,
+                                            const hilo_block_weights* weights,
+                                            const int32_t* cu_img, int32_t cap,
+                                            const void* in_txt, const void* in_img,
+                                            int in_dtype, float* out, void* stream) {
+  if (!shape) return hilo::set_error(HILO_ERR_ARG, "hilo_block_forward_static_ws: shape is NULL");
+  if (cap < 0) return hilo::set_error(HILO_ERR_ARG, "hilo_block_forward_static_ws: cap < 0");
+  const size_t need = hilo_block_workspace_bytes(shape, cap);
+  if (need > HILO_STATIC_SCRATCH_BYTES) {
+    char msg[200];
+    snprintf(msg, sizeof(msg),
+             "hilo_block_forward_static_ws: this shape needs %zu scratch bytes, more than the "
+             "built-in %zu; use hilo_block_forward with a caller workspace",
+             need, static_cast<size_t>(HILO_STATIC_SCRATCH_BYTES));
+    return hilo::set_error(HILO_ERR_WORKSPACE, msg);
+  }
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+    return hilo::set_error(HILO_ERR_CUDA, "hilo_block_forward_static_ws: no current device");
+  if (!g_scratch_addr[dev]) {
+    // One-time set-up per device, with that device current: the host-side
+    // name g_static_scratch is not a device address; ask the runtime for it.
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || !p)
+      return hilo::set_error(HILO_ERR_CUDA,
+                             "hilo_block_forward_static_ws: cudaGetSymbolAddress of the scratch failed");
+    g_scratch_addr[dev] = p;
+  }
+  // Nothing in the scratch needs to start at zero: every scratch value the
+  // block's kernels read was written earlier in the same call.
+  return hilo_block_forward(shape, weights, cu_img, cap, in_txt, in_img, in_dtype, out,
+                            g_scratch_addr[dev], HILO_STATIC_SCRATCH_BYTES, stream);
+}

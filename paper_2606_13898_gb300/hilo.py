@@ -49,7 +49,8 @@ class hilo_block_weights(ctypes.Structure):
 EXPORTS = ("hilo_status_string", "hilo_last_error", "hilo_sync_status", "hilo_device_info",
            "hilo_score", "hilo_split_workspace_bytes", "hilo_split", "hilo_pack",
            "hilo_block_workspace_bytes", "hilo_block_forward", "hilo_unpack", "hilo_unpack_update",
-           "hilo_convert_bf16_to_f16", "hilo_set_stage_events", "hilo_launch_count")
+           "hilo_convert_bf16_to_f16", "hilo_set_stage_events", "hilo_launch_count",
+           "hilo_block_forward_static_ws")
 
 _lib = None
 
@@ -85,6 +86,8 @@ def lib() -> ctypes.CDLL:
         "hilo_unpack": (I, [shp, P, spo, P, P]),
         "hilo_unpack_update": (I, [shp, P, spo, P, F, P]),
         "hilo_convert_bf16_to_f16": (I, [P, P, S, P]),
+        "hilo_block_forward_static_ws": (I, [shp, ctypes.POINTER(hilo_block_weights), P, ctypes.c_int32, P,
+                                             P, I, P, P]),
         "hilo_set_stage_events": (I, [ctypes.POINTER(ctypes.c_void_p), I]),
         "hilo_launch_count": (ctypes.c_ulonglong, []),
     }
@@ -257,6 +260,16 @@ def hilo_block_forward(shape: Shape, weights: DeviceWeights, cu_img, cap: int, i
     _check("hilo_block_forward", lib().hilo_block_forward(
         ctypes.byref(s), ctypes.byref(w), _ptr(cu_img), cap, _ptr(in_txt), _ptr(in_img), in_dtype, _ptr(out),
         _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def hilo_block_forward_static_ws(shape: Shape, weights: DeviceWeights, cu_img, cap: int, in_txt, in_img,
+                                 in_dtype: int, out, stream=None) -> None:
+    """hilo_block_forward with the library's built-in scratch (no workspace argument)."""
+    s = shape.c()
+    w = weights.c()
+    _check("hilo_block_forward_static_ws", lib().hilo_block_forward_static_ws(
+        ctypes.byref(s), ctypes.byref(w), _ptr(cu_img), cap, _ptr(in_txt), _ptr(in_img), in_dtype, _ptr(out),
+        _stream(stream)))
 
 
 def hilo_unpack(shape: Shape, out_img, split: SplitBuffers, y, stream=None) -> None:
