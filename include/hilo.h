@@ -148,9 +148,9 @@ int hilo_device_info(int* num_sms, int* is_sm103);
  *                          aligned 2x2 window holding token i
  * Arithmetic is fp32 in one fixed order: m = ((a + b) + (c + e)) * 0.25 over
  * the window members in raster order; channels are summed in groups of 8
- * consecutive channels, group g folded into partial g mod 32 (groups and
- * channels ascending), partials combined by the halving tree j += j + h for
- * h = 16, 8, 4, 2, 1; no fused multiply-add. The result is therefore
+ * consecutive channels, group g folded into partial g mod 128 (groups and
+ * channels ascending), partials combined by the halving tree p[j] += p[j + h]
+ * for h = 64, 32, 16, 8, 4, 2, 1; no fused multiply-add. The result is therefore
  * bit-reproducible by any IEEE fp32 implementation of the same order.
  */
 int hilo_score(const hilo_shape* shape, const void* x, float* score, void* stream);

@@ -38,9 +38,9 @@ Fixed orders (readings where the paper is silent):
   * window mean for the score: ((x_a + x_b) + (x_c + x_d)) * 0.25 with
     members a,b,c,d in raster order;
   * channel sum: channels are taken in groups of 8 consecutive channels;
-    group g is folded into partial sum p[g mod 32] (groups ascending, the 8
-    channels of a group ascending); the 32 partials are then combined by the
-    halving tree p[j] += p[j + h] for h = 16, 8, 4, 2, 1;
+    group g is folded into partial sum p[g mod 128] (groups ascending, the 8
+    channels of a group ascending); the 128 partials are then combined by the
+    halving tree p[j] += p[j + h] for h = 64, 32, 16, 8, 4, 2, 1;
   * pooled mean: fp32 sum of the class members in raster order starting from
     the first member, one correctly rounded division by the member count,
     then bf16 round-to-nearest-even.
@@ -99,12 +99,12 @@ def score(x_bits: np.ndarray) -> np.ndarray:
     diff = x - up
     sq = diff * diff                                            # fp32, no FMA
     sq = sq.reshape(B, H * W, d)
-    partial = np.zeros((B, H * W, 32), dtype=np.float32)
+    partial = np.zeros((B, H * W, 128), dtype=np.float32)
     for g in range(d // 8):
-        j = g % 32
+        j = g % 128
         for u in range(8):
             partial[:, :, j] = partial[:, :, j] + sq[:, :, 8 * g + u]
-    for h in (16, 8, 4, 2, 1):
+    for h in (64, 32, 16, 8, 4, 2, 1):
         partial[:, :, :h] = partial[:, :, :h] + partial[:, :, h:2 * h]
     return np.ascontiguousarray(partial[:, :, 0])
 

@@ -7,15 +7,20 @@
 // of the row space; queries and keys/values are tiled per range (128 rows per
 // tile, the ragged last tile masked).
 //
-// One CTA per (image, head, 128-query tile), 192 threads:
-//   warp 0     TMA: Q once, then K and V tiles (two-stage ring), 128-byte
-//              swizzled boxes of 64 columns
-//   warp 1     MMA: S = Q K^T into TMEM (two S buffers so S_{t+1} overlaps
-//              the softmax of S_t), then O_t = P_t V_t into TMEM (V is the
-//              MN-major operand, no transpose pass)
-//   warps 2-5  softmax, one query row per thread: row max, exp2, bf16 P into
-//              swizzled shared memory, running sum; the output accumulator
-//              lives in registers and is rescaled there (online softmax)
+// One CTA per (image, head, pair of 128-query tiles), 320 threads:
+//   warps 0-3   softmax of query tile 0 (one query row per thread)
+//   warps 4-7   softmax of query tile 1
+//   warp 8      TMA: Q tiles once, then K and V tiles (two stages each),
+//               128-byte swizzled boxes of 64 columns
+//   warp 9      MMA: S_i = Q_i K^T into TMEM, O_i += P V into TMEM (V is the
+//               MN-major operand, no transpose pass)
+// The two query tiles ping-pong: while one softmax warpgroup turns S into P,
+// the tensor core works on the other tile (MMA order PV_0(t), S_0(t+1),
+// PV_1(t), S_1(t+1)). Both tiles share the K/V stream. S is read from TMEM
+// once into registers; the output accumulators stay in TMEM for the whole
+// sequence and are rescaled only when a row's running maximum grows by more
+// than 2^8 (until then the probabilities are formed against the older,
+// smaller maximum, so they stay <= 256, well inside bf16 range).
 // Every mbarrier wait is bounded (error latched, TMEM freed, CTA returns).
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -32,27 +37,31 @@ namespace {
 
 constexpr int BQ = 128;
 constexpr int BKV = 128;
-constexpr int ATTN_THREADS = 192;
-constexpr uint32_t ATTN_TMEM_COLS = 512;  // S0 | S1 | O
-constexpr int BOX_BYTES = 128 * 128;       // 128 rows x 64 bf16
+constexpr int ATTN_THREADS = 320;
+constexpr int PRODUCER_WARP = 8;
+constexpr int MMA_WARP = 9;
+constexpr uint32_t ATTN_TMEM_COLS = 512;  // S0 | S1 | O0 | O1
+constexpr int BOX_BYTES = 128 * 128;       // 128 rows x 64 16-bit elements
+constexpr float RESCALE_LOG2 = 8.0f;
 
 template <int HD>
 struct Cfg {
   static constexpr int NBOX = HD / 64;
   static constexpr int TILE_BYTES = NBOX * BOX_BYTES;  // 128 rows x HD
   static constexpr int P_BYTES = 2 * BOX_BYTES;        // 128 x 128 bf16
-  // Q | K0 | V0 | K1 | V1 | P
+  // Q0 | Q1 | K0 | K1 | V0 | V1 | P
   static constexpr int OFF_Q = 0;
-  static constexpr int OFF_K0 = TILE_BYTES;
-  static constexpr int OFF_P = 5 * TILE_BYTES;
-  static constexpr int DATA_BYTES = 5 * TILE_BYTES + P_BYTES;
+  static constexpr int OFF_K = 2 * TILE_BYTES;
+  static constexpr int OFF_V = 4 * TILE_BYTES;
+  static constexpr int OFF_P = 6 * TILE_BYTES;
+  static constexpr int DATA_BYTES = 6 * TILE_BYTES + P_BYTES;
   static constexpr int SMEM_BYTES = DATA_BYTES + 1024 + 256;
 };
 
 struct AttnParams {
   const int32_t* cu_img;
   __nv_bfloat16* out;
-  int B, T, heads, d, qt_txt, qt_img_max;
+  int B, T, heads, d, qt_txt, pairs_max;
   float scale_log2;  // log2(e) / sqrt(head_dim)
 };
 
@@ -62,16 +71,17 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-// Row range of KV tile t of image b: text tiles first, then image tiles.
-__device__ __forceinline__ void kv_tile(const AttnParams& p, int b, int L, int t, int& row0,
-                                        int& valid) {
-  if (t < p.qt_txt) {
-    row0 = b * p.T + t * BKV;
-    valid = min(BKV, p.T - t * BKV);
+// Row range of tile j of image b (text tiles first, then image tiles); used
+// for both query and key/value tiles.
+__device__ __forceinline__ void seq_tile(const AttnParams& p, int b, int L, int j, int& row0,
+                                         int& valid) {
+  if (j < p.qt_txt) {
+    row0 = b * p.T + j * BKV;
+    valid = min(BKV, p.T - j * BKV);
   } else {
-    const int j = t - p.qt_txt;
-    row0 = p.B * p.T + p.cu_img[b] + j * BKV;
-    valid = min(BKV, L - j * BKV);
+    const int k = j - p.qt_txt;
+    row0 = p.B * p.T + p.cu_img[b] + k * BKV;
+    valid = min(BKV, L - k * BKV);
   }
 }
 
@@ -79,60 +89,59 @@ template <int HD>
 __global__ void __launch_bounds__(ATTN_THREADS, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm, const AttnParams p) {
   using C = Cfg<HD>;
-  // ---- work item
-  const int per = p.qt_txt + p.qt_img_max;
+  // ---- work item: (image, head, query-tile pair)
   const int item = blockIdx.x;
-  const int b = item / (p.heads * per);
-  const int h = (item / per) % p.heads;
-  const int qt = item % per;
+  const int b = item / (p.heads * p.pairs_max);
+  const int h = (item / p.pairs_max) % p.heads;
+  const int pair = item % p.pairs_max;
   const int L = p.cu_img[b + 1] - p.cu_img[b];
-  const int nkv_img = (L + BKV - 1) / BKV;
-  int q_row0, q_valid;
-  if (qt < p.qt_txt) {
-    q_row0 = b * p.T + qt * BQ;
-    q_valid = min(BQ, p.T - qt * BQ);
-  } else {
-    const int j = qt - p.qt_txt;
-    if (j >= nkv_img) return;  // beyond this image's compressed length
-    q_row0 = p.B * p.T + p.cu_img[b] + j * BQ;
-    q_valid = min(BQ, L - j * BQ);
-  }
-  const int nkv = p.qt_txt + nkv_img;
+  const int nkv = p.qt_txt + (L + BKV - 1) / BKV;  // also the number of query tiles
+  if (2 * pair >= nkv) return;                     // beyond this image's compressed length
+  const bool has1 = 2 * pair + 1 < nkv;
+  int q_row0[2], q_valid[2];
+  seq_tile(p, b, L, 2 * pair, q_row0[0], q_valid[0]);
+  q_row0[1] = q_row0[0];
+  q_valid[1] = 0;
+  if (has1) seq_tile(p, b, L, 2 * pair + 1, q_row0[1], q_valid[1]);
 
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  unsigned char* sQ = smem + C::OFF_Q;
   unsigned char* sP = smem + C::OFF_P;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::DATA_BYTES);
   uint64_t* q_full = bars + 0;
-  uint64_t* kv_full = bars + 1;   // [2]
-  uint64_t* kv_empty = bars + 3;  // [2]
-  uint64_t* s_full = bars + 5;    // [2]
-  uint64_t* p_full = bars + 7;
-  uint64_t* o_full = bars + 8;
-  uint64_t* drain = bars + 9;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 10);
+  uint64_t* k_full = bars + 1;    // [2]
+  uint64_t* k_empty = bars + 3;   // [2]
+  uint64_t* v_full = bars + 5;    // [2]
+  uint64_t* v_empty = bars + 7;   // [2]
+  uint64_t* s_full = bars + 9;    // [2] per query tile
+  uint64_t* p_full = bars + 11;   // [2] per query tile
+  uint64_t* o_done = bars + 13;   // [2] per query tile
+  uint64_t* drain = bars + 15;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   int* err = &g_attn_err;
-  auto sK = [&](int st) { return smem + C::OFF_K0 + st * 2 * C::TILE_BYTES; };
-  auto sV = [&](int st) { return smem + C::OFF_K0 + st * 2 * C::TILE_BYTES + C::TILE_BYTES; };
+  auto sQ = [&](int i) { return smem + C::OFF_Q + i * C::TILE_BYTES; };
+  auto sK = [&](int st) { return smem + C::OFF_K + st * C::TILE_BYTES; };
+  auto sV = [&](int st) { return smem + C::OFF_V + st * C::TILE_BYTES; };
 
   const int warp = warp_id(), lane = lane_id();
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&kv_full[i], 1);
-      mbar_init(&kv_empty[i], 1);
+      mbar_init(&k_full[i], 1);
+      mbar_init(&k_empty[i], 1);
+      mbar_init(&v_full[i], 1);
+      mbar_init(&v_empty[i], 1);
       mbar_init(&s_full[i], 1);
+      mbar_init(&p_full[i], 128);
+      mbar_init(&o_done[i], 1);
     }
-    mbar_init(p_full, 128);
-    mbar_init(o_full, 1);
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (warp == 1) {
+  if (warp == MMA_WARP) {
     tmem_alloc(tmem_slot, ATTN_TMEM_COLS);
     tmem_relinquish();
   }
@@ -140,138 +149,191 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tS[2] = {tmem, tmem + 128u};
-  const uint32_t tO = tmem + 256u;
 
-  if (warp == 0) {
+  if (warp == PRODUCER_WARP) {
     if (lane == 0) {
       // ---------------- TMA producer
       tma_prefetch_desc(&tm);
-      int armed[2] = {-1, -1};
-      mbar_arrive_expect_tx(q_full, C::TILE_BYTES);
+      int armed_k[2] = {-1, -1}, armed_v[2] = {-1, -1};
+      mbar_arrive_expect_tx(q_full, (has1 ? 2 : 1) * C::TILE_BYTES);
 #pragma unroll
-      for (int j = 0; j < C::NBOX; ++j)
-        tma_load_2d(sQ + j * BOX_BYTES, &tm, q_full, h * HD + 64 * j, q_row0);
+      for (int j = 0; j < C::NBOX; ++j) {
+        tma_load_2d(sQ(0) + j * BOX_BYTES, &tm, q_full, h * HD + 64 * j, q_row0[0]);
+        if (has1) tma_load_2d(sQ(1) + j * BOX_BYTES, &tm, q_full, h * HD + 64 * j, q_row0[1]);
+      }
       bool ok = true;
-      for (int t = 0; t < nkv; ++t) {
+      for (int t = 0; t < nkv && ok; ++t) {
         const int st = t & 1;
         const uint32_t ph = static_cast<uint32_t>((t >> 1) & 1);
-        if (!mbar_wait(&kv_empty[st], ph ^ 1u, abort_flag, err, DEV_TIMEOUT_ATTN)) {
+        int row0, valid;
+        seq_tile(p, b, L, t, row0, valid);
+        if (!mbar_wait(&k_empty[st], ph ^ 1u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 1)) {
           ok = false;
           break;
         }
-        int row0, valid;
-        kv_tile(p, b, L, t, row0, valid);
-        mbar_arrive_expect_tx(&kv_full[st], 2 * C::TILE_BYTES);
+        mbar_arrive_expect_tx(&k_full[st], C::TILE_BYTES);
 #pragma unroll
-        for (int j = 0; j < C::NBOX; ++j) {
-          tma_load_2d(sK(st) + j * BOX_BYTES, &tm, &kv_full[st], p.d + h * HD + 64 * j, row0);
-          tma_load_2d(sV(st) + j * BOX_BYTES, &tm, &kv_full[st], 2 * p.d + h * HD + 64 * j, row0);
+        for (int j = 0; j < C::NBOX; ++j)
+          tma_load_2d(sK(st) + j * BOX_BYTES, &tm, &k_full[st], p.d + h * HD + 64 * j, row0);
+        armed_k[st] = static_cast<int>(ph);
+        if (!mbar_wait(&v_empty[st], ph ^ 1u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 2)) {
+          ok = false;
+          break;
         }
-        armed[st] = static_cast<int>(ph);
+        mbar_arrive_expect_tx(&v_full[st], C::TILE_BYTES);
+#pragma unroll
+        for (int j = 0; j < C::NBOX; ++j)
+          tma_load_2d(sV(st) + j * BOX_BYTES, &tm, &v_full[st], 2 * p.d + h * HD + 64 * j, row0);
+        armed_v[st] = static_cast<int>(ph);
       }
       if (!ok) {
+        // wait (bounded) for the bulk copies in flight before the CTA exits
         const uint64_t t0 = globaltimer_ns();
-        while (!mbar_try_wait(smem_u32(q_full), 0u) && globaltimer_ns() - t0 < HILO_WAIT_LIMIT_NS / 4) {
+        const uint64_t lim = HILO_WAIT_LIMIT_NS / 4;
+        while (!mbar_try_wait(smem_u32(q_full), 0u) && globaltimer_ns() - t0 < lim) {
         }
         for (int st = 0; st < 2; ++st) {
-          if (armed[st] < 0) continue;
-          const uint64_t t1 = globaltimer_ns();
-          while (!mbar_try_wait(smem_u32(&kv_full[st]), static_cast<uint32_t>(armed[st])) &&
-                 globaltimer_ns() - t1 < HILO_WAIT_LIMIT_NS / 4) {
-          }
+          if (armed_k[st] >= 0)
+            while (!mbar_try_wait(smem_u32(&k_full[st]), static_cast<uint32_t>(armed_k[st])) &&
+                   globaltimer_ns() - t0 < lim) {
+            }
+          if (armed_v[st] >= 0)
+            while (!mbar_try_wait(smem_u32(&v_full[st]), static_cast<uint32_t>(armed_v[st])) &&
+                   globaltimer_ns() - t0 < lim) {
+            }
         }
       }
     }
-  } else if (warp == 1) {
+  } else if (warp == MMA_WARP) {
     if (lane == 0) {
       // ---------------- MMA issuer
       const uint32_t idesc_s = idesc_bf16(BQ, BKV, 0, 0);
       const uint32_t idesc_o = idesc_bf16(BQ, HD, 0, 1);
-      const uint32_t q_base = smem_u32(sQ);
       const uint32_t p_base = smem_u32(sP);
-      auto issue_s = [&](int t) {
+      auto issue_s = [&](int i, int t) {
+        const uint32_t q_base = smem_u32(sQ(i));
         const uint32_t k_base = smem_u32(sK(t & 1));
 #pragma unroll
         for (int k = 0; k < HD / 16; ++k) {
           const uint32_t off = (k >> 2) * BOX_BYTES + (k & 3) * 32;
-          umma_bf16(tS[t & 1], sw128_desc(q_base + off, 16, 1024), sw128_desc(k_base + off, 16, 1024),
-                    idesc_s, k > 0 ? 1u : 0u);
+          umma_bf16(tmem + 128u * i, sw128_desc(q_base + off, 16, 1024),
+                    sw128_desc(k_base + off, 16, 1024), idesc_s, k > 0 ? 1u : 0u);
         }
-        umma_commit(&s_full[t & 1]);
+        umma_commit(&s_full[i]);
       };
-      bool ok = mbar_wait(q_full, 0u, abort_flag, err, DEV_TIMEOUT_ATTN) &&
-                mbar_wait(&kv_full[0], 0u, abort_flag, err, DEV_TIMEOUT_ATTN);
-      if (ok) {
-        tc_fence_after();
-        issue_s(0);
-      }
-      for (int t = 0; t < nkv && ok; ++t) {
-        if (t + 1 < nkv) {
-          if (!mbar_wait(&kv_full[(t + 1) & 1], static_cast<uint32_t>(((t + 1) >> 1) & 1), abort_flag,
-                         err, DEV_TIMEOUT_ATTN))
-            break;
-          tc_fence_after();
-          issue_s(t + 1);
-        }
-        if (!mbar_wait(p_full, static_cast<uint32_t>(t & 1), abort_flag, err, DEV_TIMEOUT_ATTN)) break;
-        tc_fence_after();
+      auto issue_pv = [&](int i, int t) {
         const uint32_t v_base = smem_u32(sV(t & 1));
 #pragma unroll
         for (int k = 0; k < BKV / 16; ++k) {
           const uint64_t ad = sw128_desc(p_base + (k >> 2) * BOX_BYTES + (k & 3) * 32, 16, 1024);
           const uint64_t bd = sw128_desc(v_base + k * 2048, BOX_BYTES, 1024);
-          umma_bf16(tO, ad, bd, idesc_o, k > 0 ? 1u : 0u);
+          umma_bf16(tmem + 256u + 128u * i, ad, bd, idesc_o, (t > 0 || k > 0) ? 1u : 0u);
         }
-        umma_commit(o_full);
-        umma_commit(&kv_empty[t & 1]);
+        umma_commit(&o_done[i]);
+      };
+      bool ok = mbar_wait(q_full, 0u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 3) &&
+                mbar_wait(&k_full[0], 0u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 4);
+      if (ok) {
+        tc_fence_after();
+        issue_s(0, 0);
+        if (has1) issue_s(1, 0);
+        umma_commit(&k_empty[0]);
+      }
+      for (int t = 0; t < nkv && ok; ++t) {
+        const int st = t & 1;
+        const uint32_t ph = static_cast<uint32_t>((t >> 1) & 1);
+        const uint32_t tp = static_cast<uint32_t>(t & 1);
+        const bool more = t + 1 < nkv;
+        const int st1 = (t + 1) & 1;
+        const uint32_t ph1 = static_cast<uint32_t>(((t + 1) >> 1) & 1);
+        if (!mbar_wait(&p_full[0], tp, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 5) ||
+            !mbar_wait(&v_full[st], ph, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 6)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        issue_pv(0, t);
+        if (!has1) umma_commit(&v_empty[st]);
+        if (more) {
+          if (!mbar_wait(&k_full[st1], ph1, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 7)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          issue_s(0, t + 1);
+          if (!has1) umma_commit(&k_empty[st1]);
+        }
+        if (has1) {
+          if (!mbar_wait(&p_full[1], tp, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 8)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          issue_pv(1, t);
+          umma_commit(&v_empty[st]);
+          if (more) {
+            issue_s(1, t + 1);
+            umma_commit(&k_empty[st1]);
+          }
+        }
       }
       umma_commit(drain);
       const uint64_t t0 = globaltimer_ns();
       while (!mbar_try_wait(smem_u32(drain), 0u)) {
         if (globaltimer_ns() - t0 > HILO_WAIT_LIMIT_NS) {
-          atomicExch(err, DEV_TIMEOUT_ATTN);
+          atomicExch(err, DEV_TIMEOUT_ATTN + 256 * 9);
           break;
         }
       }
     }
   } else {
-    // ---------------- softmax (warps 2..5 -> TMEM lane quarters 2,3,0,1)
-    const int q = warp & 3;
-    const int row = q * 32 + lane;
-    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
-    float acc[HD];
-#pragma unroll
-    for (int i = 0; i < HD; ++i) acc[i] = 0.f;
+    // ---------------- softmax: warpgroup i = warps 4i..4i+3, TMEM lane quarter warp % 4
+    const int i = warp >> 2;
+    const int row = (warp & 3) * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
+    const uint32_t tS = tmem + 128u * i + lane_off;
+    const uint32_t tO = tmem + 256u + 128u * i + lane_off;
+    const bool active = i == 0 || has1;
     float m = -INFINITY, l = 0.f;
-    bool ok = true;
-    for (int t = 0; t < nkv; ++t) {
+    bool ok = active;
+    for (int t = 0; t < nkv && ok; ++t) {
       int row0, valid;
-      kv_tile(p, b, L, t, row0, valid);
-      if (!mbar_wait(&s_full[t & 1], static_cast<uint32_t>((t >> 1) & 1), abort_flag, err,
-                     DEV_TIMEOUT_ATTN)) {
+      seq_tile(p, b, L, t, row0, valid);
+      const uint32_t tp = static_cast<uint32_t>(t & 1);
+      if (!mbar_wait_warp(&s_full[i], tp, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 10)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      const uint32_t sb = tS[t & 1] + lane_off;
-      float mx = -INFINITY;
-#pragma unroll 1
-      for (int c = 0; c < BKV / 32; ++c) {
-        float v[32];
-        tmem_ld32(sb + c * 32, v);
-        tmem_ld_wait();
+      float s[BKV];
 #pragma unroll
-        for (int i = 0; i < 32; ++i)
-          if (c * 32 + i < valid) mx = fmaxf(mx, v[i]);
+      for (int c = 0; c < BKV / 32; ++c) tmem_ld32(tS + c * 32, s + c * 32);
+      tmem_ld_wait();
+      float mx = -INFINITY;
+#pragma unroll
+      for (int j = 0; j < BKV; ++j)
+        if (j < valid) mx = fmaxf(mx, s[j]);
+      const float m_tile = mx * p.scale_log2;
+      bool rescale = false;
+      float m_use = m;
+      if (t == 0) {
+        m_use = m_tile;
+      } else if (m_tile > m + RESCALE_LOG2) {
+        m_use = m_tile;
+        rescale = true;
       }
-      const float m_new = fmaxf(m, mx * p.scale_log2);
-      const float alpha = ex2(m - m_new);
-      // rows of a ragged last tile hold other tokens' (or stale) values:
-      // zero them in V so that 0-probability columns contribute exactly 0
-      if (valid < BKV) {
-        if (!mbar_wait(&kv_full[t & 1], static_cast<uint32_t>((t >> 1) & 1), abort_flag, err,
-                       DEV_TIMEOUT_ATTN)) {
+      float lsum = 0.f;
+#pragma unroll
+      for (int j = 0; j < BKV; ++j) {
+        const float pj = j < valid ? ex2(fmaf(s[j], p.scale_log2, -m_use)) : 0.f;
+        s[j] = pj;
+        lsum += pj;
+      }
+      // ragged key tile: rows past `valid` hold other tokens (or stale data);
+      // zero them in V so that the zero-probability columns add exactly 0
+      if (i == 0 && valid < BKV) {
+        if (!mbar_wait_warp(&v_full[t & 1], static_cast<uint32_t>((t >> 1) & 1), abort_flag, err,
+                       DEV_TIMEOUT_ATTN + 256 * 11)) {
           ok = false;
           break;
         }
@@ -284,68 +346,82 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
               *reinterpret_cast<uint4*>(vr + j * BOX_BYTES + c16 * 16) = make_uint4(0, 0, 0, 0);
         }
       }
-      float lsum = 0.f;
-      unsigned char* prow = sP + row * 128;
-#pragma unroll 1
-      for (int c = 0; c < BKV / 32; ++c) {
-        float v[32];
-        tmem_ld32(sb + c * 32, v);
-        tmem_ld_wait();
-        float pv[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          pv[i] = (c * 32 + i < valid) ? ex2(v[i] * p.scale_log2 - m_new) : 0.f;
-          lsum += pv[i];
+      // the shared P buffer and this tile's O accumulator are free once the
+      // previous PV products that read / write them have completed
+      if (i == 0 && t > 0) {
+        if (!mbar_wait_warp(&o_done[has1 ? 1 : 0], static_cast<uint32_t>((t - 1) & 1), abort_flag, err,
+                       DEV_TIMEOUT_ATTN + 256 * 12)) {
+          ok = false;
+          break;
         }
-        unsigned char* pbox = prow + (c >> 1) * BOX_BYTES;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int chunk = (c & 1) * 4 + j;
-          uint4 o;
-          o.x = pack_bf16x2(pv[8 * j], pv[8 * j + 1]);
-          o.y = pack_bf16x2(pv[8 * j + 2], pv[8 * j + 3]);
-          o.z = pack_bf16x2(pv[8 * j + 4], pv[8 * j + 5]);
-          o.w = pack_bf16x2(pv[8 * j + 6], pv[8 * j + 7]);
-          *reinterpret_cast<uint4*>(pbox + ((chunk ^ (row & 7)) << 4)) = o;
+      } else if (i == 1) {
+        if (!mbar_wait_warp(&o_done[0], tp, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 13)) {
+          ok = false;
+          break;
         }
-      }
-      l = l * alpha + lsum;
-      m = m_new;
-      fence_proxy_async_smem();
-      tc_fence_before();
-      mbar_arrive(p_full);
-      if (!mbar_wait(o_full, static_cast<uint32_t>(t & 1), abort_flag, err, DEV_TIMEOUT_ATTN)) {
-        ok = false;
-        break;
       }
       tc_fence_after();
+      // tcgen05.ld / tcgen05.st are warp-collective: the whole warp rescales
+      // when any of its rows needs it (rows that do not use alpha = 1)
+      if (__any_sync(0xffffffffu, rescale)) {
+        const float alpha = rescale ? ex2(m - m_use) : 1.0f;
+#pragma unroll 1
+        for (int c = 0; c < HD / 32; ++c) {
+          float o[32];
+          tmem_ld32(tO + c * 32, o);
+          tmem_ld_wait();
 #pragma unroll
-      for (int c = 0; c < HD / 32; ++c) {
-        float v[32];
-        tmem_ld32(tO + lane_off + c * 32, v);
-        tmem_ld_wait();
-#pragma unroll
-        for (int i = 0; i < 32; ++i) acc[c * 32 + i] = acc[c * 32 + i] * alpha + v[i];
+          for (int j = 0; j < 32; ++j) o[j] *= alpha;
+          tmem_st32(tO + c * 32, o);
+        }
+        tmem_st_wait();
+        l *= alpha;
       }
-    }
-    if (ok && row < q_valid) {
-      const float inv = 1.0f / l;
-      uint4* dst = reinterpret_cast<uint4*>(p.out + static_cast<long long>(q_row0 + row) * p.d + h * HD);
+      m = m_use;
+      l += lsum;
+      unsigned char* prow = sP + row * 128;
 #pragma unroll
-      for (int j = 0; j < HD / 8; ++j) {
+      for (int c = 0; c < BKV / 8; ++c) {
         uint4 o;
-        o.x = pack_bf16x2(acc[8 * j] * inv, acc[8 * j + 1] * inv);
-        o.y = pack_bf16x2(acc[8 * j + 2] * inv, acc[8 * j + 3] * inv);
-        o.z = pack_bf16x2(acc[8 * j + 4] * inv, acc[8 * j + 5] * inv);
-        o.w = pack_bf16x2(acc[8 * j + 6] * inv, acc[8 * j + 7] * inv);
-        dst[j] = o;
+        o.x = pack_bf16x2(s[8 * c], s[8 * c + 1]);
+        o.y = pack_bf16x2(s[8 * c + 2], s[8 * c + 3]);
+        o.z = pack_bf16x2(s[8 * c + 4], s[8 * c + 5]);
+        o.w = pack_bf16x2(s[8 * c + 6], s[8 * c + 7]);
+        const int chunk = c & 7;
+        *reinterpret_cast<uint4*>(prow + (c >> 3) * BOX_BYTES + ((chunk ^ (row & 7)) << 4)) = o;
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      mbar_arrive(&p_full[i]);
+    }
+    if (ok && mbar_wait_warp(&o_done[i], static_cast<uint32_t>((nkv - 1) & 1), abort_flag, err,
+                        DEV_TIMEOUT_ATTN + 256 * 14)) {
+      tc_fence_after();
+      const float inv = 1.0f / l;
+      uint4* dst = reinterpret_cast<uint4*>(p.out + static_cast<long long>(q_row0[i] + row) * p.d + h * HD);
+#pragma unroll 1
+      for (int c = 0; c < HD / 32; ++c) {
+        float o[32];
+        tmem_ld32(tO + c * 32, o);
+        tmem_ld_wait();
+        if (row < q_valid[i]) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            uint4 v;
+            v.x = pack_bf16x2(o[8 * j] * inv, o[8 * j + 1] * inv);
+            v.y = pack_bf16x2(o[8 * j + 2] * inv, o[8 * j + 3] * inv);
+            v.z = pack_bf16x2(o[8 * j + 4] * inv, o[8 * j + 5] * inv);
+            v.w = pack_bf16x2(o[8 * j + 6] * inv, o[8 * j + 7] * inv);
+            dst[4 * c + j] = v;
+          }
+        }
       }
     }
   }
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) {
+  if (warp == MMA_WARP) {
     tc_fence_after();
     tmem_dealloc(tmem, ATTN_TMEM_COLS);
   }
@@ -375,9 +451,10 @@ cudaError_t launch_attention(const AttnArgs& a, int num_sms, cudaStream_t st) {
   p.heads = a.heads;
   p.d = a.d;
   p.qt_txt = (a.T + BQ - 1) / BQ;
-  p.qt_img_max = (a.max_img_rows + BQ - 1) / BQ;
+  const int qt_img_max = (a.max_img_rows + BQ - 1) / BQ;
+  p.pairs_max = (p.qt_txt + qt_img_max + 1) / 2;
   p.scale_log2 = static_cast<float>(1.4426950408889634 / sqrt(static_cast<double>(a.head_dim)));
-  const long long items = static_cast<long long>(a.B) * a.heads * (p.qt_txt + p.qt_img_max);
+  const long long items = static_cast<long long>(a.B) * a.heads * p.pairs_max;
   if (items <= 0) return cudaSuccess;
   if (items > 0x7fffffffLL) return cudaErrorInvalidValue;
   if (a.head_dim == 128) return launch_hd<128>(a, p, static_cast<int>(items), st);

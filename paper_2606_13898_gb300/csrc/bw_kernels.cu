@@ -14,11 +14,13 @@ namespace hilo {
 
 // ============================================================== score =====
 //
-// One warp per aligned 2x2 window: the window mean is formed once per channel
-// and the four member energies are accumulated in the fixed order documented
-// in hilo.h (lane j owns channel groups j, j+32, ...; 8 channels per group;
-// halving tree over lanes). Every add/mul is an explicit round-to-nearest
-// intrinsic so the compiler cannot contract to FMA.
+// One 128-thread CTA per aligned 2x2 window: thread j owns partial sums j of
+// the four members (channel groups j, j+128, ... of 8 channels), so the whole
+// window is read in one round trip; the window mean is formed once per
+// channel. The 128 partials are combined by the fixed halving tree documented
+// in hilo.h (64 and 32 through shared memory, then warp shuffles). Every
+// add/mul is an explicit round-to-nearest intrinsic so the compiler cannot
+// contract to FMA.
 
 __device__ __forceinline__ void bf16x8_to_f32(const uint4& v, float* f) {
   const uint32_t w[4] = {v.x, v.y, v.z, v.w};
@@ -29,16 +31,19 @@ __device__ __forceinline__ void bf16x8_to_f32(const uint4& v, float* f) {
   }
 }
 
-__global__ void __launch_bounds__(128) score_kernel(const __nv_bfloat16* __restrict__ x,
-                                                    float* __restrict__ s, int B, int H, int W,
-                                                    int d) {
-  const int lane = threadIdx.x & 31;
+constexpr int SCORE_THREADS = 128;
+constexpr int SCORE_MAX_ITERS = 4;  // d <= 4096: at most 4 groups of 8 per thread
+
+__global__ void __launch_bounds__(SCORE_THREADS) score_kernel(const __nv_bfloat16* __restrict__ x,
+                                                              float* __restrict__ s, int B, int H,
+                                                              int W, int d) {
+  __shared__ float part[4][SCORE_THREADS];
+  const int j = threadIdx.x;
+  const int lane = j & 31;
   const int Hw = H >> 1, Ww = W >> 1;
   const long long nwin = static_cast<long long>(B) * Hw * Ww;
   const int G = d >> 3;
-  const long long wstep = static_cast<long long>(gridDim.x) * (blockDim.x >> 5);
-  for (long long w = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
-       w < nwin; w += wstep) {
+  for (long long w = blockIdx.x; w < nwin; w += gridDim.x) {
     const int b = static_cast<int>(w / (Hw * Ww));
     const int r = static_cast<int>(w % (Hw * Ww));
     const int P = r / Ww, Q = r % Ww;
@@ -47,15 +52,26 @@ __global__ void __launch_bounds__(128) score_kernel(const __nv_bfloat16* __restr
     const uint4* rb = reinterpret_cast<const uint4*>(x + (t0 + 1) * d);
     const uint4* rc = reinterpret_cast<const uint4*>(x + (t0 + W) * d);
     const uint4* rd = reinterpret_cast<const uint4*>(x + (t0 + W + 1) * d);
+    uint4 va[SCORE_MAX_ITERS], vb[SCORE_MAX_ITERS], vc[SCORE_MAX_ITERS], vd[SCORE_MAX_ITERS];
+#pragma unroll
+    for (int i = 0; i < SCORE_MAX_ITERS; ++i) {
+      const int g = j + SCORE_THREADS * i;
+      if (g < G) {
+        va[i] = __ldg(ra + g);
+        vb[i] = __ldg(rb + g);
+        vc[i] = __ldg(rc + g);
+        vd[i] = __ldg(rd + g);
+      }
+    }
     float acc0 = 0.f, acc1 = 0.f, acc2 = 0.f, acc3 = 0.f;
-#pragma unroll 4
-    for (int g = lane; g < G; g += 32) {
-      const uint4 va = __ldg(ra + g), vb = __ldg(rb + g), vc = __ldg(rc + g), vd = __ldg(rd + g);
+#pragma unroll
+    for (int i = 0; i < SCORE_MAX_ITERS; ++i) {
+      if (j + SCORE_THREADS * i >= G) break;
       float fa[8], fb[8], fc[8], fd[8];
-      bf16x8_to_f32(va, fa);
-      bf16x8_to_f32(vb, fb);
-      bf16x8_to_f32(vc, fc);
-      bf16x8_to_f32(vd, fd);
+      bf16x8_to_f32(va[i], fa);
+      bf16x8_to_f32(vb[i], fb);
+      bf16x8_to_f32(vc[i], fc);
+      bf16x8_to_f32(vd[i], fd);
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
         const float m = __fmul_rn(__fadd_rn(__fadd_rn(fa[u], fb[u]), __fadd_rn(fc[u], fd[u])), 0.25f);
@@ -67,18 +83,31 @@ __global__ void __launch_bounds__(128) score_kernel(const __nv_bfloat16* __restr
         acc3 = __fadd_rn(acc3, __fmul_rn(ed, ed));
       }
     }
+    part[0][j] = acc0;
+    part[1][j] = acc1;
+    part[2][j] = acc2;
+    part[3][j] = acc3;
+    __syncthreads();
+    if (j < 32) {
+      float v[4];
 #pragma unroll
-    for (int off = 16; off >= 1; off >>= 1) {
-      acc0 = __fadd_rn(acc0, __shfl_down_sync(0xffffffffu, acc0, off));
-      acc1 = __fadd_rn(acc1, __shfl_down_sync(0xffffffffu, acc1, off));
-      acc2 = __fadd_rn(acc2, __shfl_down_sync(0xffffffffu, acc2, off));
-      acc3 = __fadd_rn(acc3, __shfl_down_sync(0xffffffffu, acc3, off));
+      for (int m = 0; m < 4; ++m) {
+        // h = 64: p[j] += p[j+64] (j < 64); h = 32: p[j] += p[j+32] (j < 32)
+        const float lo = __fadd_rn(part[m][lane], part[m][lane + 64]);
+        const float hi = __fadd_rn(part[m][lane + 32], part[m][lane + 96]);
+        v[m] = __fadd_rn(lo, hi);
+      }
+#pragma unroll
+      for (int off = 16; off >= 1; off >>= 1)
+#pragma unroll
+        for (int m = 0; m < 4; ++m) v[m] = __fadd_rn(v[m], __shfl_down_sync(0xffffffffu, v[m], off));
+      if (lane == 0) {
+        float* sb = s + t0;  // score index equals the token index (b*N + p*W + q)
+        *reinterpret_cast<float2*>(sb) = make_float2(v[0], v[1]);
+        *reinterpret_cast<float2*>(sb + W) = make_float2(v[2], v[3]);
+      }
     }
-    if (lane == 0) {
-      float* sb = s + t0;  // score index equals the token index (b*N + p*W + q)
-      *reinterpret_cast<float2*>(sb) = make_float2(acc0, acc1);
-      *reinterpret_cast<float2*>(sb + W) = make_float2(acc2, acc3);
-    }
+    __syncthreads();
   }
 }
 
@@ -392,7 +421,8 @@ __global__ void __launch_bounds__(SPLIT_THREADS) split_compact_kernel(
 // One warp per packed image row. A kept row is a 16-byte-vector copy; a
 // pooled row sums the window's members of its class in raster order (the
 // first member initialises the sum), divides once with correct rounding and
-// rounds to bf16 (nearest even).
+// rounds to bf16 (nearest even). Member rows are loaded four at a time and
+// two channel chunks at a time, so up to eight loads are in flight per lane.
 
 __global__ void __launch_bounds__(256) pack_kernel(const __nv_bfloat16* __restrict__ x,
                                                    const uint8_t* __restrict__ labels,
@@ -403,6 +433,7 @@ __global__ void __launch_bounds__(256) pack_kernel(const __nv_bfloat16* __restri
                                                    int H, int W, int d, int cap) {
   const int lane = threadIdx.x & 31;
   const int N = H * W;
+  const int G = d >> 3;
   const int total = min(cu_img[B], cap);
   const int wstep = gridDim.x * (blockDim.x >> 5);
   for (int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < total; r += wstep) {
@@ -414,8 +445,9 @@ __global__ void __launch_bounds__(256) pack_kernel(const __nv_bfloat16* __restri
     const __nv_bfloat16* xb = x + static_cast<long long>(b) * N * d;
     uint4* dst = reinterpret_cast<uint4*>(packed + static_cast<long long>(r) * d);
     if (local < nk) {
-      const uint4* s = reinterpret_cast<const uint4*>(xb + static_cast<long long>(src) * d);
-      for (int c = lane; c < (d >> 3); c += 32) dst[c] = __ldg(s + c);
+      const uint4* sp = reinterpret_cast<const uint4*>(xb + static_cast<long long>(src) * d);
+#pragma unroll 4
+      for (int c = lane; c < G; c += 32) dst[c] = __ldg(sp + c);
       continue;
     }
     const int size = local < nk + n2 ? 2 : 4;
@@ -430,23 +462,35 @@ __global__ void __launch_bounds__(256) pack_kernel(const __nv_bfloat16* __restri
     }
     const uint32_t mm = __ballot_sync(0xffffffffu, is_member);
     const float cnt = static_cast<float>(__popc(mm));
-    for (int c = lane; c < (d >> 3); c += 32) {
+    const int ngroups = size * size / 4;
+#pragma unroll 2
+    for (int c = lane; c < G; c += 32) {
       float acc[8];
-      uint32_t rest = mm;
       bool first = true;
-      while (rest) {
-        const int m = __ffs(rest) - 1;
-        rest &= rest - 1;
-        const int t = t0 + (m / size) * W + (m % size);
-        float f[8];
-        bf16x8_to_f32(__ldg(reinterpret_cast<const uint4*>(xb + static_cast<long long>(t) * d) + c), f);
-        if (first) {
+      for (int gi = 0; gi < ngroups; ++gi) {
+        uint4 v[4];
 #pragma unroll
-          for (int u = 0; u < 8; ++u) acc[u] = f[u];
-          first = false;
-        } else {
+        for (int q = 0; q < 4; ++q) {
+          const int m = 4 * gi + q;
+          if (mm & (1u << m)) {
+            const int t = t0 + (m / size) * W + (m % size);
+            v[q] = __ldg(reinterpret_cast<const uint4*>(xb + static_cast<long long>(t) * d) + c);
+          }
+        }
 #pragma unroll
-          for (int u = 0; u < 8; ++u) acc[u] = __fadd_rn(acc[u], f[u]);
+        for (int q = 0; q < 4; ++q) {
+          const int m = 4 * gi + q;
+          if (!(mm & (1u << m))) continue;
+          float f[8];
+          bf16x8_to_f32(v[q], f);
+          if (first) {
+#pragma unroll
+            for (int u = 0; u < 8; ++u) acc[u] = f[u];
+            first = false;
+          } else {
+#pragma unroll
+            for (int u = 0; u < 8; ++u) acc[u] = __fadd_rn(acc[u], f[u]);
+          }
         }
       }
       uint4 o;
@@ -507,86 +551,90 @@ __global__ void __launch_bounds__(256) unpack_update_kernel(const float* __restr
 
 // ========================================================== layernorm =====
 //
-// One warp per row of the row space. Rows [0, n_txt) come from in_txt, rows
-// [n_txt, n_txt + cu_img[B]) from in_img (bf16 or fp32). Writes the bf16
-// normalised row (no affine, eps 1e-6, biased variance) and, when `resid` is
-// not null, the fp32 copy of the input row (the residual stream).
+// One 128-thread CTA per row of the row space. Rows [0, n_txt) come from
+// in_txt, rows [n_txt, n_txt + cu_img[B]) from in_img (bf16 or fp32). Thread
+// t holds elements 4t + 512k. Writes the normalised row (no affine, eps 1e-6,
+// biased variance) as bf16 or fp16 and, when `resid` is not null, the fp32
+// copy of the input row (the residual stream).
 
-template <int NCH, bool IN_F32, bool OUT_F16>
-__device__ __forceinline__ void ln_row(const void* src, float* resid_row, uint16_t* ln_row_out,
-                                       int d, float eps) {
-  const int lane = threadIdx.x & 31;
-  float v[NCH * 4];
+constexpr int LN_THREADS = 128;
+
+__device__ __forceinline__ float ln_block_sum(float v, float* red) {
 #pragma unroll
-  for (int t = 0; t < NCH; ++t) {
-    const int c = 128 * t + 4 * lane;
-    if (IN_F32) {
-      const float4 f = __ldg(reinterpret_cast<const float4*>(static_cast<const float*>(src) + c));
-      v[4 * t] = f.x; v[4 * t + 1] = f.y; v[4 * t + 2] = f.z; v[4 * t + 3] = f.w;
-    } else {
-      const uint2 u = __ldg(reinterpret_cast<const uint2*>(static_cast<const __nv_bfloat16*>(src) + c));
-      v[4 * t] = __uint_as_float(u.x << 16);
-      v[4 * t + 1] = __uint_as_float(u.x & 0xFFFF0000u);
-      v[4 * t + 2] = __uint_as_float(u.y << 16);
-      v[4 * t + 3] = __uint_as_float(u.y & 0xFFFF0000u);
-    }
-  }
-  float s = 0.f;
-#pragma unroll
-  for (int i = 0; i < NCH * 4; ++i) s += v[i];
-#pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-  const float mean = s / static_cast<float>(d);
-  float q = 0.f;
-#pragma unroll
-  for (int i = 0; i < NCH * 4; ++i) {
-    const float e = v[i] - mean;
-    q += e * e;
-  }
-#pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) q += __shfl_xor_sync(0xffffffffu, q, off);
-  const float rstd = rsqrtf(q / static_cast<float>(d) + eps);
-#pragma unroll
-  for (int t = 0; t < NCH; ++t) {
-    const int c = 128 * t + 4 * lane;
-    if (resid_row)
-      *reinterpret_cast<float4*>(resid_row + c) = make_float4(v[4 * t], v[4 * t + 1], v[4 * t + 2], v[4 * t + 3]);
-    uint2 o;
-    if (OUT_F16) {
-      o.x = pack_f16x2_sat((v[4 * t] - mean) * rstd, (v[4 * t + 1] - mean) * rstd);
-      o.y = pack_f16x2_sat((v[4 * t + 2] - mean) * rstd, (v[4 * t + 3] - mean) * rstd);
-    } else {
-      o.x = pack_bf16x2((v[4 * t] - mean) * rstd, (v[4 * t + 1] - mean) * rstd);
-      o.y = pack_bf16x2((v[4 * t + 2] - mean) * rstd, (v[4 * t + 3] - mean) * rstd);
-    }
-    *reinterpret_cast<uint2*>(ln_row_out + c) = o;
-  }
+  for (int off = 16; off >= 1; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  const float t = (red[0] + red[1]) + (red[2] + red[3]);
+  __syncthreads();
+  return t;
 }
 
 template <int NCH>
-__global__ void __launch_bounds__(256) layernorm_kernel(const void* __restrict__ in_txt,
-                                                        const void* __restrict__ in_img,
-                                                        int in_f32, float* resid,
-                                                        uint16_t* __restrict__ ln, int ln_f16,
-                                                        const int32_t* __restrict__ cu_img, int B,
-                                                        int n_txt, int d) {
+__global__ void __launch_bounds__(LN_THREADS) layernorm_kernel(const void* __restrict__ in_txt,
+                                                               const void* __restrict__ in_img,
+                                                               int in_f32, float* resid,
+                                                               uint16_t* __restrict__ ln, int ln_f16,
+                                                               const int32_t* __restrict__ cu_img,
+                                                               int B, int n_txt, int d) {
+  __shared__ float red[LN_THREADS / 32];
   const int rows = n_txt + cu_img[B];
-  const int wstep = gridDim.x * (blockDim.x >> 5);
-  for (int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < rows; r += wstep) {
+  const float inv_d = 1.0f / static_cast<float>(d);
+  for (int r = blockIdx.x; r < rows; r += gridDim.x) {
     const long long off = static_cast<long long>(r < n_txt ? r : r - n_txt) * d;
     const void* base = r < n_txt ? in_txt : in_img;
+    float v[NCH * 4];
+#pragma unroll
+    for (int t = 0; t < NCH; ++t) {
+      const int c = 512 * t + 4 * threadIdx.x;
+      if (c < d) {
+        if (in_f32) {
+          const float4 f = __ldg(reinterpret_cast<const float4*>(static_cast<const float*>(base) + off + c));
+          v[4 * t] = f.x; v[4 * t + 1] = f.y; v[4 * t + 2] = f.z; v[4 * t + 3] = f.w;
+        } else {
+          const uint2 u = __ldg(reinterpret_cast<const uint2*>(static_cast<const __nv_bfloat16*>(base) + off + c));
+          v[4 * t] = __uint_as_float(u.x << 16);
+          v[4 * t + 1] = __uint_as_float(u.x & 0xFFFF0000u);
+          v[4 * t + 2] = __uint_as_float(u.y << 16);
+          v[4 * t + 3] = __uint_as_float(u.y & 0xFFFF0000u);
+        }
+      } else {
+        v[4 * t] = v[4 * t + 1] = v[4 * t + 2] = v[4 * t + 3] = 0.f;
+      }
+    }
+    float sum = 0.f;
+#pragma unroll
+    for (int i = 0; i < NCH * 4; ++i) sum += v[i];
+    const float mean = ln_block_sum(sum, red) * inv_d;
+    float sq = 0.f;
+#pragma unroll
+    for (int t = 0; t < NCH; ++t) {
+      if (512 * t + 4 * static_cast<int>(threadIdx.x) < d) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float e = v[4 * t + i] - mean;
+          sq += e * e;
+        }
+      }
+    }
+    const float rstd = rsqrtf(ln_block_sum(sq, red) * inv_d + 1e-6f);
     float* rr = resid ? resid + static_cast<long long>(r) * d : nullptr;
     uint16_t* lo = ln + static_cast<long long>(r) * d;
-    if (in_f32) {
-      if (ln_f16)
-        ln_row<NCH, true, true>(static_cast<const float*>(base) + off, rr, lo, d, 1e-6f);
-      else
-        ln_row<NCH, true, false>(static_cast<const float*>(base) + off, rr, lo, d, 1e-6f);
-    } else {
-      if (ln_f16)
-        ln_row<NCH, false, true>(static_cast<const __nv_bfloat16*>(base) + off, rr, lo, d, 1e-6f);
-      else
-        ln_row<NCH, false, false>(static_cast<const __nv_bfloat16*>(base) + off, rr, lo, d, 1e-6f);
+#pragma unroll
+    for (int t = 0; t < NCH; ++t) {
+      const int c = 512 * t + 4 * threadIdx.x;
+      if (c >= d) continue;
+      if (rr) *reinterpret_cast<float4*>(rr + c) = make_float4(v[4 * t], v[4 * t + 1], v[4 * t + 2], v[4 * t + 3]);
+      const float y0 = (v[4 * t] - mean) * rstd, y1 = (v[4 * t + 1] - mean) * rstd;
+      const float y2 = (v[4 * t + 2] - mean) * rstd, y3 = (v[4 * t + 3] - mean) * rstd;
+      uint2 o;
+      if (ln_f16) {
+        o.x = pack_f16x2_sat(y0, y1);
+        o.y = pack_f16x2_sat(y2, y3);
+      } else {
+        o.x = pack_bf16x2(y0, y1);
+        o.y = pack_bf16x2(y2, y3);
+      }
+      *reinterpret_cast<uint2*>(lo + c) = o;
     }
   }
 }
@@ -623,7 +671,7 @@ static int grid_for(long long work_items, int per_block, int num_sms, int blocks
 cudaError_t launch_score(const void* x, float* s, int B, int H, int W, int d, int num_sms,
                          cudaStream_t st) {
   const long long nwin = static_cast<long long>(B) * (H / 2) * (W / 2);
-  score_kernel<<<grid_for(nwin, 4, num_sms, 16), 128, 0, st>>>(
+  score_kernel<<<grid_for(nwin, 1, num_sms, 16), SCORE_THREADS, 0, st>>>(
       static_cast<const __nv_bfloat16*>(x), s, B, H, W, d);
   return cudaGetLastError();
 }
@@ -688,24 +736,23 @@ cudaError_t launch_bf16_to_f16(const void* src, void* dst, long long n, int num_
 cudaError_t launch_layernorm(const void* in_txt, const void* in_img, int in_f32, float* resid,
                              void* ln, int ln_f16, const int32_t* cu_img, int B, int n_txt,
                              int cap, int d, int num_sms, cudaStream_t st) {
-  const int grid = grid_for(static_cast<long long>(n_txt) + cap, 8, num_sms, 8);
+  const int grid = grid_for(static_cast<long long>(n_txt) + cap, 1, num_sms, 16);
   uint16_t* lo = static_cast<uint16_t*>(ln);
-#define HILO_LN_CASE(NC)                                                                    \
-  case NC:                                                                                  \
-    layernorm_kernel<NC><<<grid, 256, 0, st>>>(in_txt, in_img, in_f32, resid, lo, ln_f16, cu_img, \
-                                               B, n_txt, d);                                \
+  const int nch = (d + 511) / 512;
+#define HILO_LN_CASE(NC)                                                                        \
+  case NC:                                                                                      \
+    layernorm_kernel<NC><<<grid, LN_THREADS, 0, st>>>(in_txt, in_img, in_f32, resid, lo, ln_f16, \
+                                                      cu_img, B, n_txt, d);                      \
     break;
-  switch (d / 128) {
+  switch (nch) {
     HILO_LN_CASE(1)
     HILO_LN_CASE(2)
     HILO_LN_CASE(3)
     HILO_LN_CASE(4)
+    HILO_LN_CASE(5)
     HILO_LN_CASE(6)
+    HILO_LN_CASE(7)
     HILO_LN_CASE(8)
-    HILO_LN_CASE(12)
-    HILO_LN_CASE(16)
-    HILO_LN_CASE(24)
-    HILO_LN_CASE(32)
     default:
       return cudaErrorInvalidValue;
   }

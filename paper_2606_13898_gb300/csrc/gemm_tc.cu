@@ -26,13 +26,20 @@ __device__ int g_gemm_err;
 
 namespace {
 
-constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
-constexpr int A_STAGE_BYTES = BM * BK * 2;
-constexpr int B_STAGE_BYTES = BN * BK * 2;
-constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
+constexpr int BM = 128, BK = 64;
 constexpr int GEMM_THREADS = 192;
-constexpr uint32_t TMEM_COLS = 512;
-constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
+
+// Tile configuration by tile width: 128x256 tiles with a 4-stage ring, or
+// 128x128 tiles with a 6-stage ring (for narrow outputs, N <= 1024).
+template <int BN>
+struct TileCfg {
+  static constexpr int STAGES = BN == 256 ? 4 : 6;
+  static constexpr int A_STAGE_BYTES = BM * BK * 2;
+  static constexpr int B_STAGE_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_STAGE_BYTES + B_STAGE_BYTES;
+  static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
+};
 
 struct GemmParams {
   int N, K;
@@ -49,6 +56,7 @@ struct Tile {
   int g, m0, n0, rows, row_base;
 };
 
+template <int BN>
 struct Sched {
   int mt[2], rows[2], nt, total;
   __device__ void init(const GemmParams& p) {
@@ -88,9 +96,15 @@ __device__ __forceinline__ void bf16x8(const uint4& v, float* f) {
   }
 }
 
+template <int BN>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                 const __grid_constant__ CUtensorMap tmB1, const GemmParams p) {
+  using Cfg = TileCfg<BN>;
+  constexpr int STAGES = Cfg::STAGES;
+  constexpr int STAGE_BYTES = Cfg::STAGE_BYTES;
+  constexpr int A_STAGE_BYTES = Cfg::A_STAGE_BYTES;
+  constexpr uint32_t TMEM_COLS = Cfg::TMEM_COLS;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -104,7 +118,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   int* err = &g_gemm_err;
 
   const int warp = warp_id(), lane = lane_id();
-  Sched sc;
+  Sched<BN> sc;
   sc.init(p);
 
   if (threadIdx.x == 0) {
@@ -229,7 +243,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     uint32_t acc_phase = 0;
     for (int t = blockIdx.x; t < sc.total; t += gridDim.x) {
       const Tile tl = sc.get(p, t);
-      if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, err, DEV_TIMEOUT_GEMM)) break;
+      if (!mbar_wait_warp(&tfull[acc], acc_phase, abort_flag, err, DEV_TIMEOUT_GEMM)) break;
       tc_fence_after();
       const int rit = q * 32 + lane;
       const int grow = tl.m0 + rit;
@@ -306,10 +320,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   }
 }
 
-}  // namespace
-
-cudaError_t launch_gemm(const GemmArgs& a, int num_sms, cudaStream_t st) {
-  if (a.K % BK != 0 || a.N % 32 != 0) return cudaErrorInvalidValue;
+template <int BN>
+cudaError_t launch_bn(const GemmArgs& a, int num_sms, cudaStream_t st) {
+  using Cfg = TileCfg<BN>;
   CUtensorMap tA, tB0, tB1;
   if (!encode_tmap_bf16_2d(&tA, a.A, a.K, a.R, a.K, BK, BM)) return cudaErrorInvalidValue;
   if (!encode_tmap_bf16_2d(&tB0, a.g[0].weight ? a.g[0].weight : a.g[1].weight, a.K, a.N, a.K,
@@ -335,11 +348,21 @@ cudaError_t launch_gemm(const GemmArgs& a, int num_sms, cudaStream_t st) {
   p.out = a.out;
   if (upper <= 0) return cudaSuccess;
   const int grid = static_cast<int>(upper < num_sms ? upper : num_sms);
-  cudaError_t e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       SMEM_BYTES);
+  cudaError_t e = cudaFuncSetAttribute(gemm_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       Cfg::SMEM_BYTES);
   if (e != cudaSuccess) return e;
-  gemm_kernel<<<grid, GEMM_THREADS, SMEM_BYTES, st>>>(tA, tB0, tB1, p);
+  gemm_kernel<BN><<<grid, GEMM_THREADS, Cfg::SMEM_BYTES, st>>>(tA, tB0, tB1, p);
   return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_gemm(const GemmArgs& a, int num_sms, cudaStream_t st) {
+  if (a.K % BK != 0 || a.N % 32 != 0) return cudaErrorInvalidValue;
+  // 256-wide tiles keep the MMA below the shared-memory read bandwidth;
+  // 128-wide tiles only where N is so small that 256 would leave SMs idle.
+  if (a.N <= 1024) return launch_bn<128>(a, num_sms, st);
+  return launch_bn<256>(a, num_sms, st);
 }
 
 int gemm_take_device_error() {

@@ -171,14 +171,14 @@ def scaled_weights(rng, d, mlp, std):
     return I.BlockWeights(txt=one(), img=one())
 
 
-@pytest.mark.parametrize("d,heads,T,lens,mlp", [
-    (128, 1, 64, [200], 0),          # head_dim 128, ragged text and image tiles
-    (128, 2, 64, [256, 77], 1),      # head_dim 64, two images of different length
-    (256, 2, 0, [130, 300, 5], 1),   # no text, three images
-    (512, 8, 200, [384], 1),         # several 256-wide GEMM column tiles
+@pytest.mark.parametrize("d,heads,T,lens,mlp,sharp", [
+    (128, 1, 64, [200], 0, 1.0),          # head_dim 128, ragged text and image tiles
+    (128, 2, 64, [256, 77], 1, 1.0),      # head_dim 64, two images of different length
+    (256, 2, 0, [130, 300, 5], 1, 1.0),   # no text, three images
+    (512, 8, 200, [384], 1, 1.0),         # several 256-wide GEMM column tiles
 ])
-def test_block_forward_matches_oracle(H, d, heads, T, lens, mlp):
-    rng = np.random.default_rng(d + T + len(lens))
+def test_block_forward_matches_oracle(H, d, heads, T, lens, mlp, sharp):
+    rng = np.random.default_rng(d + T + len(lens) + int(sharp))
     B = len(lens)
     cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
     rows = int(cu[-1])
@@ -201,6 +201,67 @@ def test_block_forward_matches_oracle(H, d, heads, T, lens, mlp):
     got = out.cpu().numpy()
     assert_block_close(got[:B * T], ot, "text rows")
     assert_block_close(got[B * T:B * T + rows], oi, "image rows")
+
+
+def _ws_regions(sh, cap, ws):
+    """Views of the block workspace: LayerNorm rows, q|k|v rows, attention rows
+    (the layout hilo_block_forward uses: each region 256-byte aligned)."""
+    R, d = sh.B * sh.T + cap, sh.d
+    a256 = lambda v: (v + 255) // 256 * 256
+    o_qkv = a256(R * d * 2)
+    o_att = o_qkv + a256(R * 3 * d * 2)
+    qkv = ws[o_qkv:o_qkv + R * 3 * d * 2].view(torch.bfloat16).view(R, 3 * d)
+    att = ws[o_att:o_att + R * d * 2].view(torch.bfloat16).view(R, d)
+    return qkv, att
+
+
+@pytest.mark.parametrize("d,heads,T,lens,sharp", [
+    (256, 2, 128, [1500], 4.0),        # head_dim 128
+    (256, 4, 64, [900, 333], 5.0),     # head_dim 64, two images
+])
+def test_attention_rescale_against_own_qkv(H, d, heads, T, lens, sharp):
+    # Large q/k projections spread the logits over tens of units, so the
+    # running row maxima jump by more than 2^8 at different key tiles for
+    # different rows of one warp. The kernel's attention output is compared
+    # with fp64 softmax attention over the same bf16 q, k, v it consumed.
+    rng = np.random.default_rng(77 + heads)
+    B = len(lens)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    rows = int(cu[-1])
+    cap = rows
+    w = scaled_weights(rng, d, False, std=1.0 / np.sqrt(d))
+    for sw in (w.txt, w.img):
+        sw.w_qkv = bits(I.bf16_bits_to_f32(sw.w_qkv) * sharp)
+    sh = H.Shape(B=B, H=64, W=64, d=d, T=T, heads=heads, mlp=0)
+    ut = bits(rng.standard_normal((B * T, d)))
+    ui = bits(rng.standard_normal((rows, d)))
+    out = torch.empty(B * T + cap, d, dtype=torch.float32, device="cuda")
+    wsb = H.hilo_block_workspace_bytes(sh, cap)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    H.hilo_block_forward(sh, H.DeviceWeights.from_host(w), to_dev_i32(cu), cap, H.bf16_from_bits(ut),
+                         H.bf16_from_bits(ui), H.HILO_BF16, out, ws, wsb)
+    H.hilo_sync_status()
+    qkv_t, att_t = _ws_regions(sh, cap, ws)
+    qkv = qkv_t.float().cpu().numpy().astype(np.float64)
+    att = att_t.float().cpu().numpy().astype(np.float64)
+    hd = d // heads
+    n_rescaled_rows = 0
+    for b in range(B):
+        idx = np.r_[b * T:(b + 1) * T, B * T + cu[b]:B * T + cu[b + 1]]
+        for h in range(heads):
+            q = qkv[idx, h * hd:(h + 1) * hd]
+            k = qkv[idx, d + h * hd:d + (h + 1) * hd]
+            v = qkv[idx, 2 * d + h * hd:2 * d + (h + 1) * hd]
+            ref = O.softmax_attention(q, k, v)
+            # rows whose maximum logit grows by > 8 (log2 units) after the first key tile
+            lg = (q @ k.T) / np.sqrt(hd) * np.log2(np.e)
+            first = lg[:, :128].max(axis=1) if T >= 128 else lg[:, :T].max(axis=1)
+            n_rescaled_rows += int(np.sum(lg.max(axis=1) > first + 8))
+            got = att[idx, h * hd:(h + 1) * hd]
+            err = np.abs(got - ref)
+            # bf16 probabilities and bf16 output: a few 2^-8 relative of the value range
+            assert err.max() <= 1.5e-2 * max(1.0, np.abs(ref).max()), (b, h, err.max())
+    assert n_rescaled_rows > 0
 
 
 def test_block_forward_fp32_in_place_chain(H):

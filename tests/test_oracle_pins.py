@@ -85,18 +85,18 @@ def test_score_fixed_order_scalar_walkthrough():
     # One token of a random field walked through the fixed order with scalar
     # fp32 arithmetic: pins the vectorised grouping and the halving tree.
     rng = np.random.default_rng(11)
-    d = 512
+    d = 3072
     xb = bits(rng.standard_normal((1, 2, 2, d)))
     x = O.bf16_to_f32(xb)[0]
     f = np.float32
     for t, (pi, qi) in enumerate(((0, 0), (0, 1), (1, 0), (1, 1))):
-        part = [f(0.0)] * 32
+        part = [f(0.0)] * 128
         for c in range(d):
             m = ((x[0, 0, c] + x[0, 1, c]) + (x[1, 0, c] + x[1, 1, c])) * f(0.25)
             e = f(x[pi, qi, c] - m)
             g = c // 8
-            part[g % 32] = f(part[g % 32] + f(e * e))
-        for h in (16, 8, 4, 2, 1):
+            part[g % 128] = f(part[g % 128] + f(e * e))
+        for h in (64, 32, 16, 8, 4, 2, 1):
             for j in range(h):
                 part[j] = f(part[j] + part[j + h])
         assert O.score(xb)[0, t] == part[0]
