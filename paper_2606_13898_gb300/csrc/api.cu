@@ -190,10 +190,13 @@ int hilo_sync_status(void* stream) {
   cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "hilo_sync_status: stream");
   const int g = hilo::gemm_take_device_error();
+  const int g2 = hilo::gemm2_take_device_error();
   const int a = hilo::attn_take_device_error();
-  if (g < 0 || a < 0) return fail(HILO_ERR_CUDA, "hilo_sync_status: reading the device error word failed");
-  if (g || a)
-    return fail(HILO_ERR_TIMEOUT, "device-side wait ran out (gemm=%d, attention=%d)", g, a);
+  if (g < 0 || g2 < 0 || a < 0)
+    return fail(HILO_ERR_CUDA, "hilo_sync_status: reading the device error word failed");
+  if (g || g2 || a)
+    return fail(HILO_ERR_TIMEOUT, "device-side wait ran out (gemm=%d, gemm pair=%d, attention=%d)", g, g2,
+                a);
   return HILO_OK;
 }
 

@@ -1,0 +1,385 @@
+// Grouped GEMM on CTA pairs (tcgen05 cta_group::2): same computation and
+// epilogues as gemm_tc.cu, with 256x256 output tiles per pair of SMs.
+//
+// Each CTA of a pair loads 128 rows of A and 128 rows of W (half of the
+// tile's 256 output columns) into its own shared memory at identical offsets;
+// the even CTA issues tcgen05.mma.cta_group::2 with M = 256, N = 256, which
+// reads both CTAs' halves. Compared with one SM computing a 128x256 tile,
+// each SM stages and feeds half the W bytes per MAC, so the shared-memory
+// traffic per MAC drops by a third and the ring can be 6 stages deep.
+//
+// Per CTA, 192 threads:
+//   warp 0     TMA producer: A and W halves; the completion of both CTAs'
+//              copies is counted on the even CTA's "full" barrier
+//   warp 1     TMEM allocation (both CTAs); MMA issue (even CTA only)
+//   warps 2-5  epilogue over this CTA's 128 rows x 256 columns
+// "empty" and "accumulator ready" barriers are signalled in both CTAs by a
+// multicast commit; "accumulator free" collects 8 arrivals (4 epilogue warps
+// x 2 CTAs) in the even CTA. Every wait is bounded.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace hilo {
+
+__device__ int g_gemm2_err;
+
+namespace {
+
+constexpr int PM = 256;   // rows per pair tile (128 per CTA)
+constexpr int PN = 256;   // columns per pair tile (128 of W rows staged per CTA)
+constexpr int BK = 64;
+constexpr int STAGES = 6;
+constexpr int HALF_BYTES = 128 * BK * 2;    // 16 KB: one CTA's A or W slice
+constexpr int STAGE_BYTES = 2 * HALF_BYTES; // A + W slices of this CTA
+constexpr int THREADS = 192;
+constexpr uint32_t TMEM_COLS = 512;         // two 128 x 256 fp32 accumulators
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
+
+struct Params {
+  int N, K;
+  uint32_t idesc;
+  int row_base[2];
+  int rows_static[2];
+  const int32_t* rows_dev[2];
+  const __nv_bfloat16* bias[2];
+  int epilogue;
+  void* out;
+};
+
+struct Tile {
+  int g, m0, n0, rows, row_base;
+};
+
+struct Sched {
+  int mt[2], rows[2], nt, total;
+  __device__ void init(const Params& p) {
+    nt = (p.N + PN - 1) / PN;
+    total = 0;
+#pragma unroll
+    for (int g = 0; g < 2; ++g) {
+      rows[g] = p.rows_dev[g] ? *p.rows_dev[g] : p.rows_static[g];
+      mt[g] = (rows[g] + PM - 1) / PM;
+      total += mt[g] * nt;
+    }
+  }
+  __device__ Tile get(const Params& p, int t) const {
+    Tile r;
+    r.g = t < mt[0] * nt ? 0 : 1;
+    if (r.g) t -= mt[0] * nt;
+    const int mtg = mt[r.g];
+    r.m0 = p.row_base[r.g] + (t % mtg) * PM;
+    r.n0 = (t / mtg) * PN;
+    r.rows = rows[r.g];
+    r.row_base = p.row_base[r.g];
+    return r;
+  }
+};
+
+__device__ __forceinline__ float gelu_tanh(float z) {
+  const float k0 = 0.7978845608028654f;  // sqrt(2/pi)
+  return 0.5f * z * (1.0f + tanhf(k0 * (z + 0.044715f * z * z * z)));
+}
+
+__device__ __forceinline__ void bf16x8(const uint4& v, float* f) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    f[2 * i] = __uint_as_float(w[i] << 16);
+    f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+  }
+}
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
+    gemm2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
+                 const __grid_constant__ CUtensorMap tmB1, const Params p) {
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* tfull = empty + STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  int* err = &g_gemm2_err;
+
+  const int warp = warp_id(), lane = lane_id();
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  const int cid = blockIdx.x >> 1;
+  const int ncl = gridDim.x >> 1;
+  Sched sc;
+  sc.init(p);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 8);  // 4 epilogue warps x 2 CTAs
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB0);
+    tma_prefetch_desc(&tmB1);
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(tmem_slot, TMEM_COLS);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // both CTAs' barriers are initialised before any remote use
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const int kblocks = p.K / BK;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer (both CTAs)
+      int stage = 0;
+      uint32_t phase = 0;
+      int armed[STAGES];
+      for (int s = 0; s < STAGES; ++s) armed[s] = -1;
+      bool ok = true;
+      for (int t = cid; t < sc.total && ok; t += ncl) {
+        const Tile tl = sc.get(p, t);
+        const CUtensorMap* tb = tl.g ? &tmB1 : &tmB0;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, err, DEV_TIMEOUT_GEMM + 256 * 1)) {
+            ok = false;
+            break;
+          }
+          unsigned char* sa = smem + stage * STAGE_BYTES;
+          const uint32_t full_cl = mapa_shared(smem_u32(&full[stage]), 0);
+          if (leader) mbar_arrive_expect_tx(&full[stage], 2 * STAGE_BYTES);
+          tma_load_2d_pair(sa, &tmA, full_cl, kb * BK, tl.m0 + 128 * static_cast<int>(rank));
+          tma_load_2d_pair(sa + HALF_BYTES, tb, full_cl, kb * BK, tl.n0 + 128 * static_cast<int>(rank));
+          armed[stage] = static_cast<int>(phase);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        // let the bulk copies already issued land before the CTA can exit
+        const uint64_t t0 = globaltimer_ns();
+        if (leader) {
+          for (int s = 0; s < STAGES; ++s) {
+            if (armed[s] < 0) continue;
+            while (!mbar_try_wait(smem_u32(&full[s]), static_cast<uint32_t>(armed[s])) &&
+                   globaltimer_ns() - t0 < HILO_WAIT_LIMIT_NS / 4) {
+            }
+          }
+        } else {
+          while (globaltimer_ns() - t0 < 50000ull) {
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && leader) {
+      // ---------------- MMA issuer (even CTA)
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true;
+      for (int t = cid; t < sc.total && ok; t += ncl) {
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, err, DEV_TIMEOUT_GEMM + 256 * 2)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * PN);
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag, err, DEV_TIMEOUT_GEMM + 256 * 3)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_base = smem_u32(smem + stage * STAGE_BYTES);
+          const uint32_t b_base = a_base + HALF_BYTES;
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            const uint64_t ad = sw128_desc(a_base + k * 32, 16, 1024);
+            const uint64_t bd = sw128_desc(b_base + k * 32, 16, 1024);
+            umma_f16_pair(d_tmem, ad, bd, p.idesc, (kb | k) != 0 ? 1u : 0u);
+          }
+          umma_commit_pair(&empty[stage], 0x3);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit_pair(&tfull[acc], 0x3);
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1u;
+      }
+      umma_commit_pair(drain, 0x1);
+      const uint64_t t0 = globaltimer_ns();
+      while (!mbar_try_wait(smem_u32(drain), 0u)) {
+        if (globaltimer_ns() - t0 > HILO_WAIT_LIMIT_NS) {
+          atomicExch(err, DEV_TIMEOUT_GEMM + 256 * 4);
+          break;
+        }
+      }
+    }
+  } else {
+    // ---------------- epilogue (warps 2..5 -> TMEM lane quarters 2,3,0,1), both CTAs
+    const int q = warp & 3;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int t = cid; t < sc.total; t += ncl) {
+      const Tile tl = sc.get(p, t);
+      if (!mbar_wait_warp(&tfull[acc], acc_phase, abort_flag, err, DEV_TIMEOUT_GEMM + 256 * 5)) break;
+      tc_fence_after();
+      const int rit = 128 * static_cast<int>(rank) + q * 32 + lane;
+      const int grow = tl.m0 + rit;
+      const bool valid = (tl.m0 - tl.row_base) + rit < tl.rows;
+      const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * PN);
+      const __nv_bfloat16* bias = p.bias[tl.g];
+#pragma unroll 1
+      for (int c = 0; c < PN / 32; ++c) {
+        float v[32];
+        tmem_ld32(taddr + c * 32, v);
+        tmem_ld_wait();
+        if (c == PN / 32 - 1) {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[acc]), 0));
+        }
+        const int col0 = tl.n0 + c * 32;
+        if (!valid || col0 >= p.N) continue;
+        float bv[32];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) bf16x8(__ldg(reinterpret_cast<const uint4*>(bias + col0) + j), bv + 8 * j);
+        if (p.epilogue == EPI_BIAS_RESID_F32) {
+          float4* dst = reinterpret_cast<float4*>(static_cast<float*>(p.out) +
+                                                  static_cast<long long>(grow) * p.N + col0);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            float4 r = dst[j];
+            r.x += v[4 * j] + bv[4 * j];
+            r.y += v[4 * j + 1] + bv[4 * j + 1];
+            r.z += v[4 * j + 2] + bv[4 * j + 2];
+            r.w += v[4 * j + 3] + bv[4 * j + 3];
+            dst[j] = r;
+          }
+        } else {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] += bv[i];
+          uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(p.out) +
+                                                static_cast<long long>(grow) * p.N + col0);
+          if (p.epilogue == EPI_BIAS_GELU_F16) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = gelu_tanh(v[i]);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              uint4 o;
+              o.x = pack_f16x2_sat(v[8 * j], v[8 * j + 1]);
+              o.y = pack_f16x2_sat(v[8 * j + 2], v[8 * j + 3]);
+              o.z = pack_f16x2_sat(v[8 * j + 4], v[8 * j + 5]);
+              o.w = pack_f16x2_sat(v[8 * j + 6], v[8 * j + 7]);
+              dst[j] = o;
+            }
+          } else {
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              uint4 o;
+              o.x = pack_bf16x2(v[8 * j], v[8 * j + 1]);
+              o.y = pack_bf16x2(v[8 * j + 2], v[8 * j + 3]);
+              o.z = pack_bf16x2(v[8 * j + 4], v[8 * j + 5]);
+              o.w = pack_bf16x2(v[8 * j + 6], v[8 * j + 7]);
+              dst[j] = o;
+            }
+          }
+        }
+      }
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1u;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // no remote arrivals / copies into the peer after this point
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, TMEM_COLS);
+  }
+}
+
+}  // namespace
+
+bool gemm_pair_supported(const GemmArgs& a) { return a.K % BK == 0 && a.N % PN == 0; }
+
+cudaError_t launch_gemm_pair(const GemmArgs& a, int num_sms, cudaStream_t st) {
+  if (!gemm_pair_supported(a)) return cudaErrorInvalidValue;
+  CUtensorMap tA, tB0, tB1;
+  if (!encode_tmap_bf16_2d(&tA, a.A, a.K, a.R, a.K, BK, 128)) return cudaErrorInvalidValue;
+  if (!encode_tmap_bf16_2d(&tB0, a.g[0].weight ? a.g[0].weight : a.g[1].weight, a.K, a.N, a.K, BK, 128))
+    return cudaErrorInvalidValue;
+  if (!encode_tmap_bf16_2d(&tB1, a.g[1].weight ? a.g[1].weight : a.g[0].weight, a.K, a.N, a.K, BK, 128))
+    return cudaErrorInvalidValue;
+  Params p;
+  p.N = a.N;
+  p.K = a.K;
+  p.idesc = idesc_kind_f16(PM, PN, 0, 0, a.op_f16 ? 0 : 1);
+  long long upper = 0;
+  for (int g = 0; g < 2; ++g) {
+    p.row_base[g] = a.g[g].row_base;
+    p.rows_static[g] = a.g[g].rows_static;
+    p.rows_dev[g] = a.g[g].rows_dev;
+    p.bias[g] = static_cast<const __nv_bfloat16*>(a.g[g].bias);
+    upper += (a.g[g].rows_cap + PM - 1) / PM;
+  }
+  upper *= a.N / PN;
+  p.epilogue = a.epilogue;
+  p.out = a.out;
+  if (upper <= 0) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(gemm2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  if (e != cudaSuccess) return e;
+  // persistent grid: as many co-resident CTA pairs as the device holds
+  static int max_pairs = 0;
+  if (max_pairs == 0) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * (num_sms / 2), 1, 1);
+    cfg.blockDim = dim3(THREADS, 1, 1);
+    cfg.dynamicSmemBytes = SMEM_BYTES;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = 2;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, gemm2_kernel, &cfg) != cudaSuccess || n <= 0) {
+      cudaGetLastError();
+      n = num_sms / 2;
+    }
+    max_pairs = n;
+  }
+  const long long pairs = upper < max_pairs ? upper : max_pairs;
+  gemm2_kernel<<<static_cast<int>(2 * pairs), THREADS, SMEM_BYTES, st>>>(tA, tB0, tB1, p);
+  return cudaGetLastError();
+}
+
+int gemm2_take_device_error() {
+  int v = 0, z = 0;
+  if (cudaMemcpyFromSymbol(&v, g_gemm2_err, sizeof(int)) != cudaSuccess) return -1;
+  if (v) cudaMemcpyToSymbol(g_gemm2_err, &z, sizeof(int));
+  return v;
+}
+
+}  // namespace hilo

@@ -359,8 +359,10 @@ cudaError_t launch_bn(const GemmArgs& a, int num_sms, cudaStream_t st) {
 
 cudaError_t launch_gemm(const GemmArgs& a, int num_sms, cudaStream_t st) {
   if (a.K % BK != 0 || a.N % 32 != 0) return cudaErrorInvalidValue;
-  // 256-wide tiles keep the MMA below the shared-memory read bandwidth;
-  // 128-wide tiles only where N is so small that 256 would leave SMs idle.
+  // CTA pairs with 256x256 tiles where N allows (half the W traffic per SM);
+  // else one CTA per tile: 256-wide tiles, or 128-wide where N is so small
+  // that 256 would leave SMs idle.
+  if (a.N >= 1024 && gemm_pair_supported(a)) return launch_gemm_pair(a, num_sms, st);
   if (a.N <= 1024) return launch_bn<128>(a, num_sms, st);
   return launch_bn<256>(a, num_sms, st);
 }

@@ -67,6 +67,11 @@ struct GemmArgs {
 cudaError_t launch_gemm(const GemmArgs& a, int num_sms, cudaStream_t st);
 int gemm_take_device_error();
 
+// ---- tcgen05 grouped GEMM on CTA pairs, 256x256 tiles (gemm2_tc.cu)
+bool gemm_pair_supported(const GemmArgs& a);
+cudaError_t launch_gemm_pair(const GemmArgs& a, int num_sms, cudaStream_t st);
+int gemm2_take_device_error();
+
 // ---- tcgen05 joint varlen attention (attn_tc.cu)
 struct AttnArgs {
   const void* qkv;  // bf16 [R, 3d]
