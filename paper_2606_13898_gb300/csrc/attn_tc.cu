@@ -309,10 +309,23 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
 #pragma unroll
       for (int c = 0; c < BKV / 32; ++c) tmem_ld32(tS + c * 32, s + c * 32);
       tmem_ld_wait();
-      float mx = -INFINITY;
+      // row max and (below) row sum with 8 independent partials combined by
+      // a tree, so the reductions do not form one 128-long dependent chain;
+      // only the last key tile of a segment is ragged and needs masking
+      const bool full_tile = valid == BKV;
+      float mx8[8];
 #pragma unroll
-      for (int j = 0; j < BKV; ++j)
-        if (j < valid) mx = fmaxf(mx, s[j]);
+      for (int u = 0; u < 8; ++u) mx8[u] = -INFINITY;
+      if (full_tile) {
+#pragma unroll
+        for (int j = 0; j < BKV; ++j) mx8[j & 7] = fmaxf(mx8[j & 7], s[j]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < BKV; ++j)
+          if (j < valid) mx8[j & 7] = fmaxf(mx8[j & 7], s[j]);
+      }
+      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
       const float m_tile = mx * p.scale_log2;
       bool rescale = false;
       float m_use = m;
@@ -322,13 +335,25 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
         m_use = m_tile;
         rescale = true;
       }
-      float lsum = 0.f;
+      float ls8[8];
 #pragma unroll
-      for (int j = 0; j < BKV; ++j) {
-        const float pj = j < valid ? ex2(fmaf(s[j], p.scale_log2, -m_use)) : 0.f;
-        s[j] = pj;
-        lsum += pj;
+      for (int u = 0; u < 8; ++u) ls8[u] = 0.f;
+      if (full_tile) {
+#pragma unroll
+        for (int j = 0; j < BKV; ++j) {
+          const float pj = ex2(fmaf(s[j], p.scale_log2, -m_use));
+          s[j] = pj;
+          ls8[j & 7] += pj;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < BKV; ++j) {
+          const float pj = j < valid ? ex2(fmaf(s[j], p.scale_log2, -m_use)) : 0.f;
+          s[j] = pj;
+          ls8[j & 7] += pj;
+        }
       }
+      const float lsum = ((ls8[0] + ls8[1]) + (ls8[2] + ls8[3])) + ((ls8[4] + ls8[5]) + (ls8[6] + ls8[7]));
       // ragged key tile: rows past `valid` hold other tokens (or stale data);
       // zero them in V so that the zero-probability columns add exactly 0
       if (i == 0 && valid < BKV) {
