@@ -238,6 +238,137 @@ def run_reference(args):
 
 # --------------------------------------------------------------- GPU arm --
 
+def block_flops(wl, cu) -> float:
+    """Algorithmic FLOPs of one block over the packed rows given by cu_img."""
+    d, T = wl.d, wl.T
+    M = wl.B * T + int(cu[-1])
+    gemm = (24.0 if wl.mlp else 8.0) * M * d * d
+    attn = sum(4.0 * (T + int(cu[b + 1] - cu[b])) ** 2 * d for b in range(wl.B))
+    return gemm + attn
+
+
+def time_configs(H, I, torch, stream, steps: int):
+    """Hot path, compressed block and dense block of each workload configuration.
+
+    Returns a dict keyed by workload name: hot-path ms (score -> split -> pack
+    -> block(s) -> unpack), block ms, image-tokens/s over the full grids, block
+    TFLOP/s, and the dense block (every grid token a row, same kernels). The
+    denoising loop runs its 28 steps of 8 blocks once and is compared with a
+    dense 8-block stack per step.
+    """
+    res = {}
+
+    def ev():
+        return torch.cuda.Event(enable_timing=True)
+
+    def shape_of(wl):
+        return H.Shape(B=wl.B, H=wl.H, W=wl.W, d=wl.d, T=wl.T, heads=wl.heads, mlp=int(wl.mlp), levels=wl.levels)
+
+    def inputs(b):
+        return (H.bf16_from_bits(b.x), H.bf16_from_bits(b.text), torch.from_numpy(b.mask).cuda(),
+                torch.from_numpy(b.k_keep).cuda(), torch.from_numpy(b.k_mid).cuda())
+
+    for wl in (I.tiny_layer(), I.block_64_batch4(), I.block_128_two_level()):
+        b = I.make_batch(wl)
+        dw = H.DeviceWeights.from_host(I.make_weights(wl.d, wl.mlp, seed=I.weight_seed(wl)))
+        sh = shape_of(wl)
+        hp = H.HotPath(sh, [dw])
+        x, t, m, kk, km = inputs(b)
+        for _ in range(3):
+            hp.run(x, t, m, kk, km)
+        torch.cuda.synchronize()
+        a0, a1, b0, b1 = ev(), ev(), ev(), ev()
+        marks = [(ev(), ev()) for _ in range(steps)]
+        a0.record(stream)
+        for i in range(steps):
+            H.hilo_score(sh, x, hp.score)
+            H.hilo_split(sh, hp.score, m, kk, km, hp.split)
+            H.hilo_pack(sh, x, hp.split, hp.packed, hp.cap)
+            marks[i][0].record(stream)
+            hp.blocks(t, hp.packed, H.HILO_BF16)
+            marks[i][1].record(stream)
+            H.hilo_unpack(sh, hp.out_img, hp.split, hp.y)
+        a1.record(stream)
+        torch.cuda.synchronize()
+        hot = a0.elapsed_time(a1) / steps
+        blk = sum(e0.elapsed_time(e1) for e0, e1 in marks) / steps
+        cu = hp.split.cu_img.cpu().numpy()
+        n_img = wl.B * wl.N
+        cu_dense = torch.arange(wl.B + 1, dtype=torch.int32, device="cuda") * wl.N
+        xr = x.view(wl.B * wl.N, wl.d)
+        for _ in range(3):
+            H.hilo_block_forward(sh, dw, cu_dense, hp.cap, t, xr, H.HILO_BF16, hp.out, hp.ws, hp.ws_bytes)
+        torch.cuda.synchronize()
+        b0.record(stream)
+        for _ in range(steps):
+            H.hilo_block_forward(sh, dw, cu_dense, hp.cap, t, xr, H.HILO_BF16, hp.out, hp.ws, hp.ws_bytes)
+        b1.record(stream)
+        torch.cuda.synchronize()
+        dense = b0.elapsed_time(b1) / steps
+        H.hilo_sync_status()
+        res[wl.name] = {"hot_path_ms": hot, "block_ms": blk, "image_tokens_per_s": n_img / (hot * 1e-3),
+                        "block_tflops": block_flops(wl, cu) / (blk * 1e-3) / 1e12,
+                        "packed_image_rows": cu.tolist()[1:] if wl.B > 1 else int(cu[-1]),
+                        "dense_block_ms": dense,
+                        "dense_block_tflops": block_flops(wl, cu_dense.cpu().numpy()) / (dense * 1e-3) / 1e12,
+                        "block_speedup_vs_dense": dense / blk}
+        del hp, dw
+        torch.cuda.empty_cache()
+
+    # denoising loop: 8 blocks x 28 steps, latents updated in place
+    wl = I.denoise_loop()
+    b = I.make_batch(wl)
+    dws = [H.DeviceWeights.from_host(I.make_weights(wl.d, wl.mlp, seed=I.weight_seed(wl, i))) for i in range(8)]
+    sh = shape_of(wl)
+    hp = H.HotPath(sh, dws)
+    x, t, m, kk, km = inputs(b)
+
+    def loop(n_steps):
+        for _ in range(n_steps):
+            H.hilo_score(sh, x, hp.score)
+            H.hilo_split(sh, hp.score, m, kk, km, hp.split)
+            H.hilo_pack(sh, x, hp.split, hp.packed, hp.cap)
+            hp.blocks(t, hp.packed, H.HILO_BF16)
+            H.hilo_unpack_update(sh, hp.out_img, hp.split, x, 0.035)
+
+    loop(2)
+    x.copy_(H.bf16_from_bits(b.x))
+    torch.cuda.synchronize()
+    a0, a1 = ev(), ev()
+    a0.record(stream)
+    loop(28)
+    a1.record(stream)
+    torch.cuda.synchronize()
+    total = a0.elapsed_time(a1)
+    cu_dense = torch.arange(2, dtype=torch.int32, device="cuda") * wl.N
+    xr = x.view(wl.N, wl.d)
+
+    def dense_step():
+        for i, dw in enumerate(dws):
+            if i == 0:
+                H.hilo_block_forward(sh, dw, cu_dense, hp.cap, t, xr, H.HILO_BF16, hp.out, hp.ws, hp.ws_bytes)
+            else:
+                H.hilo_block_forward(sh, dw, cu_dense, hp.cap, hp.out, hp.out_img, H.HILO_F32, hp.out, hp.ws,
+                                     hp.ws_bytes)
+
+    dense_step()
+    torch.cuda.synchronize()
+    a0.record(stream)
+    for _ in range(5):
+        dense_step()
+    a1.record(stream)
+    torch.cuda.synchronize()
+    dense_step_ms = a0.elapsed_time(a1) / 5
+    H.hilo_sync_status()
+    res[wl.name] = {"total_ms_28_steps": total, "ms_per_step": total / 28,
+                    "image_tokens_per_s": wl.N * 28 / (total * 1e-3),
+                    "dense_8_block_ms_per_step": dense_step_ms, "dense_total_ms_28_steps": dense_step_ms * 28,
+                    "speedup_vs_dense": dense_step_ms * 28 / total}
+    del hp, dws
+    torch.cuda.empty_cache()
+    return res
+
+
 def run_hilo(args):
     import torch
     import torch.distributed as dist
@@ -412,6 +543,8 @@ def run_hilo(args):
             Lr = int(hp.split.cu_img[-1].item())
             sweep[r] = {"hot_path_ms": ms_r, "image_tokens_per_s": N / (ms_r * 1e-3), "packed_image_rows": Lr}
         extras["sweep"] = sweep
+        if world == 1:
+            extras["configs"] = time_configs(H, I, torch, stream, steps=20)
         # dense block: every grid token is its own row, no score/split/pack/unpack
         cu_dense = torch.arange(wl.B + 1, dtype=torch.int32, device="cuda") * wl.N
         x_rows = x.view(wl.B * wl.N, d)
