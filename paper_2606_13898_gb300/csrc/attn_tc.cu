@@ -89,6 +89,8 @@ template <int HD>
 __global__ void __launch_bounds__(ATTN_THREADS, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm, const AttnParams p) {
   using C = Cfg<HD>;
+  pdl_trigger();
+  pdl_wait();  // cu_img and q/k/v are written by the previous kernels
   // ---- work item: (image, head, query-tile pair)
   const int item = blockIdx.x;
   const int b = item / (p.heads * p.pairs_max);
@@ -460,8 +462,7 @@ cudaError_t launch_hd(const AttnArgs& a, const AttnParams& p, int grid, cudaStre
   cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Cfg<HD>::SMEM_BYTES);
   if (e != cudaSuccess) return e;
-  attn_kernel<HD><<<grid, ATTN_THREADS, Cfg<HD>::SMEM_BYTES, st>>>(tm, p);
-  return cudaGetLastError();
+  return launch_pdl(attn_kernel<HD>, dim3(grid), dim3(ATTN_THREADS), Cfg<HD>::SMEM_BYTES, st, tm, p);
 }
 
 }  // namespace

@@ -37,6 +37,8 @@ constexpr int SCORE_MAX_ITERS = 4;  // d <= 4096: at most 4 groups of 8 per thre
 __global__ void __launch_bounds__(SCORE_THREADS) score_kernel(const __nv_bfloat16* __restrict__ x,
                                                               float* __restrict__ s, int B, int H,
                                                               int W, int d) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float part[4][SCORE_THREADS];
   const int j = threadIdx.x;
   const int lane = j & 31;
@@ -260,6 +262,8 @@ __global__ void __launch_bounds__(SPLIT_THREADS) split_select_kernel(
     const float* __restrict__ score, const uint8_t* __restrict__ mask,
     const int32_t* __restrict__ k_keep, const int32_t* __restrict__ k_mid, uint8_t* labels_out,
     int32_t* counts, int H, int W, int levels) {
+  pdl_trigger();
+  pdl_wait();
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ SelectShared sh;
   const int N = H * W;
@@ -330,6 +334,8 @@ __global__ void __launch_bounds__(SPLIT_THREADS) split_select_kernel(
 __global__ void __launch_bounds__(SPLIT_THREADS) split_compact_kernel(
     const uint8_t* __restrict__ labels, const int32_t* __restrict__ counts, int32_t* cu_img,
     int32_t* row_src, int32_t* tok_row, int H, int W, int levels) {
+  pdl_trigger();
+  pdl_wait();
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __shared__ int warp_tot[32];
   const int N = H * W;
@@ -431,6 +437,8 @@ __global__ void __launch_bounds__(256) pack_kernel(const __nv_bfloat16* __restri
                                                    const int32_t* __restrict__ cu_img,
                                                    __nv_bfloat16* __restrict__ packed, int B,
                                                    int H, int W, int d, int cap) {
+  pdl_trigger();
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const int N = H * W;
   const int G = d >> 3;
@@ -509,6 +517,8 @@ __global__ void __launch_bounds__(256) unpack_kernel(const float* __restrict__ o
                                                      const int32_t* __restrict__ tok_row,
                                                      float* __restrict__ y, long long ntok,
                                                      int d) {
+  pdl_trigger();
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const long long wstep = static_cast<long long>(gridDim.x) * (blockDim.x >> 5);
   for (long long t = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -524,6 +534,8 @@ __global__ void __launch_bounds__(256) unpack_update_kernel(const float* __restr
                                                             const int32_t* __restrict__ tok_row,
                                                             __nv_bfloat16* __restrict__ x,
                                                             long long ntok, int d, float alpha) {
+  pdl_trigger();
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const long long wstep = static_cast<long long>(gridDim.x) * (blockDim.x >> 5);
   for (long long t = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
@@ -576,6 +588,8 @@ __global__ void __launch_bounds__(LN_THREADS) layernorm_kernel(const void* __res
                                                                uint16_t* __restrict__ ln, int ln_f16,
                                                                const int32_t* __restrict__ cu_img,
                                                                int B, int n_txt, int d) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float red[LN_THREADS / 32];
   const int rows = n_txt + cu_img[B];
   const float inv_d = 1.0f / static_cast<float>(d);
@@ -645,6 +659,8 @@ __global__ void __launch_bounds__(LN_THREADS) layernorm_kernel(const void* __res
 
 __global__ void __launch_bounds__(256) bf16_to_f16_kernel(const uint4* __restrict__ src,
                                                           uint4* __restrict__ dst, long long n8) {
+  pdl_trigger();
+  pdl_wait();
   for (long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; i < n8;
        i += static_cast<long long>(gridDim.x) * blockDim.x) {
     float f[8];
@@ -671,9 +687,8 @@ static int grid_for(long long work_items, int per_block, int num_sms, int blocks
 cudaError_t launch_score(const void* x, float* s, int B, int H, int W, int d, int num_sms,
                          cudaStream_t st) {
   const long long nwin = static_cast<long long>(B) * (H / 2) * (W / 2);
-  score_kernel<<<grid_for(nwin, 1, num_sms, 16), SCORE_THREADS, 0, st>>>(
-      static_cast<const __nv_bfloat16*>(x), s, B, H, W, d);
-  return cudaGetLastError();
+  return launch_pdl(score_kernel, dim3(grid_for(nwin, 1, num_sms, 16)), dim3(SCORE_THREADS), 0, st,
+                    static_cast<const __nv_bfloat16*>(x), s, B, H, W, d);
 }
 
 size_t split_select_smem(int N) { return static_cast<size_t>(N) * 7; }
@@ -692,59 +707,53 @@ cudaError_t launch_split(const float* score, const uint8_t* mask, const int32_t*
   e = cudaFuncSetAttribute(split_compact_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            static_cast<int>(sm2));
   if (e != cudaSuccess) return e;
-  split_select_kernel<<<B, SPLIT_THREADS, sm1, st>>>(score, mask, k_keep, k_mid, labels, counts,
-                                                     H, W, levels);
-  e = cudaGetLastError();
+  e = launch_pdl(split_select_kernel, dim3(B), dim3(SPLIT_THREADS), sm1, st, score, mask, k_keep,
+                 k_mid, labels, counts, H, W, levels);
   if (e != cudaSuccess) return e;
-  split_compact_kernel<<<B, SPLIT_THREADS, sm2, st>>>(labels, counts, cu_img, row_src, tok_row, H,
-                                                      W, levels);
-  return cudaGetLastError();
+  return launch_pdl(split_compact_kernel, dim3(B), dim3(SPLIT_THREADS), sm2, st,
+                    static_cast<const uint8_t*>(labels), static_cast<const int32_t*>(counts), cu_img,
+                    row_src, tok_row, H, W, levels);
 }
 
 cudaError_t launch_pack(const void* x, const uint8_t* labels, const int32_t* row_src,
                         const int32_t* counts, const int32_t* cu_img, void* packed, int B, int H,
                         int W, int d, int cap, int num_sms, cudaStream_t st) {
-  pack_kernel<<<grid_for(cap, 8, num_sms, 8), 256, 0, st>>>(
-      static_cast<const __nv_bfloat16*>(x), labels, row_src, counts, cu_img,
-      static_cast<__nv_bfloat16*>(packed), B, H, W, d, cap);
-  return cudaGetLastError();
+  return launch_pdl(pack_kernel, dim3(grid_for(cap, 8, num_sms, 8)), dim3(256), 0, st,
+                    static_cast<const __nv_bfloat16*>(x), labels, row_src, counts, cu_img,
+                    static_cast<__nv_bfloat16*>(packed), B, H, W, d, cap);
 }
 
 cudaError_t launch_unpack(const float* out_img, const int32_t* tok_row, float* y, long long ntok,
                           int d, int num_sms, cudaStream_t st) {
-  unpack_kernel<<<grid_for(ntok, 8, num_sms, 8), 256, 0, st>>>(out_img, tok_row, y, ntok, d);
-  return cudaGetLastError();
+  return launch_pdl(unpack_kernel, dim3(grid_for(ntok, 8, num_sms, 8)), dim3(256), 0, st, out_img,
+                    tok_row, y, ntok, d);
 }
 
 cudaError_t launch_unpack_update(const float* out_img, const int32_t* tok_row, void* x,
                                  long long ntok, int d, float alpha, int num_sms,
                                  cudaStream_t st) {
-  unpack_update_kernel<<<grid_for(ntok, 8, num_sms, 8), 256, 0, st>>>(
-      out_img, tok_row, static_cast<__nv_bfloat16*>(x), ntok, d, alpha);
-  return cudaGetLastError();
+  return launch_pdl(unpack_update_kernel, dim3(grid_for(ntok, 8, num_sms, 8)), dim3(256), 0, st,
+                    out_img, tok_row, static_cast<__nv_bfloat16*>(x), ntok, d, alpha);
 }
 
 cudaError_t launch_bf16_to_f16(const void* src, void* dst, long long n, int num_sms,
                                cudaStream_t st) {
   if (n % 8) return cudaErrorInvalidValue;
   const long long n8 = n / 8;
-  bf16_to_f16_kernel<<<grid_for(n8, 256, num_sms, 8), 256, 0, st>>>(
-      static_cast<const uint4*>(src), static_cast<uint4*>(dst), n8);
-  return cudaGetLastError();
+  return launch_pdl(bf16_to_f16_kernel, dim3(grid_for(n8, 256, num_sms, 8)), dim3(256), 0, st,
+                    static_cast<const uint4*>(src), static_cast<uint4*>(dst), n8);
 }
 
 cudaError_t launch_layernorm(const void* in_txt, const void* in_img, int in_f32, float* resid,
                              void* ln, int ln_f16, const int32_t* cu_img, int B, int n_txt,
                              int cap, int d, int num_sms, cudaStream_t st) {
-  const int grid = grid_for(static_cast<long long>(n_txt) + cap, 1, num_sms, 16);
+  const dim3 grid(grid_for(static_cast<long long>(n_txt) + cap, 1, num_sms, 16));
   uint16_t* lo = static_cast<uint16_t*>(ln);
-  const int nch = (d + 511) / 512;
-#define HILO_LN_CASE(NC)                                                                        \
-  case NC:                                                                                      \
-    layernorm_kernel<NC><<<grid, LN_THREADS, 0, st>>>(in_txt, in_img, in_f32, resid, lo, ln_f16, \
-                                                      cu_img, B, n_txt, d);                      \
-    break;
-  switch (nch) {
+  switch ((d + 511) / 512) {
+#define HILO_LN_CASE(NC)                                                                      \
+  case NC:                                                                                    \
+    return launch_pdl(layernorm_kernel<NC>, grid, dim3(LN_THREADS), 0, st, in_txt, in_img, in_f32, \
+                      resid, lo, ln_f16, cu_img, B, n_txt, d);
     HILO_LN_CASE(1)
     HILO_LN_CASE(2)
     HILO_LN_CASE(3)
@@ -753,11 +762,10 @@ cudaError_t launch_layernorm(const void* in_txt, const void* in_img, int in_f32,
     HILO_LN_CASE(6)
     HILO_LN_CASE(7)
     HILO_LN_CASE(8)
+#undef HILO_LN_CASE
     default:
       return cudaErrorInvalidValue;
   }
-#undef HILO_LN_CASE
-  return cudaGetLastError();
 }
 
 }  // namespace hilo

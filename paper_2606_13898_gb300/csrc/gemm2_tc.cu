@@ -112,8 +112,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
   const bool leader = rank == 0;
   const int cid = blockIdx.x >> 1;
   const int ncl = gridDim.x >> 1;
+  pdl_trigger();
   Sched sc;
-  sc.init(p);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -143,6 +143,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const int kblocks = p.K / BK;
+  pdl_wait();  // the row counts and A are written by the previous kernel
+  sc.init(p);
 
   if (warp == 0) {
     if (lane == 0) {
@@ -371,8 +373,8 @@ cudaError_t launch_gemm_pair(const GemmArgs& a, int num_sms, cudaStream_t st) {
     max_pairs = n;
   }
   const long long pairs = upper < max_pairs ? upper : max_pairs;
-  gemm2_kernel<<<static_cast<int>(2 * pairs), THREADS, SMEM_BYTES, st>>>(tA, tB0, tB1, p);
-  return cudaGetLastError();
+  return launch_pdl(gemm2_kernel, dim3(static_cast<int>(2 * pairs)), dim3(THREADS), SMEM_BYTES, st, tA,
+                    tB0, tB1, p);
 }
 
 int gemm2_take_device_error() {

@@ -117,9 +117,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   int* err = &g_gemm_err;
 
+  pdl_trigger();
   const int warp = warp_id(), lane = lane_id();
   Sched<BN> sc;
-  sc.init(p);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -148,6 +148,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const int kblocks = p.K / BK;
+  pdl_wait();  // the row counts and A are written by the previous kernel
+  sc.init(p);
 
   if (warp == 0) {
     if (lane == 0) {
@@ -351,8 +353,8 @@ cudaError_t launch_bn(const GemmArgs& a, int num_sms, cudaStream_t st) {
   cudaError_t e = cudaFuncSetAttribute(gemm_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Cfg::SMEM_BYTES);
   if (e != cudaSuccess) return e;
-  gemm_kernel<BN><<<grid, GEMM_THREADS, Cfg::SMEM_BYTES, st>>>(tA, tB0, tB1, p);
-  return cudaGetLastError();
+  return launch_pdl(gemm_kernel<BN>, dim3(grid), dim3(GEMM_THREADS), Cfg::SMEM_BYTES, st, tA, tB0, tB1,
+                    p);
 }
 
 }  // namespace
