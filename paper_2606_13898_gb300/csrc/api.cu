@@ -295,8 +295,10 @@ int hilo_block_forward(const hilo_shape* shape, const hilo_block_weights* w, con
   const bool in_place_img = in_f32 && BT == 0 && in_img == out;
 
   stage_mark(0, s);
-  cudaError_t e = hilo::launch_layernorm(in_txt, in_img, in_f32, (in_place || in_place_img) ? nullptr : out,
-                                         ln, 0, cu_img, B, BT, cap, d, dev->num_sms, s);
+  // the residual is read from the input by the out-projection epilogue (no
+  // fp32 copy of it is made) unless the input already is the output buffer
+  cudaError_t e = hilo::launch_layernorm(in_txt, in_img, in_f32, nullptr, ln, 0, cu_img, B, BT, cap, d,
+                                         dev->num_sms, s);
   if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: layernorm 1");
   count(1);
   stage_mark(1, s);
@@ -304,6 +306,11 @@ int hilo_block_forward(const hilo_shape* shape, const hilo_block_weights* w, con
   auto gemm = [&](const void* A, int op_f16, int N, int K, int epi, void* o,
                   const void* wt, const void* bt, const void* wi, const void* bi) {
     hilo::GemmArgs g;
+    if (epi == hilo::EPI_BIAS_RESIDIN_F32) {
+      g.resid_src[0] = in_txt;
+      g.resid_src[1] = in_img;
+      g.resid_f32 = in_f32;
+    }
     g.A = A;
     g.op_f16 = op_f16;
     g.R = R;
@@ -337,7 +344,7 @@ int hilo_block_forward(const hilo_shape* shape, const hilo_block_weights* w, con
   count(1);
   stage_mark(3, s);
 
-  e = gemm(attn, 0, d, d, hilo::EPI_BIAS_RESID_F32, out, w->txt.w_o, w->txt.b_o, w->img.w_o, w->img.b_o);
+  e = gemm(attn, 0, d, d, (in_place || in_place_img) ? hilo::EPI_BIAS_RESID_F32 : hilo::EPI_BIAS_RESIDIN_F32, out, w->txt.w_o, w->txt.b_o, w->img.w_o, w->img.b_o);
   if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: out-projection gemm");
   stage_mark(4, s);
   if (shape->mlp) {

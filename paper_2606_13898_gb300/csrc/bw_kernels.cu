@@ -424,11 +424,13 @@ __global__ void __launch_bounds__(SPLIT_THREADS) split_compact_kernel(
 
 // =============================================================== pack =====
 //
-// One warp per packed image row. A kept row is a 16-byte-vector copy; a
-// pooled row sums the window's members of its class in raster order (the
-// first member initialises the sum), divides once with correct rounding and
-// rounds to bf16 (nearest even). Member rows are loaded four at a time and
-// two channel chunks at a time, so up to eight loads are in flight per lane.
+// Four warps per packed image row, each owning every fourth 8-channel chunk
+// of its lanes, so a row needs one memory round trip. A kept row is a
+// 16-byte-vector copy; a pooled row sums the window's members of its class
+// in raster order (the first member initialises the sum), divides once with
+// correct rounding and rounds to bf16 (nearest even).
+
+constexpr int PACK_WARPS_PER_ROW = 4;
 
 __global__ void __launch_bounds__(256) pack_kernel(const __nv_bfloat16* __restrict__ x,
                                                    const uint8_t* __restrict__ labels,
@@ -443,8 +445,12 @@ __global__ void __launch_bounds__(256) pack_kernel(const __nv_bfloat16* __restri
   const int N = H * W;
   const int G = d >> 3;
   const int total = min(cu_img[B], cap);
-  const int wstep = gridDim.x * (blockDim.x >> 5);
-  for (int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < total; r += wstep) {
+  const long long nwarps = static_cast<long long>(gridDim.x) * (blockDim.x >> 5);
+  for (long long gw = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+       gw < static_cast<long long>(total) * PACK_WARPS_PER_ROW; gw += nwarps) {
+    const int r = static_cast<int>(gw / PACK_WARPS_PER_ROW);
+    const int c0 = lane + 32 * static_cast<int>(gw % PACK_WARPS_PER_ROW);
+    constexpr int CSTEP = 32 * PACK_WARPS_PER_ROW;
     int b = 0;
     while (b + 1 < B && cu_img[b + 1] <= r) ++b;
     const int local = r - cu_img[b];
@@ -455,7 +461,7 @@ __global__ void __launch_bounds__(256) pack_kernel(const __nv_bfloat16* __restri
     if (local < nk) {
       const uint4* sp = reinterpret_cast<const uint4*>(xb + static_cast<long long>(src) * d);
 #pragma unroll 4
-      for (int c = lane; c < G; c += 32) dst[c] = __ldg(sp + c);
+      for (int c = c0; c < G; c += CSTEP) dst[c] = __ldg(sp + c);
       continue;
     }
     const int size = local < nk + n2 ? 2 : 4;
@@ -472,7 +478,7 @@ __global__ void __launch_bounds__(256) pack_kernel(const __nv_bfloat16* __restri
     const float cnt = static_cast<float>(__popc(mm));
     const int ngroups = size * size / 4;
 #pragma unroll 2
-    for (int c = lane; c < G; c += 32) {
+    for (int c = c0; c < G; c += CSTEP) {
       float acc[8];
       bool first = true;
       for (int gi = 0; gi < ngroups; ++gi) {
@@ -718,7 +724,8 @@ cudaError_t launch_split(const float* score, const uint8_t* mask, const int32_t*
 cudaError_t launch_pack(const void* x, const uint8_t* labels, const int32_t* row_src,
                         const int32_t* counts, const int32_t* cu_img, void* packed, int B, int H,
                         int W, int d, int cap, int num_sms, cudaStream_t st) {
-  return launch_pdl(pack_kernel, dim3(grid_for(cap, 8, num_sms, 8)), dim3(256), 0, st,
+  return launch_pdl(pack_kernel, dim3(grid_for(static_cast<long long>(cap) * PACK_WARPS_PER_ROW, 8, num_sms, 8)),
+                    dim3(256), 0, st,
                     static_cast<const __nv_bfloat16*>(x), labels, row_src, counts, cu_img,
                     static_cast<__nv_bfloat16*>(packed), B, H, W, d, cap);
 }

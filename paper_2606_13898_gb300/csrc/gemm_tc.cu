@@ -50,6 +50,8 @@ struct GemmParams {
   const __nv_bfloat16* bias[2];
   int epilogue;
   void* out;
+  const void* resid_src[2];
+  int resid_f32;
 };
 
 struct Tile {
@@ -267,18 +269,43 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         float bv[32];
 #pragma unroll
         for (int j = 0; j < 4; ++j) bf16x8(__ldg(reinterpret_cast<const uint4*>(bias + col0) + j), bv + 8 * j);
-        if (p.epilogue == EPI_BIAS_RESID_F32) {
+        if (p.epilogue == EPI_BIAS_RESID_F32 || p.epilogue == EPI_BIAS_RESIDIN_F32) {
           float4* dst = reinterpret_cast<float4*>(static_cast<float*>(p.out) +
                                                   static_cast<long long>(grow) * p.N + col0);
+          float rv[32];
+          if (p.epilogue == EPI_BIAS_RESID_F32) {
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            float4 r = dst[j];
-            r.x += v[4 * j] + bv[4 * j];
-            r.y += v[4 * j + 1] + bv[4 * j + 1];
-            r.z += v[4 * j + 2] + bv[4 * j + 2];
-            r.w += v[4 * j + 3] + bv[4 * j + 3];
-            dst[j] = r;
+            for (int j = 0; j < 8; ++j) {
+              const float4 r = dst[j];
+              rv[4 * j] = r.x;
+              rv[4 * j + 1] = r.y;
+              rv[4 * j + 2] = r.z;
+              rv[4 * j + 3] = r.w;
+            }
+          } else {
+            const long long off = static_cast<long long>(grow - tl.row_base) * p.N + col0;
+            if (p.resid_f32) {
+              const float4* src = reinterpret_cast<const float4*>(static_cast<const float*>(p.resid_src[tl.g]) + off);
+#pragma unroll
+              for (int j = 0; j < 8; ++j) {
+                const float4 r = __ldg(src + j);
+                rv[4 * j] = r.x;
+                rv[4 * j + 1] = r.y;
+                rv[4 * j + 2] = r.z;
+                rv[4 * j + 3] = r.w;
+              }
+            } else {
+              const uint4* src =
+                  reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p.resid_src[tl.g]) + off);
+#pragma unroll
+              for (int j = 0; j < 4; ++j) bf16x8(__ldg(src + j), rv + 8 * j);
+            }
           }
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            dst[j] = make_float4(rv[4 * j] + (v[4 * j] + bv[4 * j]), rv[4 * j + 1] + (v[4 * j + 1] + bv[4 * j + 1]),
+                                 rv[4 * j + 2] + (v[4 * j + 2] + bv[4 * j + 2]),
+                                 rv[4 * j + 3] + (v[4 * j + 3] + bv[4 * j + 3]));
         } else {
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] += bv[i];
@@ -348,6 +375,9 @@ cudaError_t launch_bn(const GemmArgs& a, int num_sms, cudaStream_t st) {
   upper *= (a.N + BN - 1) / BN;
   p.epilogue = a.epilogue;
   p.out = a.out;
+  p.resid_src[0] = a.resid_src[0];
+  p.resid_src[1] = a.resid_src[1];
+  p.resid_f32 = a.resid_f32;
   if (upper <= 0) return cudaSuccess;
   const int grid = static_cast<int>(upper < num_sms ? upper : num_sms);
   cudaError_t e = cudaFuncSetAttribute(gemm_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,

@@ -40,6 +40,7 @@ enum GemmEpilogue : int {
   EPI_BIAS_BF16 = 0,      // out_bf16 = acc + bias
   EPI_BIAS_GELU_F16 = 1,  // out_f16 = gelu_tanh(acc + bias)   (saturating)
   EPI_BIAS_RESID_F32 = 2, // out_f32 += acc + bias
+  EPI_BIAS_RESIDIN_F32 = 3,  // out_f32 = resid_src + acc + bias (resid_src bf16 or fp32, per group)
 };
 
 // Two row groups of the row space share the A operand (one tensor map over
@@ -62,6 +63,10 @@ struct GemmArgs {
   GemmGroupArgs g[2];
   int epilogue;
   void* out;  // bf16 or f32 [R, N]
+  // EPI_BIAS_RESIDIN_F32: the residual rows of group g start at resid_src[g]
+  // (row stride N elements), fp32 when resid_f32 else bf16
+  const void* resid_src[2] = {nullptr, nullptr};
+  int resid_f32 = 0;
 };
 
 cudaError_t launch_gemm(const GemmArgs& a, int num_sms, cudaStream_t st);
