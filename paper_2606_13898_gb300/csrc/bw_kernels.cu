@@ -257,99 +257,13 @@ __device__ void mark_topk(const uint32_t* keys, const uint8_t* cand, uint8_t* se
   __syncthreads();
 }
 
-// Labels and per-image counts. One CTA per image.
-__global__ void __launch_bounds__(SPLIT_THREADS) split_select_kernel(
-    const float* __restrict__ score, const uint8_t* __restrict__ mask,
-    const int32_t* __restrict__ k_keep, const int32_t* __restrict__ k_mid, uint8_t* labels_out,
-    int32_t* counts, int H, int W, int levels) {
-  pdl_trigger();
-  pdl_wait();
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  __shared__ SelectShared sh;
+// Packed rows of one image from its labels (in shared memory): row_src and
+// the token -> row map, kept tokens first (raster order), then 2x2 windows,
+// then 4x4 windows (window-raster order). `base` is the image's first packed
+// row. Called by all threads of the CTA.
+__device__ void compact_image(const uint8_t* lab, int b, int H, int W, int levels, int base, int nk,
+                              int n2, int32_t* row_src, int32_t* tok_row, int* warp_tot) {
   const int N = H * W;
-  const int b = blockIdx.x;
-  uint32_t* keys = reinterpret_cast<uint32_t*>(smem_raw);
-  uint8_t* lab = reinterpret_cast<uint8_t*>(keys + N);
-  uint8_t* cand = lab + N;
-  uint8_t* sel = cand + N;
-  for (int i = threadIdx.x; i < N; i += blockDim.x) {
-    // scores are >= +0, so their IEEE bit patterns order like the values
-    keys[i] = __float_as_uint(score[static_cast<long long>(b) * N + i]);
-    cand[i] = 1;
-  }
-  __syncthreads();
-  const int k = min(max(k_keep[b], 0), N);
-  mark_topk(keys, cand, sel, N, k, sh);
-  for (int i = threadIdx.x; i < N; i += blockDim.x) {
-    const bool keep = sel[i] || mask[static_cast<long long>(b) * N + i];
-    lab[i] = keep ? HILO_LABEL_KEEP : HILO_LABEL_POOL2;
-    cand[i] = keep ? 0 : 1;
-  }
-  __syncthreads();
-  if (levels == 2) {
-    const int km = min(max(k_mid[b], 0), N);
-    mark_topk(keys, cand, sel, N, km, sh);
-    for (int i = threadIdx.x; i < N; i += blockDim.x)
-      if (cand[i]) lab[i] = sel[i] ? HILO_LABEL_POOL2 : HILO_LABEL_POOL4;
-    __syncthreads();
-  }
-  int nk = 0;
-  for (int i = threadIdx.x; i < N; i += blockDim.x) {
-    labels_out[static_cast<long long>(b) * N + i] = lab[i];
-    nk += lab[i] == HILO_LABEL_KEEP ? 1 : 0;
-  }
-  // windows that hold at least one member of their class
-  int n2 = 0, n4 = 0;
-  const int W2 = W >> 1, nw2 = (H >> 1) * W2;
-  for (int w = threadIdx.x; w < nw2; w += blockDim.x) {
-    const int t = (2 * (w / W2)) * W + 2 * (w % W2);
-    n2 += (lab[t] == HILO_LABEL_POOL2 || lab[t + 1] == HILO_LABEL_POOL2 ||
-           lab[t + W] == HILO_LABEL_POOL2 || lab[t + W + 1] == HILO_LABEL_POOL2)
-              ? 1
-              : 0;
-  }
-  if (levels == 2) {
-    const int W4 = W >> 2, nw4 = (H >> 2) * W4;
-    for (int w = threadIdx.x; w < nw4; w += blockDim.x) {
-      const int t = (4 * (w / W4)) * W + 4 * (w % W4);
-      bool any = false;
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < 4; ++j) any |= lab[t + i * W + j] == HILO_LABEL_POOL4;
-      n4 += any ? 1 : 0;
-    }
-  }
-  nk = block_sum(nk, sh.warp_tot);
-  n2 = block_sum(n2, sh.warp_tot);
-  n4 = block_sum(n4, sh.warp_tot);
-  if (threadIdx.x == 0) {
-    counts[3 * b + 0] = nk;
-    counts[3 * b + 1] = n2;
-    counts[3 * b + 2] = n4;
-  }
-}
-
-// Packed offsets, row sources and token -> row map. One CTA per image.
-__global__ void __launch_bounds__(SPLIT_THREADS) split_compact_kernel(
-    const uint8_t* __restrict__ labels, const int32_t* __restrict__ counts, int32_t* cu_img,
-    int32_t* row_src, int32_t* tok_row, int H, int W, int levels) {
-  pdl_trigger();
-  pdl_wait();
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  __shared__ int warp_tot[32];
-  const int N = H * W;
-  const int b = blockIdx.x;
-  uint8_t* lab = smem_raw;
-  for (int i = threadIdx.x; i < N; i += blockDim.x) lab[i] = labels[static_cast<long long>(b) * N + i];
-  int base = 0;
-  for (int j = 0; j < b; ++j) base += counts[3 * j] + counts[3 * j + 1] + counts[3 * j + 2];
-  const int nk = counts[3 * b], n2 = counts[3 * b + 1], n4 = counts[3 * b + 2];
-  if (threadIdx.x == 0) {
-    if (b == 0) cu_img[0] = 0;
-    cu_img[b + 1] = base + nk + n2 + n4;
-  }
-  __syncthreads();
   int32_t* trow = tok_row + static_cast<long long>(b) * N;
   // kept tokens in raster order
   {
@@ -419,7 +333,110 @@ __global__ void __launch_bounds__(SPLIT_THREADS) split_compact_kernel(
       ++r;
     }
   }
-  (void)n4;
+}
+
+// Labels and per-image counts. One CTA per image. With a single image
+// (fused != 0) the same CTA also writes cu_img and the packed rows, as
+// nothing depends on other images.
+__global__ void __launch_bounds__(SPLIT_THREADS) split_select_kernel(
+    const float* __restrict__ score, const uint8_t* __restrict__ mask,
+    const int32_t* __restrict__ k_keep, const int32_t* __restrict__ k_mid, uint8_t* labels_out,
+    int32_t* counts, int H, int W, int levels, int fused, int32_t* cu_img, int32_t* row_src,
+    int32_t* tok_row) {
+  pdl_trigger();
+  pdl_wait();
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  __shared__ SelectShared sh;
+  const int N = H * W;
+  const int b = blockIdx.x;
+  uint32_t* keys = reinterpret_cast<uint32_t*>(smem_raw);
+  uint8_t* lab = reinterpret_cast<uint8_t*>(keys + N);
+  uint8_t* cand = lab + N;
+  uint8_t* sel = cand + N;
+  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+    // scores are >= +0, so their IEEE bit patterns order like the values
+    keys[i] = __float_as_uint(score[static_cast<long long>(b) * N + i]);
+    cand[i] = 1;
+  }
+  __syncthreads();
+  const int k = min(max(k_keep[b], 0), N);
+  mark_topk(keys, cand, sel, N, k, sh);
+  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+    const bool keep = sel[i] || mask[static_cast<long long>(b) * N + i];
+    lab[i] = keep ? HILO_LABEL_KEEP : HILO_LABEL_POOL2;
+    cand[i] = keep ? 0 : 1;
+  }
+  __syncthreads();
+  if (levels == 2) {
+    const int km = min(max(k_mid[b], 0), N);
+    mark_topk(keys, cand, sel, N, km, sh);
+    for (int i = threadIdx.x; i < N; i += blockDim.x)
+      if (cand[i]) lab[i] = sel[i] ? HILO_LABEL_POOL2 : HILO_LABEL_POOL4;
+    __syncthreads();
+  }
+  int nk = 0;
+  for (int i = threadIdx.x; i < N; i += blockDim.x) {
+    labels_out[static_cast<long long>(b) * N + i] = lab[i];
+    nk += lab[i] == HILO_LABEL_KEEP ? 1 : 0;
+  }
+  // windows that hold at least one member of their class
+  int n2 = 0, n4 = 0;
+  const int W2 = W >> 1, nw2 = (H >> 1) * W2;
+  for (int w = threadIdx.x; w < nw2; w += blockDim.x) {
+    const int t = (2 * (w / W2)) * W + 2 * (w % W2);
+    n2 += (lab[t] == HILO_LABEL_POOL2 || lab[t + 1] == HILO_LABEL_POOL2 ||
+           lab[t + W] == HILO_LABEL_POOL2 || lab[t + W + 1] == HILO_LABEL_POOL2)
+              ? 1
+              : 0;
+  }
+  if (levels == 2) {
+    const int W4 = W >> 2, nw4 = (H >> 2) * W4;
+    for (int w = threadIdx.x; w < nw4; w += blockDim.x) {
+      const int t = (4 * (w / W4)) * W + 4 * (w % W4);
+      bool any = false;
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) any |= lab[t + i * W + j] == HILO_LABEL_POOL4;
+      n4 += any ? 1 : 0;
+    }
+  }
+  nk = block_sum(nk, sh.warp_tot);
+  n2 = block_sum(n2, sh.warp_tot);
+  n4 = block_sum(n4, sh.warp_tot);
+  if (threadIdx.x == 0) {
+    counts[3 * b + 0] = nk;
+    counts[3 * b + 1] = n2;
+    counts[3 * b + 2] = n4;
+    if (fused) {
+      cu_img[0] = 0;
+      cu_img[1] = nk + n2 + n4;
+    }
+  }
+  if (fused) compact_image(lab, b, H, W, levels, 0, nk, n2, row_src, tok_row, sh.warp_tot);
+}
+
+// Packed offsets, row sources and token -> row map. One CTA per image.
+__global__ void __launch_bounds__(SPLIT_THREADS) split_compact_kernel(
+    const uint8_t* __restrict__ labels, const int32_t* __restrict__ counts, int32_t* cu_img,
+    int32_t* row_src, int32_t* tok_row, int H, int W, int levels) {
+  pdl_trigger();
+  pdl_wait();
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  __shared__ int warp_tot[32];
+  const int N = H * W;
+  const int b = blockIdx.x;
+  uint8_t* lab = smem_raw;
+  for (int i = threadIdx.x; i < N; i += blockDim.x) lab[i] = labels[static_cast<long long>(b) * N + i];
+  int base = 0;
+  for (int j = 0; j < b; ++j) base += counts[3 * j] + counts[3 * j + 1] + counts[3 * j + 2];
+  const int nk = counts[3 * b], n2 = counts[3 * b + 1], n4 = counts[3 * b + 2];
+  if (threadIdx.x == 0) {
+    if (b == 0) cu_img[0] = 0;
+    cu_img[b + 1] = base + nk + n2 + n4;
+  }
+  __syncthreads();
+  compact_image(lab, b, H, W, levels, base, nk, n2, row_src, tok_row, warp_tot);
 }
 
 // =============================================================== pack =====
@@ -713,9 +730,10 @@ cudaError_t launch_split(const float* score, const uint8_t* mask, const int32_t*
   e = cudaFuncSetAttribute(split_compact_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            static_cast<int>(sm2));
   if (e != cudaSuccess) return e;
+  const int fused = B == 1 ? 1 : 0;
   e = launch_pdl(split_select_kernel, dim3(B), dim3(SPLIT_THREADS), sm1, st, score, mask, k_keep,
-                 k_mid, labels, counts, H, W, levels);
-  if (e != cudaSuccess) return e;
+                 k_mid, labels, counts, H, W, levels, fused, cu_img, row_src, tok_row);
+  if (e != cudaSuccess || fused) return e;
   return launch_pdl(split_compact_kernel, dim3(B), dim3(SPLIT_THREADS), sm2, st,
                     static_cast<const uint8_t*>(labels), static_cast<const int32_t*>(counts), cu_img,
                     row_src, tok_row, H, W, levels);
