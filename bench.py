@@ -136,7 +136,7 @@ def gemm_traffic_per_launch():
     try:
         with open(path) as fh:
             t = json.load(fh)
-        g = t["gemm_kernel"]
+        g = t["gemm2_kernel"]
         if g["source_sha"] != source_sha(g["sources"]):
             return None
         return float(g["bytes_per_launch_mean"])
@@ -519,7 +519,7 @@ def run_hilo(args):
                    "packed_image_rows": L, "block_rows": M, "parallelism": f"replicas x{world}",
                    "l2": "no flush: per-step working set 0.53 GB (bf16 weights 453 MB) > 129 MB L2"},
         "block_ms": t_block, "block_tflops": block_tflops,
-        "roofline": {"bound": "tensor", "kernel": "gemm_kernel (tcgen05)", "achieved": gemm_tflops,
+        "roofline": {"bound": "tensor", "kernel": "gemm2_kernel (tcgen05 cta_group::2)", "achieved": gemm_tflops,
                      "peak": bf16_peak, "unit": "TFLOP/s", "frac": gemm_tflops / bf16_peak,
                      "traffic": traffic, "peak_source": f"{peak_src} bf16 dense (burst)",
                      "algorithmic": f"24*M*d^2 FLOP per step over 4 launches, M={M} rows",

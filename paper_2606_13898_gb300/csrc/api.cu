@@ -137,18 +137,30 @@ static EncodeTiledFn encode_fn() {
   return fn;
 }
 
-bool encode_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
-                         uint64_t row_stride_elems, uint32_t box_inner, uint32_t box_outer) {
+bool encode_tmap_2d(CUtensorMap* map, TmapType type, const void* base, uint64_t inner, uint64_t outer,
+                    uint64_t row_stride_elems, uint32_t box_inner, uint32_t box_outer) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
+  CUtensorMapDataType dt = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  uint64_t esize = 2;
+  if (type == TMAP_F16) dt = CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
+  if (type == TMAP_F32) {
+    dt = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
+    esize = 4;
+  }
   cuuint64_t dims[2] = {inner, outer};
-  cuuint64_t strides[1] = {row_stride_elems * 2};
+  cuuint64_t strides[1] = {row_stride_elems * esize};
   cuuint32_t box[2] = {box_inner, box_outer};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
-                  estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = fn(map, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+bool encode_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+                         uint64_t row_stride_elems, uint32_t box_inner, uint32_t box_outer) {
+  return encode_tmap_2d(map, TMAP_BF16, base, inner, outer, row_stride_elems, box_inner, box_outer);
 }
 
 // Sets the calling thread's hilo_last_error() text and returns `status`

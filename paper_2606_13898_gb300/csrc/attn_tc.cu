@@ -87,7 +87,7 @@ __device__ __forceinline__ void seq_tile(const AttnParams& p, int b, int L, int 
 
 template <int HD>
 __global__ void __launch_bounds__(ATTN_THREADS, 1)
-    attn_kernel(const __grid_constant__ CUtensorMap tm, const AttnParams p) {
+    attn_kernel(const __grid_constant__ CUtensorMap tm, const __grid_constant__ AttnParams p) {
   using C = Cfg<HD>;
   pdl_trigger();
   pdl_wait();  // cu_img and q/k/v are written by the previous kernels
@@ -100,11 +100,13 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
   const int nkv = p.qt_txt + (L + BKV - 1) / BKV;  // also the number of query tiles
   if (2 * pair >= nkv) return;                     // beyond this image's compressed length
   const bool has1 = 2 * pair + 1 < nkv;
-  int q_row0[2], q_valid[2];
-  seq_tile(p, b, L, 2 * pair, q_row0[0], q_valid[0]);
-  q_row0[1] = q_row0[0];
-  q_valid[1] = 0;
-  if (has1) seq_tile(p, b, L, 2 * pair + 1, q_row0[1], q_valid[1]);
+  // the two query tiles (scalars: a runtime-indexed array would live in
+  // local memory)
+  int q_row0_0, q_valid_0, q_row0_1, q_valid_1;
+  seq_tile(p, b, L, 2 * pair, q_row0_0, q_valid_0);
+  q_row0_1 = q_row0_0;
+  q_valid_1 = 0;
+  if (has1) seq_tile(p, b, L, 2 * pair + 1, q_row0_1, q_valid_1);
 
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
@@ -156,12 +158,13 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
     if (lane == 0) {
       // ---------------- TMA producer
       tma_prefetch_desc(&tm);
-      int armed_k[2] = {-1, -1}, armed_v[2] = {-1, -1};
+      // per stage (bit st): armed at least once, and the parity of the last arming
+      uint32_t armed_k = 0, par_k = 0, armed_v = 0, par_v = 0;
       mbar_arrive_expect_tx(q_full, (has1 ? 2 : 1) * C::TILE_BYTES);
 #pragma unroll
       for (int j = 0; j < C::NBOX; ++j) {
-        tma_load_2d(sQ(0) + j * BOX_BYTES, &tm, q_full, h * HD + 64 * j, q_row0[0]);
-        if (has1) tma_load_2d(sQ(1) + j * BOX_BYTES, &tm, q_full, h * HD + 64 * j, q_row0[1]);
+        tma_load_2d(sQ(0) + j * BOX_BYTES, &tm, q_full, h * HD + 64 * j, q_row0_0);
+        if (has1) tma_load_2d(sQ(1) + j * BOX_BYTES, &tm, q_full, h * HD + 64 * j, q_row0_1);
       }
       bool ok = true;
       for (int t = 0; t < nkv && ok; ++t) {
@@ -177,7 +180,8 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
 #pragma unroll
         for (int j = 0; j < C::NBOX; ++j)
           tma_load_2d(sK(st) + j * BOX_BYTES, &tm, &k_full[st], p.d + h * HD + 64 * j, row0);
-        armed_k[st] = static_cast<int>(ph);
+        armed_k |= 1u << st;
+        par_k = (par_k & ~(1u << st)) | (ph << st);
         if (!mbar_wait(&v_empty[st], ph ^ 1u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 2)) {
           ok = false;
           break;
@@ -186,7 +190,8 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
 #pragma unroll
         for (int j = 0; j < C::NBOX; ++j)
           tma_load_2d(sV(st) + j * BOX_BYTES, &tm, &v_full[st], 2 * p.d + h * HD + 64 * j, row0);
-        armed_v[st] = static_cast<int>(ph);
+        armed_v |= 1u << st;
+        par_v = (par_v & ~(1u << st)) | (ph << st);
       }
       if (!ok) {
         // wait (bounded) for the bulk copies in flight before the CTA exits
@@ -195,12 +200,12 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
         while (!mbar_try_wait(smem_u32(q_full), 0u) && globaltimer_ns() - t0 < lim) {
         }
         for (int st = 0; st < 2; ++st) {
-          if (armed_k[st] >= 0)
-            while (!mbar_try_wait(smem_u32(&k_full[st]), static_cast<uint32_t>(armed_k[st])) &&
+          if ((armed_k >> st) & 1u)
+            while (!mbar_try_wait(smem_u32(&k_full[st]), (par_k >> st) & 1u) &&
                    globaltimer_ns() - t0 < lim) {
             }
-          if (armed_v[st] >= 0)
-            while (!mbar_try_wait(smem_u32(&v_full[st]), static_cast<uint32_t>(armed_v[st])) &&
+          if ((armed_v >> st) & 1u)
+            while (!mbar_try_wait(smem_u32(&v_full[st]), (par_v >> st) & 1u) &&
                    globaltimer_ns() - t0 < lim) {
             }
         }
@@ -425,13 +430,14 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
                         DEV_TIMEOUT_ATTN + 256 * 14)) {
       tc_fence_after();
       const float inv = 1.0f / l;
-      uint4* dst = reinterpret_cast<uint4*>(p.out + static_cast<long long>(q_row0[i] + row) * p.d + h * HD);
+      const int qr0 = i ? q_row0_1 : q_row0_0, qv = i ? q_valid_1 : q_valid_0;
+      uint4* dst = reinterpret_cast<uint4*>(p.out + static_cast<long long>(qr0 + row) * p.d + h * HD);
 #pragma unroll 1
       for (int c = 0; c < HD / 32; ++c) {
         float o[32];
         tmem_ld32(tO + c * 32, o);
         tmem_ld_wait();
-        if (row < q_valid[i]) {
+        if (row < qv) {
 #pragma unroll
           for (int j = 0; j < 4; ++j) {
             uint4 v;

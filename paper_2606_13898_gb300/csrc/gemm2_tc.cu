@@ -20,6 +20,7 @@
 #include <cuda_runtime.h>
 
 #include "common.cuh"
+#include "gemm_epi.cuh"
 #include "internal.h"
 
 namespace hilo {
@@ -36,7 +37,7 @@ constexpr int HALF_BYTES = 128 * BK * 2;    // 16 KB: one CTA's A or W slice
 constexpr int STAGE_BYTES = 2 * HALF_BYTES; // A + W slices of this CTA
 constexpr int THREADS = 192;
 constexpr uint32_t TMEM_COLS = 512;         // two 128 x 256 fp32 accumulators
-constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EPI_SMEM_BYTES + 1024 + 256;
 
 struct Params {
   int N, K;
@@ -56,51 +57,39 @@ struct Tile {
 };
 
 struct Sched {
-  int mt[2], rows[2], nt, total;
+  // two row groups, kept in scalars (no runtime-indexed arrays, which would
+  // live in local memory)
+  int mt0, mt1, rows0, rows1, nt, total;
   __device__ void init(const Params& p) {
     nt = (p.N + PN - 1) / PN;
-    total = 0;
-#pragma unroll
-    for (int g = 0; g < 2; ++g) {
-      rows[g] = p.rows_dev[g] ? *p.rows_dev[g] : p.rows_static[g];
-      mt[g] = (rows[g] + PM - 1) / PM;
-      total += mt[g] * nt;
-    }
+    rows0 = p.rows_dev[0] ? *p.rows_dev[0] : p.rows_static[0];
+    rows1 = p.rows_dev[1] ? *p.rows_dev[1] : p.rows_static[1];
+    mt0 = (rows0 + PM - 1) / PM;
+    mt1 = (rows1 + PM - 1) / PM;
+    total = (mt0 + mt1) * nt;
   }
   __device__ Tile get(const Params& p, int t) const {
     Tile r;
-    r.g = t < mt[0] * nt ? 0 : 1;
-    if (r.g) t -= mt[0] * nt;
-    const int mtg = mt[r.g];
-    r.m0 = p.row_base[r.g] + (t % mtg) * PM;
+    r.g = t < mt0 * nt ? 0 : 1;
+    if (r.g) t -= mt0 * nt;
+    const int mtg = r.g ? mt1 : mt0;
+    r.row_base = r.g ? p.row_base[1] : p.row_base[0];
+    r.m0 = r.row_base + (t % mtg) * PM;
     r.n0 = (t / mtg) * PN;
-    r.rows = rows[r.g];
-    r.row_base = p.row_base[r.g];
+    r.rows = r.g ? rows1 : rows0;
     return r;
   }
 };
 
-__device__ __forceinline__ float gelu_tanh(float z) {
-  const float k0 = 0.7978845608028654f;  // sqrt(2/pi)
-  return 0.5f * z * (1.0f + tanhf(k0 * (z + 0.044715f * z * z * z)));
-}
-
-__device__ __forceinline__ void bf16x8(const uint4& v, float* f) {
-  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    f[2 * i] = __uint_as_float(w[i] << 16);
-    f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
-  }
-}
-
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     gemm2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
-                 const __grid_constant__ CUtensorMap tmB1, const Params p) {
+                 const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmOut,
+                 const __grid_constant__ Params p) {
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  unsigned char* epi_stage = smem + STAGES * STAGE_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(epi_stage + EPI_SMEM_BYTES);
   uint64_t* empty = full + STAGES;
   uint64_t* tfull = empty + STAGES;
   uint64_t* tempty = tfull + 2;
@@ -153,8 +142,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       // ---------------- TMA producer (both CTAs)
       int stage = 0;
       uint32_t phase = 0;
-      int armed[STAGES];
-      for (int s = 0; s < STAGES; ++s) armed[s] = -1;
+      uint32_t armed = 0, armed_par = 0;  // per stage: armed at least once, parity of the last arming
       bool ok = true;
       for (int t = cid; t < sc.total && ok; t += ncl) {
         const Tile tl = sc.get(p, t);
@@ -169,7 +157,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
           if (leader) mbar_arrive_expect_tx(&full[stage], 2 * STAGE_BYTES);
           tma_load_2d_pair(sa, &tmA, full_cl, kb * BK, tl.m0 + 128 * static_cast<int>(rank));
           tma_load_2d_pair(sa + HALF_BYTES, tb, full_cl, kb * BK, tl.n0 + 128 * static_cast<int>(rank));
-          armed[stage] = static_cast<int>(phase);
+          armed |= 1u << stage;
+          armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1u;
@@ -181,8 +170,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
         const uint64_t t0 = globaltimer_ns();
         if (leader) {
           for (int s = 0; s < STAGES; ++s) {
-            if (armed[s] < 0) continue;
-            while (!mbar_try_wait(smem_u32(&full[s]), static_cast<uint32_t>(armed[s])) &&
+            if (!((armed >> s) & 1u)) continue;
+            while (!mbar_try_wait(smem_u32(&full[s]), (armed_par >> s) & 1u) &&
                    globaltimer_ns() - t0 < HILO_WAIT_LIMIT_NS / 4) {
             }
           }
@@ -241,102 +230,34 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
   } else {
     // ---------------- epilogue (warps 2..5 -> TMEM lane quarters 2,3,0,1), both CTAs
     const int q = warp & 3;
+    unsigned char* stage = epi_stage + q * EPI_WARP_BYTES;
+    int buf = 0;
     int acc = 0;
     uint32_t acc_phase = 0;
+    if (warp == 2 && lane == 0) tma_prefetch_desc(&tmOut);
     for (int t = cid; t < sc.total; t += ncl) {
       const Tile tl = sc.get(p, t);
+      const uint4 bpre = epi_bias_preload<PN>(tl.g ? p.bias[1] : p.bias[0], tl.n0, p.N);
       if (!mbar_wait_warp(&tfull[acc], acc_phase, abort_flag, err, DEV_TIMEOUT_GEMM + 256 * 5)) break;
       tc_fence_after();
-      const int rit = 128 * static_cast<int>(rank) + q * 32 + lane;
-      const int grow = tl.m0 + rit;
-      const bool valid = (tl.m0 - tl.row_base) + rit < tl.rows;
+      const int off = 128 * static_cast<int>(rank) + q * 32;  // slab offset in the pair tile
+      EpiSlab sl;
+      sl.g = tl.g;
+      sl.row0 = tl.m0 + off;
+      sl.nvalid = min(32, max(0, tl.rows - (tl.m0 - tl.row_base) - off));
+      sl.row_base = tl.row_base;
+      sl.n0 = tl.n0;
       const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * PN);
-      const __nv_bfloat16* bias = p.bias[tl.g];
-#pragma unroll 1
-      for (int c = 0; c < PN / 32; ++c) {
-        float v[32];
-        tmem_ld32(taddr + c * 32, v);
-        tmem_ld_wait();
-        if (c == PN / 32 - 1) {
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[acc]), 0));
-        }
-        const int col0 = tl.n0 + c * 32;
-        if (!valid || col0 >= p.N) continue;
-        float bv[32];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) bf16x8(__ldg(reinterpret_cast<const uint4*>(bias + col0) + j), bv + 8 * j);
-        if (p.epilogue == EPI_BIAS_RESID_F32 || p.epilogue == EPI_BIAS_RESIDIN_F32) {
-          float4* dst = reinterpret_cast<float4*>(static_cast<float*>(p.out) +
-                                                  static_cast<long long>(grow) * p.N + col0);
-          float rv[32];
-          if (p.epilogue == EPI_BIAS_RESID_F32) {
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-              const float4 r = dst[j];
-              rv[4 * j] = r.x;
-              rv[4 * j + 1] = r.y;
-              rv[4 * j + 2] = r.z;
-              rv[4 * j + 3] = r.w;
-            }
-          } else {
-            const long long off = static_cast<long long>(grow - tl.row_base) * p.N + col0;
-            if (p.resid_f32) {
-              const float4* src = reinterpret_cast<const float4*>(static_cast<const float*>(p.resid_src[tl.g]) + off);
-#pragma unroll
-              for (int j = 0; j < 8; ++j) {
-                const float4 r = __ldg(src + j);
-                rv[4 * j] = r.x;
-                rv[4 * j + 1] = r.y;
-                rv[4 * j + 2] = r.z;
-                rv[4 * j + 3] = r.w;
-              }
-            } else {
-              const uint4* src =
-                  reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p.resid_src[tl.g]) + off);
-#pragma unroll
-              for (int j = 0; j < 4; ++j) bf16x8(__ldg(src + j), rv + 8 * j);
-            }
-          }
-#pragma unroll
-          for (int j = 0; j < 8; ++j)
-            dst[j] = make_float4(rv[4 * j] + (v[4 * j] + bv[4 * j]), rv[4 * j + 1] + (v[4 * j + 1] + bv[4 * j + 1]),
-                                 rv[4 * j + 2] + (v[4 * j + 2] + bv[4 * j + 2]),
-                                 rv[4 * j + 3] + (v[4 * j + 3] + bv[4 * j + 3]));
-        } else {
-#pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] += bv[i];
-          uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(p.out) +
-                                                static_cast<long long>(grow) * p.N + col0);
-          if (p.epilogue == EPI_BIAS_GELU_F16) {
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = gelu_tanh(v[i]);
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              uint4 o;
-              o.x = pack_f16x2_sat(v[8 * j], v[8 * j + 1]);
-              o.y = pack_f16x2_sat(v[8 * j + 2], v[8 * j + 3]);
-              o.z = pack_f16x2_sat(v[8 * j + 4], v[8 * j + 5]);
-              o.w = pack_f16x2_sat(v[8 * j + 6], v[8 * j + 7]);
-              dst[j] = o;
-            }
-          } else {
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              uint4 o;
-              o.x = pack_bf16x2(v[8 * j], v[8 * j + 1]);
-              o.y = pack_bf16x2(v[8 * j + 2], v[8 * j + 3]);
-              o.z = pack_bf16x2(v[8 * j + 4], v[8 * j + 5]);
-              o.w = pack_bf16x2(v[8 * j + 6], v[8 * j + 7]);
-              dst[j] = o;
-            }
-          }
-        }
-      }
+      const int a = acc;
+      epilogue_warp<PN>(p, &tmOut, taddr, sl, bpre, stage, buf, [&] {
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[a]), 0));
+      });
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1u;
     }
+    epilogue_drain();
   }
 
   tc_fence_before();
@@ -360,6 +281,8 @@ cudaError_t launch_gemm_pair(const GemmArgs& a, int num_sms, cudaStream_t st) {
     return cudaErrorInvalidValue;
   if (!encode_tmap_bf16_2d(&tB1, a.g[1].weight ? a.g[1].weight : a.g[0].weight, a.K, a.N, a.K, BK, 128))
     return cudaErrorInvalidValue;
+  CUtensorMap tOut;
+  if (!encode_epilogue_map(&tOut, a)) return cudaErrorInvalidValue;
   Params p;
   p.N = a.N;
   p.K = a.K;
@@ -404,7 +327,7 @@ cudaError_t launch_gemm_pair(const GemmArgs& a, int num_sms, cudaStream_t st) {
   }
   const long long pairs = upper < max_pairs ? upper : max_pairs;
   return launch_pdl(gemm2_kernel, dim3(static_cast<int>(2 * pairs)), dim3(THREADS), SMEM_BYTES, st, tA,
-                    tB0, tB1, p);
+                    tB0, tB1, tOut, p);
 }
 
 int gemm2_take_device_error() {

@@ -90,7 +90,10 @@ int attn_take_device_error();
 // ---- error text of the calling thread (api.cu)
 int set_error(int status, const char* msg);
 
-// ---- tensor maps (api.cu)
+// ---- tensor maps (api.cu): 2-D, row-major, 128-byte swizzled boxes
+enum TmapType : int { TMAP_BF16 = 0, TMAP_F16 = 1, TMAP_F32 = 2 };
+bool encode_tmap_2d(CUtensorMap* map, TmapType type, const void* base, uint64_t inner, uint64_t outer,
+                    uint64_t row_stride_elems, uint32_t box_inner, uint32_t box_outer);
 bool encode_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
                          uint64_t row_stride_elems, uint32_t box_inner, uint32_t box_outer);
 
