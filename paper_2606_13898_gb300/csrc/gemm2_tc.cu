@@ -38,6 +38,7 @@ constexpr int STAGE_BYTES = 2 * HALF_BYTES; // A + W slices of this CTA
 constexpr int THREADS = 192;
 constexpr uint32_t TMEM_COLS = 512;         // two 128 x 256 fp32 accumulators
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EPI_SMEM_BYTES + 1024 + 256;
+constexpr int SPLIT_MIN_KB = 16;            // shortest K piece of a tile cut along K
 
 struct Params {
   int N, K;
@@ -78,6 +79,57 @@ struct Sched {
     r.n0 = (t / mtg) * PN;
     r.rows = r.g ? rows1 : rows0;
     return r;
+  }
+};
+
+// One unit of a pair's work: k-blocks [k0, k1) of tile t.
+struct Work {
+  int t, k0, k1;
+};
+
+// The work of pair `cid` of `ncl`. Tiles are dealt round-robin, whole, while
+// a full round remains. When the output is accumulated in place (fp32 +=,
+// written by TMA reduce-add) the tiles of the last, partial round are instead
+// cut along K so that every pair gets the same number of k-blocks
+// (stream-K): each piece adds its partial sum to the output, and only the
+// piece that starts at k = 0 adds the bias. Other epilogues deal every tile
+// whole. All roles of the pair walk the same sequence.
+struct WorkIter {
+  int t, t_end, ncl, kb;
+  long long lo, hi;  // this pair's k-block range in the partial round
+  __device__ WorkIter(const Sched& sc, int cid, int ncl_, int kblocks, bool split) {
+    ncl = ncl_;
+    kb = kblocks;
+    const int rem = split && sc.total > ncl ? sc.total % ncl : 0;
+    t_end = sc.total - rem;
+    t = cid;
+    // pieces of at least SPLIT_MIN_KB k-blocks: the partial round goes to
+    // fewer pairs when it is short
+    const long long w = static_cast<long long>(rem) * kblocks;
+    const int np = static_cast<int>(max(1LL, min(static_cast<long long>(ncl), w / SPLIT_MIN_KB)));
+    lo = hi = 0;
+    if (cid < np) {
+      lo = w * cid / np;
+      hi = w * (cid + 1) / np;
+    }
+    lo += static_cast<long long>(t_end) * kblocks;  // in k-blocks of the whole tile sequence
+    hi += static_cast<long long>(t_end) * kblocks;
+  }
+  __device__ bool next(Work& w) {
+    if (t < t_end) {
+      w.t = t;
+      w.k0 = 0;
+      w.k1 = kb;
+      t += ncl;
+      return true;
+    }
+    if (lo >= hi) return false;
+    w.t = static_cast<int>(lo / kb);
+    w.k0 = static_cast<int>(lo % kb);
+    const long long end = min(hi, static_cast<long long>(w.t + 1) * kb);
+    w.k1 = w.k0 + static_cast<int>(end - lo);
+    lo = end;
+    return true;
   }
 };
 
@@ -136,6 +188,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
   const int kblocks = p.K / BK;
   pdl_wait();  // the row counts and A are written by the previous kernel
   sc.init(p);
+  const bool split_k = p.epilogue == EPI_BIAS_RESID_F32;
 
   if (warp == 0) {
     if (lane == 0) {
@@ -144,10 +197,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       uint32_t phase = 0;
       uint32_t armed = 0, armed_par = 0;  // per stage: armed at least once, parity of the last arming
       bool ok = true;
-      for (int t = cid; t < sc.total && ok; t += ncl) {
-        const Tile tl = sc.get(p, t);
+      WorkIter it(sc, cid, ncl, kblocks, split_k);
+      Work w;
+      while (ok && it.next(w)) {
+        const Tile tl = sc.get(p, w.t);
         const CUtensorMap* tb = tl.g ? &tmB1 : &tmB0;
-        for (int kb = 0; kb < kblocks; ++kb) {
+        for (int kb = w.k0; kb < w.k1; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, err, DEV_TIMEOUT_GEMM + 256 * 1)) {
             ok = false;
             break;
@@ -189,11 +244,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       int acc = 0;
       uint32_t acc_phase = 0;
       bool ok = true;
-      for (int t = cid; t < sc.total && ok; t += ncl) {
+      WorkIter it(sc, cid, ncl, kblocks, split_k);
+      Work w;
+      while (ok && it.next(w)) {
         if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, err, DEV_TIMEOUT_GEMM + 256 * 2)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem + static_cast<uint32_t>(acc * PN);
-        for (int kb = 0; kb < kblocks; ++kb) {
+        for (int kb = w.k0; kb < w.k1; ++kb) {
           if (!mbar_wait(&full[stage], phase, abort_flag, err, DEV_TIMEOUT_GEMM + 256 * 3)) {
             ok = false;
             break;
@@ -205,7 +262,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
           for (int k = 0; k < BK / 16; ++k) {
             const uint64_t ad = sw128_desc(a_base + k * 32, 16, 1024);
             const uint64_t bd = sw128_desc(b_base + k * 32, 16, 1024);
-            umma_f16_pair(d_tmem, ad, bd, p.idesc, (kb | k) != 0 ? 1u : 0u);
+            umma_f16_pair(d_tmem, ad, bd, p.idesc, (kb > w.k0 || k > 0) ? 1u : 0u);
           }
           umma_commit_pair(&empty[stage], 0x3);
           if (++stage == STAGES) {
@@ -235,9 +292,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     int acc = 0;
     uint32_t acc_phase = 0;
     if (warp == 2 && lane == 0) tma_prefetch_desc(&tmOut);
-    for (int t = cid; t < sc.total; t += ncl) {
-      const Tile tl = sc.get(p, t);
-      const uint4 bpre = epi_bias_preload<PN>(tl.g ? p.bias[1] : p.bias[0], tl.n0, p.N);
+    WorkIter it(sc, cid, ncl, kblocks, split_k);
+    Work w;
+    while (it.next(w)) {
+      const Tile tl = sc.get(p, w.t);
+      // the bias is added once per tile, by the piece that starts at k = 0
+      const uint4 bpre = w.k0 == 0 ? epi_bias_preload<PN>(tl.g ? p.bias[1] : p.bias[0], tl.n0, p.N)
+                                   : make_uint4(0u, 0u, 0u, 0u);
       if (!mbar_wait_warp(&tfull[acc], acc_phase, abort_flag, err, DEV_TIMEOUT_GEMM + 256 * 5)) break;
       tc_fence_after();
       const int off = 128 * static_cast<int>(rank) + q * 32;  // slab offset in the pair tile

@@ -8,13 +8,14 @@
 // in turn). One lane then hands the box to the TMA engine:
 //   bf16 / fp16 outputs      bulk tensor store
 //   fp32 += (residual in C)  bulk tensor reduce-add, so the old value is
-//                            never loaded by the SM
+//                            never loaded by the SM (and partial sums of a
+//                            tile cut along K can be added independently)
 //   fp32 = residual + ...    bulk tensor store; the residual rows are loaded
 //                            one column chunk ahead of their use
 // so every global write leaves the SM as whole 128-byte lines and the
 // epilogue does not wait on memory latency. A slab that is only partly inside
 // its row group (the ragged last tile of the image rows) is written with
-// per-lane stores of the valid rows instead.
+// per-lane stores (atomic adds for +=) of the valid rows instead.
 #pragma once
 
 #include <cuda_bf16.h>
@@ -236,14 +237,14 @@ __device__ __forceinline__ void epilogue_warp(const P& p, const CUtensorMap* tm_
     } else if (mine) {
       float4* dst = reinterpret_cast<float4*>(static_cast<float*>(out) +
                                               static_cast<long long>(s.row0 + lane) * N + col0);
+      if (inplace) {
+        // atomic: pieces of a tile cut along K may add to the same rows
+        float* d = reinterpret_cast<float*>(dst);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        float4 w = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-        if (inplace) {
-          const float4 r = dst[j];
-          w = make_float4(r.x + w.x, r.y + w.y, r.z + w.z, r.w + w.w);
-        }
-        dst[j] = w;
+        for (int i = 0; i < 32; ++i) atomicAdd(d + i, v[i]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
       }
     }
   }
