@@ -349,3 +349,69 @@ class HotPath:
             else:
                 hilo_block_forward(sh, w, self.split.cu_img, self.cap, self.out, self.out_img, HILO_F32,
                                    self.out, self.ws, self.ws_bytes, stream)
+
+
+# ---------------------------------------------------------------------------
+# A stream of host-resident batches through the hot path
+# ---------------------------------------------------------------------------
+
+
+class PipelinedHotPath:
+    """Runs the hot path over a sequence of host-resident batches with the
+    host->device copy of batch i+1 and the device->host copy of result i-1
+    overlapped with the kernels of batch i.
+
+    Two sets of device input buffers and two device results are used in turn.
+    Transfers run on their own streams: `h2d` for the inputs, `d2h` for the
+    results. Events order them against the compute stream, so that a buffer
+    is rewritten only after its last reader is done. This class only orders
+    copies and calls; every step of the path runs in libhilo's kernels, as
+    in `HotPath.run`.
+    """
+
+    def __init__(self, shape: Shape, weights: list, host_inputs, device="cuda"):
+        self.hp = HotPath(shape, weights, device)
+        self.h2d = torch.cuda.Stream(device=device)
+        self.d2h = torch.cuda.Stream(device=device)
+        self.dev_in = [tuple(torch.empty_like(t, device=device) for t in host_inputs) for _ in range(2)]
+        self.dev_y = [torch.empty_like(self.hp.y) for _ in range(2)]
+        self.in_ready = [torch.cuda.Event() for _ in range(2)]
+        self.in_free = [torch.cuda.Event() for _ in range(2)]
+        self.y_ready = [torch.cuda.Event() for _ in range(2)]
+        self.y_free = [torch.cuda.Event() for _ in range(2)]
+        self.i = 0
+
+    def submit(self, host_inputs, host_y, compute=None) -> None:
+        """Queue one batch: host_inputs = (x, text, mask, k_keep, k_mid) in
+        pinned host memory; host_y receives y (pinned, B x H x W x d fp32)."""
+        compute = compute or torch.cuda.current_stream()
+        b = self.i & 1
+        with torch.cuda.stream(self.h2d):
+            if self.i >= 2:
+                self.h2d.wait_event(self.in_free[b])
+            for d, h in zip(self.dev_in[b], host_inputs):
+                d.copy_(h, non_blocking=True)
+            self.in_ready[b].record(self.h2d)
+        compute.wait_event(self.in_ready[b])
+        if self.i >= 2:
+            compute.wait_event(self.y_free[b])
+        hp, sh = self.hp, self.hp.shape
+        x, text, mask, k_keep, k_mid = self.dev_in[b]
+        hilo_score(sh, x, hp.score, compute)
+        hilo_split(sh, hp.score, mask, k_keep, k_mid, hp.split, None, 0, compute)
+        hilo_pack(sh, x, hp.split, hp.packed, hp.cap, compute)
+        hp.blocks(text, hp.packed, HILO_BF16, compute)
+        self.in_free[b].record(compute)
+        hilo_unpack(sh, hp.out_img, hp.split, self.dev_y[b], compute)
+        self.y_ready[b].record(compute)
+        with torch.cuda.stream(self.d2h):
+            self.d2h.wait_event(self.y_ready[b])
+            host_y.copy_(self.dev_y[b], non_blocking=True)
+            self.y_free[b].record(self.d2h)
+        self.i += 1
+
+    def drain(self, compute=None) -> None:
+        """Make `compute` wait for every queued transfer."""
+        compute = compute or torch.cuda.current_stream()
+        compute.wait_stream(self.h2d)
+        compute.wait_stream(self.d2h)
