@@ -245,7 +245,7 @@ int hilo_split(const hilo_shape* shape, const float* score, const uint8_t* mask,
                                      out->labels, out->row_src, out->counts, out->cu_img,
                                      out->tok_row, shape->B, shape->H, shape->W, shape->levels,
                                      static_cast<cudaStream_t>(stream));
-  if (e == cudaSuccess) count(2);
+  if (e == cudaSuccess) count(shape->B == 1 ? 1 : 2);  // one image: the select kernel also compacts
   return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_split");
 }
 

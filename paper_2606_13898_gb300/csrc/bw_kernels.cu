@@ -151,26 +151,67 @@ __device__ __forceinline__ int block_sum(int v, int* warp_tot) {
 }
 
 struct SelectShared {
-  int hist[256];
+  int hist[2][256];  // radix passes alternate between the two
   int warp_tot[32];
+  int warp_tot3[3][32];
   int sel_digit;
   int sel_k;
 };
 
-// MSB-first radix select over the candidates (cand[i] != 0): the key of the
-// k-th largest candidate (1 <= k <= #candidates) and how many candidates with
-// exactly that key belong to the top k (those with the lowest token ids).
+// Exclusive scans of three ints per thread at once (one pass of barriers).
+__device__ __forceinline__ void block_excl_scan3(int& a, int& b, int& c, int (*wt)[32], int& ta, int& tb,
+                                                 int& tc) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  int v[3] = {a, b, c}, incl[3] = {a, b, c};
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1)
+#pragma unroll
+    for (int q = 0; q < 3; ++q) {
+      const int n = __shfl_up_sync(0xffffffffu, incl[q], off);
+      if (lane >= off) incl[q] += n;
+    }
+  if (lane == 31)
+#pragma unroll
+    for (int q = 0; q < 3; ++q) wt[q][wid] = incl[q];
+  __syncthreads();
+  if (wid < 3) {
+    int t = wt[wid][lane];
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int n = __shfl_up_sync(0xffffffffu, t, off);
+      if (lane >= off) t += n;
+    }
+    wt[wid][lane] = t;
+  }
+  __syncthreads();
+  a = incl[0] - v[0] + (wid > 0 ? wt[0][wid - 1] : 0);
+  b = incl[1] - v[1] + (wid > 0 ? wt[1][wid - 1] : 0);
+  c = incl[2] - v[2] + (wid > 0 ? wt[2][wid - 1] : 0);
+  ta = wt[0][31];
+  tb = wt[1][31];
+  tc = wt[2][31];
+  __syncthreads();
+}
+
+// MSB-first radix select over the candidates (cand[i] != 0, or every key when
+// cand is null): the key of the k-th largest candidate (1 <= k <=
+// #candidates) and how many candidates with exactly that key belong to the
+// top k (those with the lowest token ids). The passes alternate between two
+// histograms, so clearing the next one needs no barrier of its own.
 __device__ void radix_select(const uint32_t* keys, const uint8_t* cand, int N, int k,
                              SelectShared& sh, uint32_t& thr, int& take) {
   uint32_t prefix = 0, pmask = 0;
   int kk = k;
-  for (int shift = 24; shift >= 0; shift -= 8) {
-    for (int i = threadIdx.x; i < 256; i += blockDim.x) sh.hist[i] = 0;
-    __syncthreads();
+  if (threadIdx.x < 256) sh.hist[0][threadIdx.x] = 0;
+  __syncthreads();
+  int h = 0;
+  for (int shift = 24; shift >= 0; shift -= 8, h ^= 1) {
+    int* hist = sh.hist[h];
     for (int i = threadIdx.x; i < N; i += blockDim.x) {
       const uint32_t key = keys[i];
-      if (cand[i] && (key & pmask) == prefix) atomicAdd(&sh.hist[(key >> shift) & 255u], 1);
+      if ((!cand || cand[i]) && (key & pmask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1);
     }
+    if (threadIdx.x >= 768) sh.hist[h ^ 1][threadIdx.x - 768] = 0;
     __syncthreads();
     if (threadIdx.x < 32) {
       const int lane = threadIdx.x;
@@ -178,7 +219,7 @@ __device__ void radix_select(const uint32_t* keys, const uint8_t* cand, int N, i
       int cnt[8], lsum = 0;
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
-        cnt[j] = sh.hist[255 - 8 * lane - j];
+        cnt[j] = hist[255 - 8 * lane - j];
         lsum += cnt[j];
       }
       int incl = lsum;
@@ -203,10 +244,11 @@ __device__ void radix_select(const uint32_t* keys, const uint8_t* cand, int N, i
       }
     }
     __syncthreads();
+    // sel_digit / sel_k are rewritten only after the next pass's barrier,
+    // which every thread reaches after these reads
     prefix |= static_cast<uint32_t>(sh.sel_digit) << shift;
     pmask |= 255u << shift;
     kk = sh.sel_k;
-    __syncthreads();
   }
   thr = prefix;
   take = kk;
@@ -215,8 +257,8 @@ __device__ void radix_select(const uint32_t* keys, const uint8_t* cand, int N, i
 // Marks sel[i] = 1 for the top-k candidates under (key desc, index asc).
 __device__ void mark_topk(const uint32_t* keys, const uint8_t* cand, uint8_t* sel, int N, int k,
                           SelectShared& sh) {
-  int ncand = 0;
-  {
+  int ncand = N;  // cand == nullptr: every key is a candidate
+  if (cand) {
     int c = 0;
     for (int i = threadIdx.x; i < N; i += blockDim.x) c += cand[i] ? 1 : 0;
     ncand = block_sum(c, sh.warp_tot);
@@ -227,7 +269,7 @@ __device__ void mark_topk(const uint32_t* keys, const uint8_t* cand, uint8_t* se
     return;
   }
   if (k >= ncand) {
-    for (int i = threadIdx.x; i < N; i += blockDim.x) sel[i] = cand[i] ? 1 : 0;
+    for (int i = threadIdx.x; i < N; i += blockDim.x) sel[i] = (!cand || cand[i]) ? 1 : 0;
     __syncthreads();
     return;
   }
@@ -239,11 +281,11 @@ __device__ void mark_topk(const uint32_t* keys, const uint8_t* cand, uint8_t* se
   const int i0 = threadIdx.x * chunk;
   const int i1 = min(N, i0 + chunk);
   int eq = 0;
-  for (int i = i0; i < i1; ++i) eq += (cand[i] && keys[i] == thr) ? 1 : 0;
+  for (int i = i0; i < i1; ++i) eq += ((!cand || cand[i]) && keys[i] == thr) ? 1 : 0;
   int rank = block_excl_scan(eq, sh.warp_tot, nullptr);
   for (int i = i0; i < i1; ++i) {
     uint8_t v = 0;
-    if (cand[i]) {
+    if (!cand || cand[i]) {
       const uint32_t key = keys[i];
       if (key > thr) {
         v = 1;
@@ -353,57 +395,64 @@ __global__ void __launch_bounds__(SPLIT_THREADS) split_select_kernel(
   uint8_t* lab = reinterpret_cast<uint8_t*>(keys + N);
   uint8_t* cand = lab + N;
   uint8_t* sel = cand + N;
+  const int k = min(max(k_keep[b], 0), N);
+  const int km = levels == 2 ? min(max(k_mid[b], 0), N) : 0;
+  // the first selection has every token as a candidate, so `cand` holds the
+  // mask until the keep labels are formed
   for (int i = threadIdx.x; i < N; i += blockDim.x) {
     // scores are >= +0, so their IEEE bit patterns order like the values
     keys[i] = __float_as_uint(score[static_cast<long long>(b) * N + i]);
-    cand[i] = 1;
+    cand[i] = mask[static_cast<long long>(b) * N + i];
   }
   __syncthreads();
-  const int k = min(max(k_keep[b], 0), N);
-  mark_topk(keys, cand, sel, N, k, sh);
+  mark_topk(keys, nullptr, sel, N, k, sh);
   for (int i = threadIdx.x; i < N; i += blockDim.x) {
-    const bool keep = sel[i] || mask[static_cast<long long>(b) * N + i];
+    const bool keep = sel[i] || cand[i];
     lab[i] = keep ? HILO_LABEL_KEEP : HILO_LABEL_POOL2;
     cand[i] = keep ? 0 : 1;
   }
   __syncthreads();
   if (levels == 2) {
-    const int km = min(max(k_mid[b], 0), N);
     mark_topk(keys, cand, sel, N, km, sh);
     for (int i = threadIdx.x; i < N; i += blockDim.x)
       if (cand[i]) lab[i] = sel[i] ? HILO_LABEL_POOL2 : HILO_LABEL_POOL4;
     __syncthreads();
   }
-  int nk = 0;
-  for (int i = threadIdx.x; i < N; i += blockDim.x) {
-    labels_out[static_cast<long long>(b) * N + i] = lab[i];
-    nk += lab[i] == HILO_LABEL_KEEP ? 1 : 0;
-  }
-  // windows that hold at least one member of their class
-  int n2 = 0, n4 = 0;
+  // Per thread, a contiguous chunk of tokens, of 2x2 windows and of 4x4
+  // windows: kept tokens, and windows holding at least one member of their
+  // class, are counted, and one three-way block scan gives both the image's
+  // counts and each thread's first packed row.
+  const int tch = (N + blockDim.x - 1) / blockDim.x;
+  const int i0 = min(N, static_cast<int>(threadIdx.x) * tch), i1 = min(N, i0 + tch);
   const int W2 = W >> 1, nw2 = (H >> 1) * W2;
-  for (int w = threadIdx.x; w < nw2; w += blockDim.x) {
+  const int wch = (nw2 + blockDim.x - 1) / blockDim.x;
+  const int w0 = min(nw2, static_cast<int>(threadIdx.x) * wch), w1 = min(nw2, w0 + wch);
+  const int W4 = W >> 2, nw4 = levels == 2 ? (H >> 2) * W4 : 0;
+  const int vch = (nw4 + blockDim.x - 1) / blockDim.x;
+  const int v0 = min(nw4, static_cast<int>(threadIdx.x) * vch), v1 = min(nw4, v0 + vch);
+  auto has2 = [&](int w) {
     const int t = (2 * (w / W2)) * W + 2 * (w % W2);
-    n2 += (lab[t] == HILO_LABEL_POOL2 || lab[t + 1] == HILO_LABEL_POOL2 ||
-           lab[t + W] == HILO_LABEL_POOL2 || lab[t + W + 1] == HILO_LABEL_POOL2)
-              ? 1
-              : 0;
-  }
-  if (levels == 2) {
-    const int W4 = W >> 2, nw4 = (H >> 2) * W4;
-    for (int w = threadIdx.x; w < nw4; w += blockDim.x) {
-      const int t = (4 * (w / W4)) * W + 4 * (w % W4);
-      bool any = false;
+    return lab[t] == HILO_LABEL_POOL2 || lab[t + 1] == HILO_LABEL_POOL2 || lab[t + W] == HILO_LABEL_POOL2 ||
+           lab[t + W + 1] == HILO_LABEL_POOL2;
+  };
+  auto has4 = [&](int v) {
+    const int t = (4 * (v / W4)) * W + 4 * (v % W4);
+    bool any = false;
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
+    for (int i = 0; i < 4; ++i)
 #pragma unroll
-        for (int j = 0; j < 4; ++j) any |= lab[t + i * W + j] == HILO_LABEL_POOL4;
-      n4 += any ? 1 : 0;
-    }
+      for (int j = 0; j < 4; ++j) any |= lab[t + i * W + j] == HILO_LABEL_POOL4;
+    return any;
+  };
+  int rk = 0, r2 = 0, r4 = 0;
+  for (int i = i0; i < i1; ++i) {
+    labels_out[static_cast<long long>(b) * N + i] = lab[i];
+    rk += lab[i] == HILO_LABEL_KEEP ? 1 : 0;
   }
-  nk = block_sum(nk, sh.warp_tot);
-  n2 = block_sum(n2, sh.warp_tot);
-  n4 = block_sum(n4, sh.warp_tot);
+  for (int w = w0; w < w1; ++w) r2 += has2(w) ? 1 : 0;
+  for (int v = v0; v < v1; ++v) r4 += has4(v) ? 1 : 0;
+  int nk, n2, n4;
+  block_excl_scan3(rk, r2, r4, sh.warp_tot3, nk, n2, n4);
   if (threadIdx.x == 0) {
     counts[3 * b + 0] = nk;
     counts[3 * b + 1] = n2;
@@ -413,7 +462,38 @@ __global__ void __launch_bounds__(SPLIT_THREADS) split_select_kernel(
       cu_img[1] = nk + n2 + n4;
     }
   }
-  if (fused) compact_image(lab, b, H, W, levels, 0, nk, n2, row_src, tok_row, sh.warp_tot);
+  if (!fused) return;
+  // packed rows: kept tokens (raster order), then 2x2, then 4x4 windows
+  int32_t* trow = tok_row + static_cast<long long>(b) * N;
+  for (int i = i0; i < i1; ++i)
+    if (lab[i] == HILO_LABEL_KEEP) {
+      row_src[rk] = i;
+      trow[i] = rk;
+      ++rk;
+    }
+  r2 += nk;
+  for (int w = w0; w < w1; ++w) {
+    if (!has2(w)) continue;
+    const int t = (2 * (w / W2)) * W + 2 * (w % W2);
+    row_src[r2] = w;
+    const int mem[4] = {t, t + 1, t + W, t + W + 1};
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (lab[mem[j]] == HILO_LABEL_POOL2) trow[mem[j]] = r2;
+    ++r2;
+  }
+  r4 += nk + n2;
+  for (int v = v0; v < v1; ++v) {
+    if (!has4(v)) continue;
+    const int t = (4 * (v / W4)) * W + 4 * (v % W4);
+    row_src[r4] = v;
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (lab[t + i * W + j] == HILO_LABEL_POOL4) trow[t + i * W + j] = r4;
+    ++r4;
+  }
 }
 
 // Packed offsets, row sources and token -> row map. One CTA per image.

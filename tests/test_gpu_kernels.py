@@ -76,13 +76,15 @@ def check_split(sp, ref, B, N):
     assert np.array_equal(sp.tok_row.cpu().numpy().reshape(B, N), ref.tok_row)
 
 
+@pytest.mark.parametrize("B", [1, 3])
 @pytest.mark.parametrize("levels", [1, 2])
 @pytest.mark.parametrize("seed", range(4))
-def test_split_bitexact_random_ties(H, seed, levels):
+def test_split_bitexact_random_ties(H, seed, levels, B):
+    """B = 1 runs the single-kernel path (selection and compaction in one
+    CTA), B = 3 the two-kernel path with offsets across images."""
     rng = np.random.default_rng(seed)
     Hh, W = [(8, 8), (16, 12), (64, 64), (128, 128)][seed]
     N = Hh * W
-    B = 3
     # coarse scores: many exact ties decided by the token index
     s = (rng.integers(0, 7, size=(B, N)) * 0.25).astype(np.float32)
     mask = (rng.random((B, N)) < 0.2).astype(np.uint8)
@@ -92,15 +94,16 @@ def test_split_bitexact_random_ties(H, seed, levels):
     check_split(sp, O.split(s, mask, kk, km, Hh, W, levels), B, N)
 
 
+@pytest.mark.parametrize("B", [1, 2])
 @pytest.mark.parametrize("case", ["k0", "kN", "all_mask", "no_mask", "all_equal", "wide_range"])
-def test_split_edge_cases(H, case):
+def test_split_edge_cases(H, case, B):
     rng = np.random.default_rng(7)
-    Hh, W, B = 32, 32, 2
+    Hh, W = 32, 32
     N = Hh * W
     s = rng.random((B, N)).astype(np.float32)
     mask = (rng.random((B, N)) < 0.15).astype(np.uint8)
-    kk = np.array([N // 4, 3], dtype=np.int32)
-    km = np.array([N // 3, 0], dtype=np.int32)
+    kk = np.array([N // 4, 3][:B], dtype=np.int32)
+    km = np.array([N // 3, 0][:B], dtype=np.int32)
     if case == "k0":
         kk[:] = 0
     elif case == "kN":
@@ -118,6 +121,21 @@ def test_split_edge_cases(H, case):
     for levels in (1, 2):
         sp = run_split(H, s, mask, kk, km, Hh, W, levels)
         check_split(sp, O.split(s, mask, kk, km, Hh, W, levels), B, N)
+
+
+@pytest.mark.parametrize("levels", [1, 2])
+def test_split_largest_image(H, levels):
+    """The largest image the ABI accepts (32768 tokens): the selection CTA's
+    shared memory is 7 bytes per token, just inside the per-CTA limit."""
+    rng = np.random.default_rng(11 + levels)
+    Hh, W, B = 128, 256, 1
+    N = Hh * W
+    s = (rng.integers(0, 50, size=(B, N)) * 0.125).astype(np.float32)
+    mask = (rng.random((B, N)) < 0.05).astype(np.uint8)
+    kk = np.array([N // 4], dtype=np.int32)
+    km = np.array([N // 4], dtype=np.int32)
+    sp = run_split(H, s, mask, kk, km, Hh, W, levels)
+    check_split(sp, O.split(s, mask, kk, km, Hh, W, levels), B, N)
 
 
 # ------------------------------------------------------------ pack/unpack --
