@@ -37,9 +37,14 @@ namespace {
 
 constexpr int BQ = 128;
 constexpr int BKV = 128;
-constexpr int ATTN_THREADS = 320;
+// Three warpgroups: two softmax warpgroups and one for TMA, MMA and two idle
+// warps. The control warpgroup gives registers to the softmax warpgroups
+// (setmaxnreg); launch_hd checks that the shares fit the launch allocation.
+constexpr int ATTN_THREADS = 384;
 constexpr int PRODUCER_WARP = 8;
 constexpr int MMA_WARP = 9;
+constexpr uint32_t SOFTMAX_REGS = 208;
+constexpr uint32_t CONTROL_REGS = 88;
 constexpr uint32_t ATTN_TMEM_COLS = 512;  // S0 | S1 | O0 | O1
 constexpr int BOX_BYTES = 128 * 128;       // 128 rows x 64 16-bit elements
 constexpr float RESCALE_LOG2 = 8.0f;
@@ -153,8 +158,10 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-
-  if (warp == PRODUCER_WARP) {
+  if (warp >= 8) {
+    // control warpgroup: TMA producer, MMA issuer, two idle warps
+    setmaxnreg_dec<CONTROL_REGS>();
+    if (warp == PRODUCER_WARP) {
     if (lane == 0) {
       // ---------------- TMA producer
       tma_prefetch_desc(&tm);
@@ -293,7 +300,9 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
         }
       }
     }
+    }
   } else {
+    setmaxnreg_inc<SOFTMAX_REGS>();
     // ---------------- softmax: warpgroup i = warps 4i..4i+3, TMEM lane quarter warp % 4
     const int i = warp >> 2;
     const int row = (warp & 3) * 32 + lane;
@@ -468,6 +477,17 @@ cudaError_t launch_hd(const AttnArgs& a, const AttnParams& p, int grid, cudaStre
   cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Cfg<HD>::SMEM_BYTES);
   if (e != cudaSuccess) return e;
+  // the register split must fit what the CTA is launched with, or the
+  // softmax warpgroups' setmaxnreg.inc would wait for registers forever
+  static int regs = -1;
+  if (regs < 0) {
+    cudaFuncAttributes fa;
+    e = cudaFuncGetAttributes(&fa, attn_kernel<HD>);
+    if (e != cudaSuccess) return e;
+    regs = fa.numRegs;
+  }
+  if (static_cast<long long>(regs) * ATTN_THREADS < 256LL * SOFTMAX_REGS + 128LL * CONTROL_REGS)
+    return cudaErrorInvalidConfiguration;
   return launch_pdl(attn_kernel<HD>, dim3(grid), dim3(ATTN_THREADS), Cfg<HD>::SMEM_BYTES, st, tm, p);
 }
 

@@ -367,6 +367,18 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, int a_mn_major, 
 // predecessor's completion and memory (pdl_wait) before its first global
 // memory access; only the prologue (barrier init, TMEM allocation, tensor-map
 // prefetch) runs before that. Both are no-ops without a predecessor.
+// Per-warpgroup register budget (all 128 threads of the warpgroup execute
+// it). inc waits until enough registers were released by dec elsewhere in
+// the CTA, so the shares must add up to the launch's allocation.
+template <uint32_t R>
+__device__ __forceinline__ void setmaxnreg_inc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(R));
+}
+template <uint32_t R>
+__device__ __forceinline__ void setmaxnreg_dec() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(R));
+}
+
 __device__ __forceinline__ void pdl_trigger() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
