@@ -186,6 +186,26 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const int kblocks = p.K / BK;
+  // The weights do not depend on the previous kernel: while it finishes,
+  // pull the first k-blocks of this pair's first weight tile into L2. The
+  // tile is exact when it lies in a group whose row count is static (the
+  // text rows); in the image rows, whose count is read only after the wait,
+  // the column block is a guess, and a wrong one costs only the prefetch.
+  if (warp == 0 && lane == 0) {
+    const int nt = p.N / PN;
+    const int mt0 = p.rows_dev[0] ? 0 : (p.rows_static[0] + PM - 1) / PM;
+    const CUtensorMap* tb;
+    int n;
+    if (cid < mt0 * nt) {
+      tb = &tmB0;
+      n = cid / mt0;
+    } else {
+      tb = &tmB1;
+      n = (cid - mt0 * nt) % nt;
+    }
+    const int y = n * PN + 128 * static_cast<int>(rank);
+    for (int kb = 0; kb < min(kblocks, STAGES); ++kb) tma_prefetch_l2_2d(tb, kb * BK, y);
+  }
   pdl_wait();  // the row counts and A are written by the previous kernel
   sc.init(p);
   const bool split_k = p.epilogue == EPI_BIAS_RESID_F32;
