@@ -129,7 +129,7 @@ __device__ __forceinline__ int block_excl_scan(int v, int* warp_tot, int* total)
   if (lane == 31) warp_tot[wid] = incl;
   __syncthreads();
   if (wid == 0) {
-    int t = warp_tot[lane];
+    int t = lane < static_cast<int>(blockDim.x >> 5) ? warp_tot[lane] : 0;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
       const int n = __shfl_up_sync(0xffffffffu, t, off);
@@ -139,7 +139,7 @@ __device__ __forceinline__ int block_excl_scan(int v, int* warp_tot, int* total)
   }
   __syncthreads();
   const int res = incl - v + (wid > 0 ? warp_tot[wid - 1] : 0);
-  if (total) *total = warp_tot[31];
+  if (total) *total = warp_tot[(blockDim.x >> 5) - 1];
   __syncthreads();
   return res;
 }
@@ -175,7 +175,7 @@ __device__ __forceinline__ void block_excl_scan3(int& a, int& b, int& c, int (*w
     for (int q = 0; q < 3; ++q) wt[q][wid] = incl[q];
   __syncthreads();
   if (wid < 3) {
-    int t = wt[wid][lane];
+    int t = lane < static_cast<int>(blockDim.x >> 5) ? wt[wid][lane] : 0;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
       const int n = __shfl_up_sync(0xffffffffu, t, off);
@@ -187,9 +187,10 @@ __device__ __forceinline__ void block_excl_scan3(int& a, int& b, int& c, int (*w
   a = incl[0] - v[0] + (wid > 0 ? wt[0][wid - 1] : 0);
   b = incl[1] - v[1] + (wid > 0 ? wt[1][wid - 1] : 0);
   c = incl[2] - v[2] + (wid > 0 ? wt[2][wid - 1] : 0);
-  ta = wt[0][31];
-  tb = wt[1][31];
-  tc = wt[2][31];
+  const int lw = (blockDim.x >> 5) - 1;
+  ta = wt[0][lw];
+  tb = wt[1][lw];
+  tc = wt[2][lw];
   __syncthreads();
 }
 
@@ -211,7 +212,7 @@ __device__ void radix_select(const uint32_t* keys, const uint8_t* cand, int N, i
       const uint32_t key = keys[i];
       if ((!cand || cand[i]) && (key & pmask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1);
     }
-    if (threadIdx.x >= 768) sh.hist[h ^ 1][threadIdx.x - 768] = 0;
+    if (threadIdx.x >= blockDim.x - 256) sh.hist[h ^ 1][threadIdx.x - (blockDim.x - 256)] = 0;
     __syncthreads();
     if (threadIdx.x < 32) {
       const int lane = threadIdx.x;
