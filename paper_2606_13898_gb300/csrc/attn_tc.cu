@@ -7,20 +7,26 @@
 // of the row space; queries and keys/values are tiled per range (128 rows per
 // tile, the ragged last tile masked).
 //
-// One CTA per (image, head, pair of 128-query tiles), 320 threads:
-//   warps 0-3   softmax of query tile 0 (one query row per thread)
-//   warps 4-7   softmax of query tile 1
-//   warp 8      TMA: Q tiles once, then K and V tiles (two stages each),
-//               128-byte swizzled boxes of 64 columns
-//   warp 9      MMA: S_i = Q_i K^T into TMEM, O_i += P V into TMEM (V is the
-//               MN-major operand, no transpose pass)
-// The two query tiles ping-pong: while one softmax warpgroup turns S into P,
-// the tensor core works on the other tile (MMA order PV_0(t), S_0(t+1),
-// PV_1(t), S_1(t+1)). Both tiles share the K/V stream. S is read from TMEM
-// once into registers; the output accumulators stay in TMEM for the whole
-// sequence and are rescaled only when a row's running maximum grows by more
-// than 2^8 (until then the probabilities are formed against the older,
-// smaller maximum, so they stay <= 256, well inside bf16 range).
+// One CTA per (image, head, pair of 128-query tiles), 384 threads in three
+// warpgroups:
+//   warps 0-3    softmax of query tile 0 (one query row per thread)
+//   warps 4-7    softmax of query tile 1
+//   warp 8       TMA: Q tiles once, then K and V tiles (two stages each),
+//                128-byte swizzled boxes of 64 columns
+//   warp 9       MMA: S_i = Q_i K^T into TMEM, O_i += P_i V into TMEM
+//   warps 10-11  idle (the third warpgroup gives its registers away)
+// Tensor memory holds S_0 | S_1 | O_0 | O_1 (128 columns each). A softmax
+// warpgroup reads S_i once into registers and writes the probabilities P_i
+// back over the first 64 columns of S_i as packed bf16; the PV product takes
+// P_i from tensor memory (A operand) and V from shared memory (MN-major, no
+// transpose pass). The two query tiles ping-pong on the tensor core (MMA
+// order PV_0(t), S_0(t+1), PV_1(t), S_1(t+1)); S_i(t+1) overwrites P_i(t)
+// only after PV_i(t), in issue order. When a softmax warpgroup sees S_i(t),
+// every earlier MMA has completed, so O_i may be rescaled and P_i written
+// without a further wait. The output accumulators are rescaled only when a
+// row's running maximum grows by more than 2^8 (until then the
+// probabilities are formed against the older, smaller maximum, so they stay
+// <= 256, well inside bf16 range).
 // Every mbarrier wait is bounded (error latched, TMEM freed, CTA returns).
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -43,8 +49,8 @@ constexpr int BKV = 128;
 constexpr int ATTN_THREADS = 384;
 constexpr int PRODUCER_WARP = 8;
 constexpr int MMA_WARP = 9;
-constexpr uint32_t SOFTMAX_REGS = 208;
-constexpr uint32_t CONTROL_REGS = 88;
+constexpr uint32_t SOFTMAX_REGS = 216;
+constexpr uint32_t CONTROL_REGS = 72;
 constexpr uint32_t ATTN_TMEM_COLS = 512;  // S0 | S1 | O0 | O1
 constexpr int BOX_BYTES = 128 * 128;       // 128 rows x 64 16-bit elements
 constexpr float RESCALE_LOG2 = 8.0f;
@@ -53,13 +59,11 @@ template <int HD>
 struct Cfg {
   static constexpr int NBOX = HD / 64;
   static constexpr int TILE_BYTES = NBOX * BOX_BYTES;  // 128 rows x HD
-  static constexpr int P_BYTES = 2 * BOX_BYTES;        // 128 x 128 bf16
-  // Q0 | Q1 | K0 | K1 | V0 | V1 | P
+  // Q0 | Q1 | K0 | K1 | V0 | V1
   static constexpr int OFF_Q = 0;
   static constexpr int OFF_K = 2 * TILE_BYTES;
   static constexpr int OFF_V = 4 * TILE_BYTES;
-  static constexpr int OFF_P = 6 * TILE_BYTES;
-  static constexpr int DATA_BYTES = 6 * TILE_BYTES + P_BYTES;
+  static constexpr int DATA_BYTES = 6 * TILE_BYTES;
   static constexpr int SMEM_BYTES = DATA_BYTES + 1024 + 256;
 };
 
@@ -116,7 +120,6 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  unsigned char* sP = smem + C::OFF_P;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::DATA_BYTES);
   uint64_t* q_full = bars + 0;
   uint64_t* k_full = bars + 1;    // [2]
@@ -223,7 +226,6 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
       // ---------------- MMA issuer
       const uint32_t idesc_s = idesc_bf16(BQ, BKV, 0, 0);
       const uint32_t idesc_o = idesc_bf16(BQ, HD, 0, 1);
-      const uint32_t p_base = smem_u32(sP);
       auto issue_s = [&](int i, int t) {
         const uint32_t q_base = smem_u32(sQ(i));
         const uint32_t k_base = smem_u32(sK(t & 1));
@@ -235,13 +237,15 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
         }
         umma_commit(&s_full[i]);
       };
+      // O_i += P_i V: P_i from the first 64 TMEM columns of S_i (8 columns =
+      // 16 keys per MMA), V from shared memory
       auto issue_pv = [&](int i, int t) {
         const uint32_t v_base = smem_u32(sV(t & 1));
 #pragma unroll
         for (int k = 0; k < BKV / 16; ++k) {
-          const uint64_t ad = sw128_desc(p_base + (k >> 2) * BOX_BYTES + (k & 3) * 32, 16, 1024);
           const uint64_t bd = sw128_desc(v_base + k * 2048, BOX_BYTES, 1024);
-          umma_bf16(tmem + 256u + 128u * i, ad, bd, idesc_o, (t > 0 || k > 0) ? 1u : 0u);
+          umma_bf16_tmem_a(tmem + 256u + 128u * i, tmem + 128u * i + 8u * k, bd, idesc_o,
+                           (t > 0 || k > 0) ? 1u : 0u);
         }
         umma_commit(&o_done[i]);
       };
@@ -387,21 +391,8 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
               *reinterpret_cast<uint4*>(vr + j * BOX_BYTES + c16 * 16) = make_uint4(0, 0, 0, 0);
         }
       }
-      // the shared P buffer and this tile's O accumulator are free once the
-      // previous PV products that read / write them have completed
-      if (i == 0 && t > 0) {
-        if (!mbar_wait_warp(&o_done[has1 ? 1 : 0], static_cast<uint32_t>((t - 1) & 1), abort_flag, err,
-                       DEV_TIMEOUT_ATTN + 256 * 12)) {
-          ok = false;
-          break;
-        }
-      } else if (i == 1) {
-        if (!mbar_wait_warp(&o_done[0], tp, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 13)) {
-          ok = false;
-          break;
-        }
-      }
-      tc_fence_after();
+      // S_i(t) complete means every earlier MMA is too (PV_i(t-1) included),
+      // so O_i can be rescaled and P_i written over S_i without another wait.
       // tcgen05.ld / tcgen05.st are warp-collective: the whole warp rescales
       // when any of its rows needs it (rows that do not use alpha = 1)
       if (__any_sync(0xffffffffu, rescale)) {
@@ -415,23 +406,22 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
           for (int j = 0; j < 32; ++j) o[j] *= alpha;
           tmem_st32(tO + c * 32, o);
         }
-        tmem_st_wait();
         l *= alpha;
       }
       m = m_use;
       l += lsum;
-      unsigned char* prow = sP + row * 128;
+      // P_i as bf16 pairs (keys 2c, 2c+1 in column c) over the first 64
+      // columns of S_i, the A operand of the PV product
 #pragma unroll
-      for (int c = 0; c < BKV / 8; ++c) {
-        uint4 o;
-        o.x = pack_bf16x2(s[8 * c], s[8 * c + 1]);
-        o.y = pack_bf16x2(s[8 * c + 2], s[8 * c + 3]);
-        o.z = pack_bf16x2(s[8 * c + 4], s[8 * c + 5]);
-        o.w = pack_bf16x2(s[8 * c + 6], s[8 * c + 7]);
-        const int chunk = c & 7;
-        *reinterpret_cast<uint4*>(prow + (c >> 3) * BOX_BYTES + ((chunk ^ (row & 7)) << 4)) = o;
+      for (int h2 = 0; h2 < 2; ++h2) {
+        float pk[32];
+#pragma unroll
+        for (int c = 0; c < 32; ++c)
+          pk[c] = __uint_as_float(pack_bf16x2(s[64 * h2 + 2 * c], s[64 * h2 + 2 * c + 1]));
+        tmem_st32(tS + 32 * h2, pk);
       }
-      fence_proxy_async_smem();
+      tmem_st_wait();
+      fence_proxy_async_smem();  // the zeroed V rows, if any, are read by the tensor core
       tc_fence_before();
       mbar_arrive(&p_full[i]);
     }
