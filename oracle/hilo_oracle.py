@@ -27,6 +27,11 @@ the DiT it feeds; the concrete variant -- token-space score, top-k split,
   unpack  every grid token reads the output row of its kept token or of its
           window (nearest broadcast).
   update  x <- bf16(x - alpha * y) for the denoising loop.
+  sobel_select  the paper's own selector (Sec. 2.3): a Sobel frequency map
+          of the input image, normalised by its maximum, thresholded, pooled
+          onto the token grid (a token of P x P pixels is selected when any
+          of its pixels exceeds the threshold), united with the user mask
+          dilated by R tokens. It yields the keep map used with k_keep = 0.
 
 Precision. Where a float decides an integer or a stored bf16 code (the score
 decides the split; the pooled mean is stored as bf16; the loop update is
@@ -44,6 +49,14 @@ Fixed orders (readings where the paper is silent):
   * pooled mean: fp32 sum of the class members in raster order starting from
     the first member, one correctly rounded division by the member count,
     then bf16 round-to-nearest-even.
+
+  * Sobel map (readings: the paper names the operator, not the border rule,
+    the channel combination or the norm): replicate borders; per channel
+    gx = ((P(y-1,x+1) + 2P(y,x+1)) + P(y+1,x+1)) - ((P(y-1,x-1) + 2P(y,x-1))
+    + P(y+1,x-1)) and gy likewise with rows; g = sqrt(sum over channels in
+    ascending order of (gx*gx + gy*gy)), fp32, correctly rounded sqrt; the
+    map is normalised by its per-image maximum with one fp32 division per
+    token maximum, and the comparison with the threshold is strict.
 
 Bit patterns of bf16 arrays are carried as numpy uint16.
 """
@@ -361,6 +374,66 @@ def update(x_bits: np.ndarray, y: np.ndarray, alpha: float) -> np.ndarray:
     x = bf16_to_f32(x_bits)
     t = np.float32(alpha) * np.asarray(y, dtype=np.float32)
     return f32_to_bf16(x - t)
+
+
+# ---------------------------------------------------------------------------
+# The paper's selector: Sobel frequency map, threshold, 16x regionalisation,
+# dilated mask (Sec. 2.3 "HiLo-Token Selection")
+# ---------------------------------------------------------------------------
+
+
+def sobel_magnitude(img: np.ndarray) -> np.ndarray:
+    """Per-pixel Sobel gradient magnitude of img [B, Hp, Wp, C] fp32 (Sec. 2.3:
+    the spatial-frequency map), fp32 in the fixed order of the module header,
+    replicate borders. Returns g [B, Hp, Wp] fp32."""
+    img = np.ascontiguousarray(img, dtype=np.float32)
+    p = np.pad(img, ((0, 0), (1, 1), (1, 1), (0, 0)), mode="edge")
+    two = np.float32(2.0)
+    # p[:, y + 1, x + 1] is pixel (y, x)
+    up, mid, dn = p[:, :-2], p[:, 1:-1], p[:, 2:]
+    right = (up[:, :, 2:] + two * mid[:, :, 2:]) + dn[:, :, 2:]
+    left = (up[:, :, :-2] + two * mid[:, :, :-2]) + dn[:, :, :-2]
+    gx = right - left
+    lt, ct, rt = p[:, :, :-2], p[:, :, 1:-1], p[:, :, 2:]
+    bottom = (lt[:, 2:] + two * ct[:, 2:]) + rt[:, 2:]
+    top = (lt[:, :-2] + two * ct[:, :-2]) + rt[:, :-2]
+    gy = bottom - top
+    acc = np.zeros(img.shape[:3], dtype=np.float32)
+    for c in range(img.shape[3]):
+        acc = acc + (gx[..., c] * gx[..., c] + gy[..., c] * gy[..., c])
+    return np.sqrt(acc)
+
+
+def dilate_mask(mask: np.ndarray, H: int, W: int, radius: int) -> np.ndarray:
+    """Mask [B, N] dilated on the H x W token grid by a square of radius R
+    tokens (Sec. 2.3: the user mask is dilated to keep nearby context)."""
+    m = np.asarray(mask, dtype=np.uint8).reshape(-1, H, W) != 0
+    out = np.zeros_like(m)
+    for dy in range(-radius, radius + 1):
+        for dx in range(-radius, radius + 1):
+            sh = np.zeros_like(m)
+            ys, yd = (slice(0, H - dy), slice(dy, H)) if dy >= 0 else (slice(-dy, H), slice(0, H + dy))
+            xs, xd = (slice(0, W - dx), slice(dx, W)) if dx >= 0 else (slice(-dx, W), slice(0, W + dx))
+            sh[:, yd, xd] = m[:, ys, xs]
+            out |= sh
+    return out.reshape(mask.shape).astype(np.uint8)
+
+
+def sobel_select(img: np.ndarray, mask: np.ndarray, H: int, W: int, patch: int, radius: int,
+                 threshold: float) -> np.ndarray:
+    """Keep map [B, N] u8 of the paper's selector (Sec. 2.3), in its order:
+    normalised Sobel frequency map -> tokens whose magnitude exceeds the
+    threshold, regionalised to the token grid by pooling each P x P patch
+    (the token is selected when its largest normalised value exceeds the
+    threshold) -> union with the user mask dilated by `radius` tokens."""
+    g = sobel_magnitude(img)
+    B = g.shape[0]
+    tokmax = g.reshape(B, H, patch, W, patch).max(axis=(2, 4)).reshape(B, H * W)
+    gmax = g.reshape(B, -1).max(axis=1).astype(np.float32)
+    with np.errstate(invalid="ignore", divide="ignore"):
+        f = tokmax / gmax[:, None]  # fp32 division; 0/0 = nan selects nothing
+    hf = f > np.float32(threshold)
+    return (hf | (dilate_mask(mask, H, W, radius) != 0)).astype(np.uint8)
 
 
 def hot_path(x_bits, text_bits, mask, k_keep, k_mid, levels, weights_list, heads, mlp):

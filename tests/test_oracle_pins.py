@@ -427,3 +427,120 @@ def test_weights_f64_same_block():
     a = O.block(ut, ui, [0, 7], T, w, heads, True)
     b = O.block(ut, ui, [0, 7], T, O.weights_f64(w), heads, True)
     assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
+
+
+# ------------------------------------------------ Sobel selector (Sec. 2.3) --
+
+def _brute_sobel_select(img, mask, H, W, P, R, t):
+    """Pixel-by-pixel loops, written independently of the oracle's slicing."""
+    B, Hp, Wp, C = img.shape
+    keep = np.zeros((B, H * W), dtype=np.uint8)
+    for b in range(B):
+        def px(y, x, c):
+            return np.float32(img[b, min(max(y, 0), Hp - 1), min(max(x, 0), Wp - 1), c])
+        g = np.zeros((Hp, Wp), dtype=np.float32)
+        for y in range(Hp):
+            for x in range(Wp):
+                acc = np.float32(0.0)
+                for c in range(C):
+                    gx = ((px(y - 1, x + 1, c) + np.float32(2) * px(y, x + 1, c)) + px(y + 1, x + 1, c)) - \
+                         ((px(y - 1, x - 1, c) + np.float32(2) * px(y, x - 1, c)) + px(y + 1, x - 1, c))
+                    gy = ((px(y + 1, x - 1, c) + np.float32(2) * px(y + 1, x, c)) + px(y + 1, x + 1, c)) - \
+                         ((px(y - 1, x - 1, c) + np.float32(2) * px(y - 1, x, c)) + px(y - 1, x + 1, c))
+                    acc = np.float32(acc + np.float32(np.float32(gx * gx) + np.float32(gy * gy)))
+                g[y, x] = np.sqrt(acc)
+        gmax = g.max()
+        for i in range(H):
+            for j in range(W):
+                hf = False
+                if gmax > 0:
+                    hf = np.float32(g[i * P:(i + 1) * P, j * P:(j + 1) * P].max() / gmax) > np.float32(t)
+                dil = any(mask[b, ii * W + jj] for ii in range(max(0, i - R), min(H, i + R + 1))
+                          for jj in range(max(0, j - R), min(W, j + R + 1)))
+                keep[b, i * W + j] = 1 if (hf or dil) else 0
+    return keep
+
+
+@pytest.mark.parametrize("R,t", [(0, 0.1), (1, 0.3), (2, 0.05)])
+def test_sobel_select_brute_force(R, t):
+    rng = np.random.default_rng(40 + R)
+    B, H, W, P, C = 2, 3, 4, 4, 3
+    img = rng.random((B, H * P, W * P, C)).astype(np.float32)
+    img[:, :, :5] *= 0.1   # a flat-ish region, so the threshold matters
+    mask = (rng.random((B, H * W)) < 0.15).astype(np.uint8)
+    assert np.array_equal(O.sobel_select(img, mask, H, W, P, R, t), _brute_sobel_select(img, mask, H, W, P, R, t))
+
+
+def test_sobel_magnitude_matches_scipy_per_channel():
+    nd = pytest.importorskip("scipy.ndimage")
+    rng = np.random.default_rng(41)
+    img = rng.standard_normal((2, 24, 40, 3)).astype(np.float32)
+    ref = np.zeros(img.shape[:3])
+    for b in range(2):
+        acc = 0.0
+        for c in range(3):
+            a = img[b, :, :, c].astype(np.float64)
+            acc = acc + nd.sobel(a, axis=1, mode="nearest") ** 2 + nd.sobel(a, axis=0, mode="nearest") ** 2
+        ref[b] = np.sqrt(acc)
+    assert np.abs(O.sobel_magnitude(img) - ref).max() <= 1e-6 * ref.max()
+
+
+def test_sobel_select_constant_image_keeps_only_dilated_mask():
+    H, W, P = 4, 5, 8
+    img = np.full((1, H * P, W * P, 3), 0.7, dtype=np.float32)
+    mask = np.zeros((1, H * W), dtype=np.uint8)
+    mask[0, 2 * W + 2] = 1
+    keep = O.sobel_select(img, mask, H, W, P, 1, 0.1).reshape(H, W)
+    exp = np.zeros((H, W), dtype=np.uint8)
+    exp[1:4, 1:4] = 1
+    assert np.array_equal(keep, exp)
+
+
+def test_sobel_select_step_edge_closed_form():
+    """A vertical step between pixel columns e-1 and e gives |G| = 4 exactly in
+    those two columns and 0 elsewhere (the 3-wide Sobel support), so exactly the
+    token columns holding pixel column e-1 or e are selected, in every row."""
+    H, W, P = 3, 6, 8
+    for e in (8, 13, 40):
+        img = np.zeros((1, H * P, W * P, 1), dtype=np.float32)
+        img[:, :, e:] = 1.0
+        g = O.sobel_magnitude(img)[0]
+        assert np.all(g[:, e - 1:e + 1] == 4.0) and np.count_nonzero(g) == 2 * H * P
+        keep = O.sobel_select(img, np.zeros((1, H * W), np.uint8), H, W, P, 0, 0.1).reshape(H, W)
+        cols = {(e - 1) // P, e // P}
+        exp = np.zeros((H, W), dtype=np.uint8)
+        exp[:, sorted(cols)] = 1
+        assert np.array_equal(keep, exp)
+
+
+def test_sobel_select_ramp_and_strict_threshold():
+    """A ramp P(y, x) = a x has |G| = 8a inside and 4a in the two replicated
+    border columns: normalised 1 and 1/2. Every token is selected at t = 0.1 and
+    at t = 0.5 (its largest value is 1), none at t = 1 (the test is strict)."""
+    H, W, P, a = 2, 3, 4, 0.25
+    x = np.arange(W * P, dtype=np.float32) * np.float32(a)
+    img = np.broadcast_to(x[None, None, :, None], (1, H * P, W * P, 1)).copy()
+    g = O.sobel_magnitude(img)[0]
+    assert np.all(g[:, 1:-1] == np.float32(8 * a)) and np.all(g[:, [0, -1]] == np.float32(4 * a))
+    z = np.zeros((1, H * W), np.uint8)
+    assert O.sobel_select(img, z, H, W, P, 0, 0.1).all()
+    assert O.sobel_select(img, z, H, W, P, 0, 0.5).all()
+    assert not O.sobel_select(img, z, H, W, P, 0, 1.0).any()
+
+
+def test_dilate_mask_brute_and_monotone_threshold():
+    rng = np.random.default_rng(42)
+    H, W = 7, 9
+    m = (rng.random((2, H * W)) < 0.1).astype(np.uint8)
+    for R in (0, 1, 3):
+        d = O.dilate_mask(m, H, W, R).reshape(2, H, W)
+        for b in range(2):
+            mm = m[b].reshape(H, W)
+            for i in range(H):
+                for j in range(W):
+                    assert d[b, i, j] == int(mm[max(0, i - R):i + R + 1, max(0, j - R):j + R + 1].any())
+    assert np.array_equal(O.dilate_mask(m, H, W, 0), m)
+    img = rng.random((2, H * 4, W * 4, 3)).astype(np.float32)
+    k1 = O.sobel_select(img, m, H, W, 4, 1, 0.2)
+    k2 = O.sobel_select(img, m, H, W, 4, 1, 0.4)
+    assert np.all(k2 <= k1)
