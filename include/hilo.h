@@ -175,6 +175,39 @@ int hilo_split(const hilo_shape* shape, const float* score, const uint8_t* mask,
                const int32_t* k_keep, const int32_t* k_mid, const hilo_split_out* out,
                void* ws, size_t ws_bytes, void* stream);
 
+/* Workspace bytes hilo_sobel_select needs (token maxima and image maxima). */
+size_t hilo_sobel_workspace_bytes(const hilo_shape* shape);
+
+/*
+ * hilo_sobel_select -- the paper's own token selector (Sec. 2.3 "HiLo-Token
+ * Selection"): a Sobel spatial-frequency map of the input image, normalised
+ * by its per-image maximum, thresholded and regionalised onto the token grid,
+ * united with the user mask dilated by `radius` tokens. The keep map it
+ * writes goes to hilo_split as the mask, with k_keep = 0, for an
+ * input-adaptive number of kept tokens.
+ *   img        fp32 [B, H*patch, W*patch, channels], channels last, device;
+ *              channels in [1, 4]
+ *   patch      pixels per token side: 16 (the paper's 16x pooling) or 8
+ *   mask       uint8 [B, H*W] device, nonzero = inside the edit mask
+ *   radius     mask dilation in tokens (square window), >= 0
+ *   threshold  on the normalised map, finite; a token is selected when the
+ *              largest normalised magnitude of its pixels is > threshold
+ *   keep       uint8 [B, H*W] device output, 1 = kept
+ *   ws         device workspace of hilo_sobel_workspace_bytes bytes, 16-byte
+ *              aligned; overwritten
+ * Per pixel and channel gx = ((P(y-1,x+1) + 2P(y,x+1)) + P(y+1,x+1)) -
+ * ((P(y-1,x-1) + 2P(y,x-1)) + P(y+1,x-1)) and gy likewise over rows, with
+ * replicate borders; g = sqrt(sum over channels ascending of (gx*gx +
+ * gy*gy)); every step a correctly rounded fp32 operation, so the keep map is
+ * reproducible bit for bit. The normalised value of a token is one correctly
+ * rounded division tokmax / imgmax; an image with no gradient selects
+ * nothing. Errors: HILO_ERR_ARG (NULL pointer, bad channels, patch, radius or
+ * threshold), HILO_ERR_SHAPE, HILO_ERR_WORKSPACE, HILO_ERR_CUDA.
+ */
+int hilo_sobel_select(const hilo_shape* shape, const float* img, int channels, int patch,
+                      const uint8_t* mask, int radius, float threshold, uint8_t* keep, void* ws,
+                      size_t ws_bytes, void* stream);
+
 /*
  * hilo_pack -- the packed image sequence (paper Sec. 2.3: selected tokens and
  * low-frequency tokens concatenated along the token axis).

@@ -19,7 +19,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libhilo.so")
-SOURCES = ["api.cu", "bw_kernels.cu", "gemm_tc.cu", "gemm2_tc.cu", "attn_tc.cu", "noalloc.cu"]
+SOURCES = ["api.cu", "bw_kernels.cu", "gemm_tc.cu", "gemm2_tc.cu", "attn_tc.cu", "noalloc.cu", "select.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fno-strict-aliasing",
          "--expt-relaxed-constexpr", "-I", INCLUDE, "-I", CSRC]

@@ -249,6 +249,36 @@ int hilo_split(const hilo_shape* shape, const float* score, const uint8_t* mask,
   return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_split");
 }
 
+size_t hilo_sobel_workspace_bytes(const hilo_shape* shape) {
+  if (check_shape(shape, false)) return 0;
+  return hilo::sobel_workspace_bytes(shape->B, shape->H, shape->W);
+}
+
+int hilo_sobel_select(const hilo_shape* shape, const float* img, int channels, int patch,
+                      const uint8_t* mask, int radius, float threshold, uint8_t* keep, void* ws,
+                      size_t ws_bytes, void* stream) {
+  int st = check_shape(shape, false);
+  if (st) return st;
+  if (!img || !mask || !keep || !ws) return fail(HILO_ERR_ARG, "hilo_sobel_select: NULL pointer");
+  if (channels < 1 || channels > 4)
+    return fail(HILO_ERR_ARG, "hilo_sobel_select: channels=%d must be in [1, 4]", channels);
+  if (patch != 8 && patch != 16) return fail(HILO_ERR_ARG, "hilo_sobel_select: patch=%d must be 8 or 16", patch);
+  if (radius < 0) return fail(HILO_ERR_ARG, "hilo_sobel_select: radius=%d must be >= 0", radius);
+  if (!(threshold == threshold) || threshold > 3.0e38f || threshold < -3.0e38f)
+    return fail(HILO_ERR_ARG, "hilo_sobel_select: threshold must be finite");
+  if (reinterpret_cast<uintptr_t>(ws) & 15)
+    return fail(HILO_ERR_ARG, "hilo_sobel_select: workspace must be 16-byte aligned");
+  const size_t need = hilo::sobel_workspace_bytes(shape->B, shape->H, shape->W);
+  if (ws_bytes < need)
+    return fail(HILO_ERR_WORKSPACE, "hilo_sobel_select: workspace %zu < %zu bytes", ws_bytes, need);
+  DevInfo* dev;
+  if ((st = current_device(&dev))) return st;
+  cudaError_t e = hilo::launch_sobel_select(img, shape->B, shape->H, shape->W, channels, patch, mask, radius,
+                                            threshold, keep, ws, dev->num_sms, static_cast<cudaStream_t>(stream));
+  if (e == cudaSuccess) count(2);
+  return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_sobel_select");
+}
+
 int hilo_pack(const hilo_shape* shape, const void* x, const hilo_split_out* split, void* packed,
               int32_t cap, void* stream) {
   int st = check_shape(shape, false);

@@ -35,6 +35,12 @@ cudaError_t launch_layernorm(const void* in_txt, const void* in_img, int in_f32,
 cudaError_t launch_bf16_to_f16(const void* src, void* dst, long long n, int num_sms,
                                cudaStream_t st);
 
+// ---- the paper's Sobel selector (select.cu)
+size_t sobel_workspace_bytes(int B, int H, int W);
+cudaError_t launch_sobel_select(const float* img, int B, int H, int W, int C, int patch,
+                                const uint8_t* mask, int radius, float threshold, uint8_t* keep, void* ws,
+                                int num_sms, cudaStream_t st);
+
 // ---- tcgen05 grouped GEMM (gemm_tc.cu)
 enum GemmEpilogue : int {
   EPI_BIAS_BF16 = 0,      // out_bf16 = acc + bias

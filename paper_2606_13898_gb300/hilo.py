@@ -50,7 +50,7 @@ EXPORTS = ("hilo_status_string", "hilo_last_error", "hilo_sync_status", "hilo_de
            "hilo_score", "hilo_split_workspace_bytes", "hilo_split", "hilo_pack",
            "hilo_block_workspace_bytes", "hilo_block_forward", "hilo_unpack", "hilo_unpack_update",
            "hilo_convert_bf16_to_f16", "hilo_set_stage_events", "hilo_launch_count",
-           "hilo_block_forward_static_ws")
+           "hilo_block_forward_static_ws", "hilo_sobel_workspace_bytes", "hilo_sobel_select")
 
 _lib = None
 
@@ -90,6 +90,8 @@ def lib() -> ctypes.CDLL:
                                              P, I, P, P]),
         "hilo_set_stage_events": (I, [ctypes.POINTER(ctypes.c_void_p), I]),
         "hilo_launch_count": (ctypes.c_ulonglong, []),
+        "hilo_sobel_workspace_bytes": (S, [shp]),
+        "hilo_sobel_select": (I, [shp, P, I, I, P, I, F, P, P, S, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -239,6 +241,19 @@ def hilo_split(shape: Shape, score, mask, k_keep, k_mid, out: SplitBuffers, ws=N
     o = out.c()
     _check("hilo_split", lib().hilo_split(ctypes.byref(s), _ptr(score), _ptr(mask), _ptr(k_keep), _ptr(k_mid),
                                           ctypes.byref(o), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def hilo_sobel_workspace_bytes(shape: Shape) -> int:
+    s = shape.c()
+    return int(lib().hilo_sobel_workspace_bytes(ctypes.byref(s)))
+
+
+def hilo_sobel_select(shape: Shape, img, channels: int, patch: int, mask, radius: int, threshold: float, keep,
+                      ws, ws_bytes: int, stream=None) -> None:
+    s = shape.c()
+    _check("hilo_sobel_select", lib().hilo_sobel_select(ctypes.byref(s), _ptr(img), channels, patch, _ptr(mask),
+                                                        radius, ctypes.c_float(threshold), _ptr(keep), _ptr(ws),
+                                                        ws_bytes, _stream(stream)))
 
 
 def hilo_pack(shape: Shape, x, split: SplitBuffers, packed, cap: int, stream=None) -> None:

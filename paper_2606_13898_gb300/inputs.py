@@ -16,7 +16,12 @@ below stand in for them:
   modelled on the paper's mask statistics (Sec. 2.3, "Mask Distribution":
   most masks small, scattered or elongated holes);
 * masked tokens are overwritten with N(0,1) noise, text tokens are N(0,1);
-* all linear weights and biases are N(0, 0.02^2).
+* all linear weights and biases are N(0, 0.02^2);
+* input image for the paper's Sobel selector (pixel space, P x P pixels per
+  token): a smooth field (three sinusoids per channel, wavelengths of 4..16
+  tokens) in [0.2, 0.8] with sharp-edged rectangles and discs of random
+  colour painted over it, and a small N(0, 0.01^2) noise, fp32 in [0, 1]; the
+  edges carry most of the gradient, as object boundaries do in photographs.
 
 Every floating value is drawn in fp32 and rounded to bf16 (round to nearest
 even); arrays of bf16 are carried as numpy ``uint16`` bit patterns. Small
@@ -193,6 +198,41 @@ def _ellipse_mask(rng: np.random.Generator, H: int, W: int, lo: float, hi: float
         if lo <= m.mean() <= hi:
             return m.astype(np.uint8)
     raise RuntimeError("ellipse mask rejection sampling failed")  # pragma: no cover
+
+
+def make_image(B: int, H: int, W: int, patch: int = 16, channels: int = 3, seed: int = 0,
+               n_shapes: int = 16) -> np.ndarray:
+    """Synthetic image [B, H*patch, W*patch, channels] fp32 (see the module
+    header). Image b uses numpy default_rng(seed + b)."""
+    Hp, Wp = H * patch, W * patch
+    y = np.arange(Hp, dtype=np.float32)[:, None]
+    x = np.arange(Wp, dtype=np.float32)[None, :]
+    out = np.empty((B, Hp, Wp, channels), dtype=np.float32)
+    for b in range(B):
+        rng = np.random.default_rng(seed + b)
+        img = np.zeros((Hp, Wp, channels), dtype=np.float32)
+        for c in range(channels):
+            f = np.zeros((Hp, Wp), dtype=np.float32)
+            for _ in range(3):
+                lam = np.float32(rng.uniform(4.0, 16.0) * patch)
+                th = rng.uniform(0.0, math.pi)
+                ph = rng.uniform(0.0, 2.0 * math.pi)
+                f += np.sin(2.0 * np.pi * (x * np.float32(math.cos(th)) + y * np.float32(math.sin(th))) / lam
+                            + np.float32(ph)).astype(np.float32)
+            img[:, :, c] = 0.5 + 0.1 * f
+        for _ in range(n_shapes):
+            col = rng.uniform(0.0, 1.0, size=channels).astype(np.float32)
+            if rng.random() < 0.5:
+                h, w = int(rng.integers(Hp // 16, Hp // 4 + 1)), int(rng.integers(Wp // 16, Wp // 4 + 1))
+                t0, l0 = int(rng.integers(0, Hp - h + 1)), int(rng.integers(0, Wp - w + 1))
+                img[t0:t0 + h, l0:l0 + w] = col
+            else:
+                r = rng.uniform(Hp / 32, Hp / 8)
+                cy, cx = rng.uniform(0, Hp), rng.uniform(0, Wp)
+                img[(y - cy) ** 2 + (x - cx) ** 2 <= r * r] = col
+        img += rng.normal(0.0, 0.01, size=img.shape).astype(np.float32)
+        out[b] = np.clip(img, 0.0, 1.0)
+    return out
 
 
 @dataclasses.dataclass

@@ -97,3 +97,22 @@ def test_workspace_size_and_check(H):
             setattr(sw, n, 1)
     rc = H.lib().hilo_block_forward(ctypes.byref(s), ctypes.byref(w), 1, cap, 1, 1, 0, 1, 1, nb - 1, None)
     assert rc == -4
+
+
+@pytest.mark.parametrize("channels,patch,radius,thr,code", [
+    (0, 16, 1, 0.1, -1), (5, 16, 1, 0.1, -1), (3, 12, 1, 0.1, -1), (3, 16, -1, 0.1, -1),
+    (3, 16, 1, float("nan"), -1), (3, 16, 1, float("inf"), -1),
+])
+def test_sobel_select_arguments_rejected_before_launch(H, channels, patch, radius, thr, code):
+    s = H.hilo_shape(1, 8, 8, 128, 4, 1, 0, 1)
+    L = H.lib()
+    assert L.hilo_sobel_select(ctypes.byref(s), 1, channels, patch, 1, radius, ctypes.c_float(thr), 1, 16,
+                               1 << 20, None) == code
+
+
+def test_sobel_workspace_query(H):
+    s = H.hilo_shape(2, 8, 8, 128, 4, 1, 0, 1)
+    n = H.lib().hilo_sobel_workspace_bytes(ctypes.byref(s))
+    assert n >= 2 * 64 * 4 + 2 * 4
+    s0 = H.hilo_shape(2, 7, 8, 128, 4, 1, 0, 1)
+    assert H.lib().hilo_sobel_workspace_bytes(ctypes.byref(s0)) == 0
