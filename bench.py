@@ -247,6 +247,70 @@ def block_flops(wl, cu) -> float:
     return gemm + attn
 
 
+def time_sobel_selector(H, I, torch, stream, wl, batch, hp, hbm_peak: float, steps: int) -> dict:
+    """The paper's own selector (Sec. 2.3) on a synthetic image of the
+    workload's grid at 16 x 16 pixels per token (1024 x 1024 x 3 fp32 for
+    64 x 64 tokens): Sobel map, threshold 0.1, regionalisation, the
+    workload's mask dilated by one token. Times the selector alone (HBM-bound:
+    the image is read once) and the hot path driven by its keep map (split
+    with k_keep = 0)."""
+    patch, C, radius, thr = 16, 3, 1, 0.1
+    img = torch.from_numpy(I.make_image(wl.B, wl.H, wl.W, patch, C, seed=77)).cuda()
+    mask = torch.from_numpy(batch.mask).cuda()
+    sh = hp.shape
+    ws_bytes = H.hilo_sobel_workspace_bytes(sh)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
+    keep = torch.empty(wl.B, wl.N, dtype=torch.uint8, device="cuda")
+    zeros = torch.zeros(wl.B, dtype=torch.int32, device="cuda")
+    x = H.bf16_from_bits(batch.x)
+    text = H.bf16_from_bits(batch.text)
+
+    def sel():
+        H.hilo_sobel_select(sh, img, C, patch, mask, radius, thr, keep, ws, ws_bytes, stream)
+
+    def path():
+        sel()
+        hp.run(x, text, keep, zeros, zeros, stream)
+
+    out = {}
+    for name, fn in (("select_host_loop", sel), ("hot_path", path)):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for _ in range(steps):
+            fn()
+        s1.record(stream)
+        torch.cuda.synchronize()
+        out[name + "_ms"] = s0.elapsed_time(s1) / steps
+    # the selector's GPU time: a few microseconds of work per call, so the
+    # host loop above measures mostly submission; replay a captured graph
+    cs = torch.cuda.Stream()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=cs):
+        H.hilo_sobel_select(sh, img, C, patch, mask, radius, thr, keep, ws, ws_bytes, cs)
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s0.record(stream)
+    for _ in range(steps):
+        g.replay()
+    s1.record(stream)
+    torch.cuda.synchronize()
+    out["select_ms"] = s0.elapsed_time(s1) / steps
+    H.hilo_sync_status()
+    nbytes = img.numel() * 4 + 3 * wl.B * wl.N  # image read; mask read, keep written
+    gbs = nbytes / (out["select_ms"] * 1e-3) / 1e9
+    out.update({"image": f"{wl.B}x{wl.H * patch}x{wl.W * patch}x{C} fp32", "threshold": thr, "dilation": radius,
+                "kept_fraction": float(keep.float().mean().item()),
+                "packed_image_rows": int(hp.split.cu_img[-1].item()),
+                "select_GB/s": gbs, "select_frac_hbm": gbs / hbm_peak,
+                "hot_path_image_tokens_per_s": wl.B * wl.N / (out["hot_path_ms"] * 1e-3)})
+    return out
+
+
 def time_configs(H, I, torch, stream, steps: int):
     """Hot path, compressed block and dense block of each workload configuration.
 
@@ -549,6 +613,7 @@ def run_hilo(args):
             Lr = int(hp.split.cu_img[-1].item())
             sweep[r] = {"hot_path_ms": ms_r, "image_tokens_per_s": N / (ms_r * 1e-3), "packed_image_rows": Lr}
         extras["sweep"] = sweep
+        extras["sobel_selector"] = time_sobel_selector(H, I, torch, stream, wl, batch, hp, hbm_peak, Ks)
         if world == 1:
             extras["configs"] = time_configs(H, I, torch, stream, steps=20)
         # dense block: every grid token is its own row, no score/split/pack/unpack

@@ -189,7 +189,7 @@ size_t hilo_sobel_workspace_bytes(const hilo_shape* shape);
  *              channels in [1, 4]
  *   patch      pixels per token side: 16 (the paper's 16x pooling) or 8
  *   mask       uint8 [B, H*W] device, nonzero = inside the edit mask
- *   radius     mask dilation in tokens (square window), >= 0
+ *   radius     mask dilation in tokens (square window), in [0, 64]
  *   threshold  on the normalised map, finite; a token is selected when the
  *              largest normalised magnitude of its pixels is > threshold
  *   keep       uint8 [B, H*W] device output, 1 = kept

@@ -263,7 +263,7 @@ int hilo_sobel_select(const hilo_shape* shape, const float* img, int channels, i
   if (channels < 1 || channels > 4)
     return fail(HILO_ERR_ARG, "hilo_sobel_select: channels=%d must be in [1, 4]", channels);
   if (patch != 8 && patch != 16) return fail(HILO_ERR_ARG, "hilo_sobel_select: patch=%d must be 8 or 16", patch);
-  if (radius < 0) return fail(HILO_ERR_ARG, "hilo_sobel_select: radius=%d must be >= 0", radius);
+  if (radius < 0 || radius > 64) return fail(HILO_ERR_ARG, "hilo_sobel_select: radius=%d must be in [0, 64]", radius);
   if (!(threshold == threshold) || threshold > 3.0e38f || threshold < -3.0e38f)
     return fail(HILO_ERR_ARG, "hilo_sobel_select: threshold must be finite");
   if (reinterpret_cast<uintptr_t>(ws) & 15)

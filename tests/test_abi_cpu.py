@@ -101,7 +101,7 @@ def test_workspace_size_and_check(H):
 
 @pytest.mark.parametrize("channels,patch,radius,thr,code", [
     (0, 16, 1, 0.1, -1), (5, 16, 1, 0.1, -1), (3, 12, 1, 0.1, -1), (3, 16, -1, 0.1, -1),
-    (3, 16, 1, float("nan"), -1), (3, 16, 1, float("inf"), -1),
+    (3, 16, 1, float("nan"), -1), (3, 16, 1, float("inf"), -1), (3, 16, 65, 0.1, -1),
 ])
 def test_sobel_select_arguments_rejected_before_launch(H, channels, patch, radius, thr, code):
     s = H.hilo_shape(1, 8, 8, 128, 4, 1, 0, 1)
