@@ -175,7 +175,8 @@ int hilo_split(const hilo_shape* shape, const float* score, const uint8_t* mask,
                const int32_t* k_keep, const int32_t* k_mid, const hilo_split_out* out,
                void* ws, size_t ws_bytes, void* stream);
 
-/* Workspace bytes hilo_sobel_select needs (token maxima and image maxima). */
+/* Workspace bytes hilo_sobel_select needs (token maxima and one maximum per
+ * 32 x 64-pixel tile). */
 size_t hilo_sobel_workspace_bytes(const hilo_shape* shape);
 
 /*

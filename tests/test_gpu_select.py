@@ -53,6 +53,28 @@ def test_sobel_select_bitexact(H, B, Hh, W, patch, C, radius, thr):
     assert 0 < ref.sum() < ref.size
 
 
+def test_sobel_select_unaligned_image(H):
+    """An image that starts 4 bytes past a 16-byte boundary takes the scalar
+    load path of every tile; the keep map is unchanged in definition."""
+    B, Hh, W, patch, C = 2, 8, 12, 16, 3
+    img = I.make_image(B, Hh, W, patch, C, seed=5)
+    rng = np.random.default_rng(9)
+    mask = (rng.random((B, Hh * W)) < 0.05).astype(np.uint8)
+    buf = torch.empty(img.size + 1, dtype=torch.float32, device="cuda")
+    view = buf[1:].view(img.shape)
+    view.copy_(torch.from_numpy(img))
+    assert view.data_ptr() % 16 != 0
+    sh = H.Shape(B=B, H=Hh, W=W, d=128)
+    ws_bytes = H.hilo_sobel_workspace_bytes(sh)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
+    keep = torch.full((B, Hh * W), 7, dtype=torch.uint8, device="cuda")
+    H.hilo_sobel_select(sh, view, C, patch, torch.from_numpy(mask).cuda(), 1, 0.1, keep, ws, ws_bytes)
+    H.hilo_sync_status()
+    ref = O.sobel_select(img, mask, Hh, W, patch, 1, 0.1)
+    assert np.array_equal(keep.cpu().numpy(), ref)
+    assert 0 < ref.sum() < ref.size
+
+
 def test_sobel_select_constant_and_step_images(H):
     Hh, W, patch = 4, 6, 16
     const = np.full((1, Hh * patch, W * patch, 3), 0.25, dtype=np.float32)
