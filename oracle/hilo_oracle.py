@@ -26,6 +26,12 @@ the DiT it feeds; the concrete variant -- token-space score, top-k split,
           softmax attention, tanh-GELU 4x MLP, residual adds.
   unpack  every grid token reads the output row of its kept token or of its
           window (nearest broadcast).
+  split(granular=True), unpack_delta  the window-granular (regionalised)
+          split -- each pooling window takes the finest class of any member,
+          so kept regions are whole 2x2 windows and every pooled window is
+          full -- and the delta unpool, where a pooled member keeps its own
+          value plus its window's update (Sec. 2.3's coherent, region-level
+          selection read in token space).
   update  x <- bf16(x - alpha * y) for the denoising loop.
   sobel_select  the paper's own selector (Sec. 2.3): a Sobel frequency map
           of the input image, normalised by its maximum, thresholded, pooled
@@ -151,8 +157,17 @@ def ranking(s: np.ndarray) -> np.ndarray:
     return np.lexsort((idx, -s.astype(np.float64)))
 
 
-def split(s: np.ndarray, mask: np.ndarray, k_keep, k_mid, H: int, W: int, levels: int) -> Split:
-    """Deterministic keep/pool split of each image (see module docstring)."""
+def split(s: np.ndarray, mask: np.ndarray, k_keep, k_mid, H: int, W: int, levels: int,
+          granular: bool = False) -> Split:
+    """Deterministic keep/pool split of each image (see module docstring).
+
+    granular=True is the window-granular (regionalised) variant, the token-
+    space reading of the coherent region-level selection of Sec. 2.3: every
+    pooling window takes the finest class any of its members has. An aligned
+    2x2 window with a member in top-k_keep or the mask is kept whole; with two
+    levels, an aligned 4x4 block is pooled 4x4 only when all 16 of its members
+    rank below the k_mid cut, otherwise its (whole, non-kept) 2x2 windows are
+    pooled 2x2. Every pooled window is then full."""
     B, N = s.shape
     assert N == H * W and levels in (1, 2)
     labels = np.empty((B, N), dtype=np.uint8)
@@ -168,11 +183,17 @@ def split(s: np.ndarray, mask: np.ndarray, k_keep, k_mid, H: int, W: int, levels
         order = ranking(s[b])
         keep = mask[b].astype(bool).copy()
         keep[order[:int(k_keep[b])]] = True
+        if granular:
+            keep = np.isin(win2_of, win2_of[keep])
         lab = np.full(N, POOL2, dtype=np.uint8)
         lab[keep] = KEEP
         if levels == 2:
             rest = order[~keep[order]]
             lab[rest[int(k_mid[b]):]] = POOL4
+            if granular:
+                whole4 = np.ones((H // 4) * (W // 4), dtype=bool)
+                np.logical_and.at(whole4, win4_of, lab == POOL4)
+                lab[(lab == POOL4) & ~whole4[win4_of]] = POOL2
         labels[b] = lab
         kept = np.nonzero(lab == KEEP)[0]
         w2 = np.unique(win2_of[lab == POOL2])
@@ -367,6 +388,28 @@ def block_dense(x_bits, text_bits, weights, heads: int, mlp: bool):
 def unpack(out_img: np.ndarray, sp: Split) -> np.ndarray:
     """y[b, i] = out_img[tok_row[b, i]]  ->  [B, N, d]."""
     return out_img[sp.tok_row]
+
+
+def unpack_delta(out_img: np.ndarray, packed_bits: np.ndarray, x_bits: np.ndarray, sp: Split) -> np.ndarray:
+    """Delta unpool (the additive reading of restoring pooled tokens to the
+    grid): a kept token takes its own output row; a pooled member i of window
+    row r keeps its own value and receives the window's update,
+    y_i = x_i + (out_r - packed_r), two fp32 operations in that order, with
+    x_i and packed_r the bf16 values widened to fp32. Returns fp32
+    [B, H, W, d]."""
+    B, H, W, d = x_bits.shape
+    x = bf16_to_f32(x_bits).reshape(B, H * W, d)
+    p = bf16_to_f32(packed_bits)
+    out = np.asarray(out_img, dtype=np.float32)
+    y = np.empty((B, H * W, d), dtype=np.float32)
+    for b in range(B):
+        for i in range(H * W):
+            r = int(sp.tok_row[b, i])
+            if sp.labels[b, i] == KEEP:
+                y[b, i] = out[r]
+            else:
+                y[b, i] = x[b, i] + (out[r] - p[r])
+    return y.reshape(B, H, W, d)
 
 
 def update(x_bits: np.ndarray, y: np.ndarray, alpha: float) -> np.ndarray:

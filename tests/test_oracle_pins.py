@@ -198,7 +198,102 @@ def test_split_count_law():
     assert int(sp.counts[0, 0]) == len(top | set(np.nonzero(b.mask[0])[0].tolist()))
 
 
+def test_split_granular_hand_worked():
+    """4 x 4 grid, one level, k_keep = 1, no mask. The largest score sits at
+    token 5 (row 1, column 1), so its 2 x 2 window {0, 1, 4, 5} is kept whole
+    and the three other windows are pooled with all four members each."""
+    s = np.zeros((1, 16), dtype=np.float32)
+    s[0, 5] = 3.0
+    s[0, 10] = 2.0
+    sp = O.split(s, np.zeros((1, 16), np.uint8), [1], [0], 4, 4, 1, granular=True)
+    assert sp.labels[0].tolist() == [0, 0, 1, 1, 0, 0, 1, 1, 1, 1, 1, 1, 1, 1, 1, 1]
+    assert sp.counts[0].tolist() == [4, 3, 0]
+    assert sp.row_src.tolist() == [0, 1, 4, 5, 1, 2, 3]
+    assert sp.tok_row[0].tolist() == [0, 1, 4, 4, 2, 3, 4, 4, 5, 5, 6, 6, 5, 5, 6, 6]
+    # two levels on a 4 x 8 grid (4 x 4 blocks: columns 0-3 and 4-7; 2 x 2
+    # window id = 4 * (row // 2) + col // 2): token 9 (row 1, column 1) ranks
+    # first, token 22 (row 2, column 6, right block) second. k_keep = 1 keeps
+    # window 0 = {0, 1, 8, 9} whole. With k_mid = 1 token 22 is above the
+    # cut, so neither block is entirely below it: the left block's windows
+    # 1, 4, 5 and the right block's 2, 3, 6, 7 are pooled 2 x 2.
+    s = np.zeros((1, 32), dtype=np.float32)
+    s[0, 9] = 3.0
+    s[0, 22] = 2.0
+    sp = O.split(s, np.zeros((1, 32), np.uint8), [1], [1], 4, 8, 2, granular=True)
+    assert sp.counts[0].tolist() == [4, 7, 0]
+    assert sp.row_src.tolist() == [0, 1, 8, 9, 1, 2, 3, 4, 5, 6, 7]
+    # k_mid = 0: the whole right block is below the cut and is pooled 4 x 4
+    # (4 x 4 window 1); the left block still holds the kept window
+    sp = O.split(s, np.zeros((1, 32), np.uint8), [1], [0], 4, 8, 2, granular=True)
+    assert sp.counts[0].tolist() == [4, 3, 1]
+    assert sp.row_src.tolist() == [0, 1, 8, 9, 1, 4, 5, 1]
+
+
+def _brute_split_granular(s, m, k, kmid, H, W, levels):
+    """Pure-Python window-granular split of one image from the rule."""
+    N = H * W
+    order = sorted(range(N), key=lambda i: (-float(s[i]), i))
+    sel = set(order[:k]) | {i for i in range(N) if m[i]}
+    win2 = lambda i: (i // W // 2, (i % W) // 2)
+    win4 = lambda i: (i // W // 4, (i % W) // 4)
+    kept_w = {win2(i) for i in sel}
+    keep = {i for i in range(N) if win2(i) in kept_w}
+    rest = [i for i in order if i not in keep]
+    if levels == 1:
+        return keep, set(rest), set()
+    below = set(rest[kmid:])
+    pool4 = set()
+    for bp in range(H // 4):
+        for bq in range(W // 4):
+            mem = [(4 * bp + i) * W + 4 * bq + j for i in range(4) for j in range(4)]
+            if all(t in below for t in mem):
+                pool4 |= set(mem)
+    pool2 = set(rest) - pool4
+    return keep, pool2, pool4
+
+
+@pytest.mark.parametrize("levels", [1, 2])
+@pytest.mark.parametrize("seed", range(6))
+def test_split_granular_brute_force_and_invariants(seed, levels):
+    rng = np.random.default_rng(100 + seed)
+    H, W = (8, 8) if seed % 2 else (4, 12)
+    N, B = H * W, 3
+    s = (rng.integers(0, 6, size=(B, N)) * 0.5).astype(np.float32)
+    m = (rng.random((B, N)) < 0.1).astype(np.uint8)
+    kk = rng.integers(0, N // 3, size=B)
+    km = rng.integers(0, N // 2, size=B)
+    sp = O.split(s, m, kk, km, H, W, levels, granular=True)
+    flat = O.split(s, m, kk, km, H, W, levels)
+    for b in range(B):
+        keep, pool2, pool4 = _brute_split_granular(s[b], m[b], int(kk[b]), int(km[b]), H, W, levels)
+        lab = sp.labels[b]
+        assert {i for i in range(N) if lab[i] == O.KEEP} == keep
+        assert {i for i in range(N) if lab[i] == O.POOL2} == pool2
+        assert {i for i in range(N) if lab[i] == O.POOL4} == pool4
+        # every kept 2x2 window holds a token the flat split keeps, and the
+        # flat kept set is covered
+        fk = flat.labels[b] == O.KEEP
+        assert np.all(lab[fk] == O.KEEP)
+        g = lab.reshape(H // 2, 2, W // 2, 2).transpose(0, 2, 1, 3).reshape(-1, 4)
+        f = fk.reshape(H // 2, 2, W // 2, 2).transpose(0, 2, 1, 3).reshape(-1, 4)
+        for wl, wf in zip(g, f):
+            assert len(set(wl.tolist())) == 1 or not np.any(wl == O.KEEP)   # kept windows are whole
+            assert (wl[0] == O.KEEP) == bool(wf.any())
+        nk, n2, n4 = (int(c) for c in sp.counts[b])
+        assert nk == 4 * int(f.any(axis=1).sum())
+        # pooled windows are full
+        assert 4 * n2 == int(np.sum(lab == O.POOL2)) and 16 * n4 == int(np.sum(lab == O.POOL4))
+        base = int(sp.cu_img[b])
+        for i in range(N):
+            r = int(sp.tok_row[b, i]) - base
+            if lab[i] == O.KEEP:
+                assert int(sp.row_src[base + r]) == i
+    spN = O.split(s, m, [N] * B, [0] * B, H, W, levels, granular=True)
+    assert np.all(spN.labels == O.KEEP)
+
+
 # ---------------------------------------------------------- pack/unpack ----
+
 
 def test_pack_constant_windows_lossless():
     rng = np.random.default_rng(4)
@@ -240,7 +335,61 @@ def test_unpack_pack_identity_on_kept_rows_and_brute_mean():
         assert np.all(np.abs(got - ref) <= np.abs(ref) * 2 ** -8 + 1e-30)
 
 
+def _delta_case(granular=True, levels=2):
+    rng = np.random.default_rng(21)
+    H, W, d = 16, 16, 32
+    x = rng.uniform(-4, 4, size=(1, H, W, d)).astype(np.float32)
+    xb = bits(x)
+    s = O.score(xb)
+    # at most 8 of the 16 4 x 4 blocks hold a kept or above-cut token
+    sp = O.split(s, np.zeros((1, H * W), np.uint8), [4], [4], H, W, levels, granular=granular)
+    return xb, sp, O.pack(xb, sp)
+
+
+@pytest.mark.parametrize("granular", [False, True])
+def test_unpack_delta_identity_block_returns_x(granular):
+    """A block that changes nothing (out = packed) leaves every pooled member
+    at its own value, bit for bit; kept tokens read their own rows."""
+    xb, sp, packed = _delta_case(granular)
+    out = O.bf16_to_f32(packed)
+    y = O.unpack_delta(out, packed, xb, sp)
+    assert np.array_equal(y, O.bf16_to_f32(xb))
+
+
+def test_unpack_delta_shift_is_exact():
+    """A block that adds 0.5 everywhere: out - packed = 0.5 exactly and
+    x + 0.5 is exact for |x| < 4, so every pooled member moves by exactly 0.5
+    while kept tokens take their output rows."""
+    xb, sp, packed = _delta_case()
+    out = O.bf16_to_f32(packed) + np.float32(0.5)
+    y = O.unpack_delta(out, packed, xb, sp).reshape(-1, xb.shape[-1])
+    xf = O.bf16_to_f32(xb).reshape(-1, xb.shape[-1])
+    lab = sp.labels[0]
+    assert np.array_equal(y[lab != O.KEEP], xf[lab != O.KEEP] + np.float32(0.5))
+    assert np.array_equal(y[lab == O.KEEP], xf[lab == O.KEEP] + np.float32(0.5))
+
+
+def test_unpack_delta_window_mean_is_window_output():
+    """Over a full window the members' mean equals the window's output up to
+    the bf16 rounding of the pooled value: mean(y) - out = mean(x) - packed."""
+    xb, sp, packed = _delta_case()
+    rng = np.random.default_rng(5)
+    out = rng.standard_normal((packed.shape[0], packed.shape[1])).astype(np.float32)
+    y = O.unpack_delta(out, packed, xb, sp).reshape(-1, xb.shape[-1]).astype(np.float64)
+    xf = O.bf16_to_f32(xb).reshape(-1, xb.shape[-1]).astype(np.float64)
+    pf = O.bf16_to_f32(packed).astype(np.float64)
+    nk, n2, n4 = (int(c) for c in sp.counts[0])
+    assert n2 > 0 and n4 > 0
+    for r in range(nk, nk + n2 + n4):
+        mem = np.nonzero(sp.tok_row[0] == r)[0]
+        assert len(mem) in (4, 16)
+        lhs = y[mem].mean(axis=0) - out[r]
+        rhs = xf[mem].mean(axis=0) - pf[r]
+        assert np.all(np.abs(lhs - rhs) <= 4 * 2.0 ** -22 * (np.abs(out[r]) + 8))
+
+
 # --------------------------------------------------------------- block -----
+
 
 def test_layer_norm_and_gelu_closed_forms():
     ln = O.layer_norm(np.array([[1.0, -1.0, 1.0, -1.0], [3.0, 3.0, 3.0, 3.0]]))
