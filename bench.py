@@ -311,6 +311,45 @@ def time_sobel_selector(H, I, torch, stream, wl, batch, hp, hbm_peak: float, ste
     return out
 
 
+def time_regions(H, torch, stream, wl, hp, inputs, hbm_peak: float, steps: int) -> dict:
+    """The window-granular split with the delta unpool on the timed workload:
+    the whole hot path in that mode, and the delta unpool alone against its
+    algorithmic bytes (every token's output written; kept rows' outputs,
+    pooled rows' outputs and bf16 inputs, and pooled members' bf16 tokens
+    read once)."""
+    x, text, mask, kk, km = inputs
+    d = wl.d
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for _ in range(steps):
+            fn()
+        s1.record(stream)
+        torch.cuda.synchronize()
+        return s0.elapsed_time(s1) / steps
+
+    path_ms = timed(lambda: hp.run(x, text, mask, kk, km, regions=True))
+    H.hilo_sync_status()
+    counts = hp.split.counts.view(-1, 3).sum(0).tolist()
+    nk, n2, n4 = (int(c) for c in counts)
+    rows = int(hp.split.cu_img[-1].item())
+    ntok = wl.B * wl.N
+    delta_ms = timed(lambda: H.hilo_unpack_delta(hp.shape, hp.out_img, hp.packed, x, hp.split, hp.y, stream))
+    nearest_ms = timed(lambda: H.hilo_unpack(hp.shape, hp.out_img, hp.split, hp.y, stream))
+    H.hilo_sync_status()
+    pooled_tok = ntok - nk
+    nbytes = ntok * d * 4 + rows * d * 4 + (n2 + n4) * d * 2 + pooled_tok * d * 2 + ntok * 5
+    gbs = nbytes / (delta_ms * 1e-3) / 1e9
+    return {"hot_path_ms": path_ms, "image_tokens_per_s": ntok / (path_ms * 1e-3), "packed_image_rows": rows,
+            "kept_tokens": nk, "windows_2x2": n2, "windows_4x4": n4,
+            "unpack_delta_ms": delta_ms, "unpack_delta_GB/s": gbs, "unpack_delta_frac_hbm": gbs / hbm_peak,
+            "unpack_nearest_ms_same_split": nearest_ms}
+
+
 def time_configs(H, I, torch, stream, steps: int):
     """Hot path, compressed block and dense block of each workload configuration.
 
@@ -614,6 +653,7 @@ def run_hilo(args):
             sweep[r] = {"hot_path_ms": ms_r, "image_tokens_per_s": N / (ms_r * 1e-3), "packed_image_rows": Lr}
         extras["sweep"] = sweep
         extras["sobel_selector"] = time_sobel_selector(H, I, torch, stream, wl, batch, hp, hbm_peak, Ks)
+        extras["regions"] = time_regions(H, torch, stream, wl, hp, (x, text, mask, kk, km), hbm_peak, Ks)
         if world == 1:
             extras["configs"] = time_configs(H, I, torch, stream, steps=20)
         # dense block: every grid token is its own row, no score/split/pack/unpack

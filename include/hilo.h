@@ -175,6 +175,24 @@ int hilo_split(const hilo_shape* shape, const float* score, const uint8_t* mask,
                const int32_t* k_keep, const int32_t* k_mid, const hilo_split_out* out,
                void* ws, size_t ws_bytes, void* stream);
 
+/*
+ * hilo_split_regions -- the window-granular (regionalised) split: the token-
+ * space reading of the coherent, region-level selection of paper Sec. 2.3.
+ * Arguments, outputs and ranking are those of hilo_split; the labels then
+ * give every pooling window the finest class of any of its members:
+ *   - an aligned 2x2 window holding a token of top-k_keep ∪ mask is kept
+ *     whole (all four members HILO_KEEP);
+ *   - levels == 2: the remaining tokens are ranked as in hilo_split and the
+ *     first k_mid are "above the cut"; an aligned 4x4 block is pooled 4x4
+ *     only when all 16 members are below the cut, otherwise its non-kept
+ *     members are pooled 2x2.
+ * Every pooled window is therefore full (4 or 16 members), and kept regions
+ * are whole 2x2 windows. Errors as hilo_split.
+ */
+int hilo_split_regions(const hilo_shape* shape, const float* score, const uint8_t* mask,
+                       const int32_t* k_keep, const int32_t* k_mid, const hilo_split_out* out,
+                       void* ws, size_t ws_bytes, void* stream);
+
 /* Workspace bytes hilo_sobel_select needs (token maxima and one maximum per
  * 32 x 64-pixel tile). */
 size_t hilo_sobel_workspace_bytes(const hilo_shape* shape);
@@ -258,6 +276,21 @@ int hilo_block_forward(const hilo_shape* shape, const hilo_block_weights* weight
  */
 int hilo_unpack(const hilo_shape* shape, const float* out_img, const hilo_split_out* split,
                 float* y, void* stream);
+
+/*
+ * hilo_unpack_delta -- back to the full grid with the delta unpool: a kept
+ * token takes its own output row; a pooled member keeps its own value and
+ * receives its window's update,
+ *     y[b, i] = x[b, i] + (out_img[r] - packed[r]),   r = tok_row[b, i],
+ * one fp32 subtract then one fp32 add, x and packed widened from bf16.
+ *   out_img  fp32 [cap, d]  image rows of the block output
+ *   packed   bf16 [cap, d]  the block's input rows, as hilo_pack wrote them
+ *   x        bf16 [B, H, W, d]  the tokens hilo_pack read
+ *   y        fp32 [B, H, W, d]
+ * All four pointers 16-byte aligned (HILO_ERR_ARG otherwise).
+ */
+int hilo_unpack_delta(const hilo_shape* shape, const float* out_img, const void* packed, const void* x,
+                      const hilo_split_out* split, float* y, void* stream);
 
 /*
  * hilo_unpack_update -- unpack fused with the denoising-loop update

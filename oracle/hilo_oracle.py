@@ -479,16 +479,18 @@ def sobel_select(img: np.ndarray, mask: np.ndarray, H: int, W: int, patch: int, 
     return (hf | (dilate_mask(mask, H, W, radius) != 0)).astype(np.uint8)
 
 
-def hot_path(x_bits, text_bits, mask, k_keep, k_mid, levels, weights_list, heads, mlp):
-    """score -> split -> pack -> blocks -> unpack for one batch.
+def hot_path(x_bits, text_bits, mask, k_keep, k_mid, levels, weights_list, heads, mlp, regions=False):
+    """score -> split -> pack -> blocks -> unpack for one batch; regions=True
+    takes the window-granular split and the delta unpool.
 
     Returns (split, packed, (txt_out, img_out), y) with the block outputs in fp64.
     """
     B, H, W, d = x_bits.shape
     T = text_bits.shape[1]
-    sp = split(score(x_bits), mask, k_keep, k_mid, H, W, levels)
+    sp = split(score(x_bits), mask, k_keep, k_mid, H, W, levels, granular=regions)
     packed = pack(x_bits, sp)
     ut, ui = text_bits.reshape(B * T, d), packed
     for wts in weights_list:
         ut, ui = block(ut, ui, sp.cu_img, T, wts, heads, mlp)
-    return sp, packed, (ut, ui), unpack(ui, sp)
+    y = unpack_delta(ui, packed, x_bits, sp) if regions else unpack(ui, sp)
+    return sp, packed, (ut, ui), y

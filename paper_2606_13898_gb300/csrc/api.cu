@@ -229,24 +229,38 @@ size_t hilo_split_workspace_bytes(const hilo_shape* shape) {
   return 0;
 }
 
+static int split_common(const char* name, const hilo_shape* shape, const float* score, const uint8_t* mask,
+                        const int32_t* k_keep, const int32_t* k_mid, const hilo_split_out* out, int granular,
+                        void* stream) {
+  int st = check_shape(shape, false);
+  if (st) return st;
+  if ((st = check_split(out))) return st;
+  if (!score || !mask || !k_keep) return fail(HILO_ERR_ARG, "%s: NULL pointer", name);
+  if (shape->levels == 2 && !k_mid) return fail(HILO_ERR_ARG, "%s: k_mid is NULL with levels=2", name);
+  DevInfo* dev;
+  if ((st = current_device(&dev))) return st;
+  cudaError_t e = hilo::launch_split(score, mask, k_keep, shape->levels == 2 ? k_mid : k_keep,
+                                     out->labels, out->row_src, out->counts, out->cu_img,
+                                     out->tok_row, shape->B, shape->H, shape->W, shape->levels, granular,
+                                     static_cast<cudaStream_t>(stream));
+  if (e == cudaSuccess) count(shape->B == 1 ? 1 : 2);  // one image: the select kernel also compacts
+  return e == cudaSuccess ? HILO_OK : cuda_fail(e, name);
+}
+
 int hilo_split(const hilo_shape* shape, const float* score, const uint8_t* mask,
                const int32_t* k_keep, const int32_t* k_mid, const hilo_split_out* out, void* ws,
                size_t ws_bytes, void* stream) {
   (void)ws;
   (void)ws_bytes;
-  int st = check_shape(shape, false);
-  if (st) return st;
-  if ((st = check_split(out))) return st;
-  if (!score || !mask || !k_keep) return fail(HILO_ERR_ARG, "hilo_split: NULL pointer");
-  if (shape->levels == 2 && !k_mid) return fail(HILO_ERR_ARG, "hilo_split: k_mid is NULL with levels=2");
-  DevInfo* dev;
-  if ((st = current_device(&dev))) return st;
-  cudaError_t e = hilo::launch_split(score, mask, k_keep, shape->levels == 2 ? k_mid : k_keep,
-                                     out->labels, out->row_src, out->counts, out->cu_img,
-                                     out->tok_row, shape->B, shape->H, shape->W, shape->levels,
-                                     static_cast<cudaStream_t>(stream));
-  if (e == cudaSuccess) count(shape->B == 1 ? 1 : 2);  // one image: the select kernel also compacts
-  return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_split");
+  return split_common("hilo_split", shape, score, mask, k_keep, k_mid, out, 0, stream);
+}
+
+int hilo_split_regions(const hilo_shape* shape, const float* score, const uint8_t* mask,
+                       const int32_t* k_keep, const int32_t* k_mid, const hilo_split_out* out, void* ws,
+                       size_t ws_bytes, void* stream) {
+  (void)ws;
+  (void)ws_bytes;
+  return split_common("hilo_split_regions", shape, score, mask, k_keep, k_mid, out, 1, stream);
 }
 
 size_t hilo_sobel_workspace_bytes(const hilo_shape* shape) {
@@ -418,6 +432,24 @@ int hilo_unpack(const hilo_shape* shape, const float* out_img, const hilo_split_
                                       static_cast<cudaStream_t>(stream));
   if (e == cudaSuccess) count(1);
   return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_unpack");
+}
+
+int hilo_unpack_delta(const hilo_shape* shape, const float* out_img, const void* packed, const void* x,
+                      const hilo_split_out* split, float* y, void* stream) {
+  int st = check_shape(shape, false);
+  if (st) return st;
+  if ((st = check_split(split))) return st;
+  if (!out_img || !packed || !x || !y) return fail(HILO_ERR_ARG, "hilo_unpack_delta: NULL pointer");
+  if ((reinterpret_cast<uintptr_t>(out_img) | reinterpret_cast<uintptr_t>(packed) |
+       reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 15)
+    return fail(HILO_ERR_ARG, "hilo_unpack_delta: pointers must be 16-byte aligned");
+  DevInfo* dev;
+  if ((st = current_device(&dev))) return st;
+  const long long ntok = static_cast<long long>(shape->B) * shape->H * shape->W;
+  cudaError_t e = hilo::launch_unpack_delta(out_img, packed, x, split->labels, split->tok_row, y, ntok,
+                                            shape->d, dev->num_sms, static_cast<cudaStream_t>(stream));
+  if (e == cudaSuccess) count(1);
+  return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_unpack_delta");
 }
 
 int hilo_unpack_update(const hilo_shape* shape, const float* out_img, const hilo_split_out* split,

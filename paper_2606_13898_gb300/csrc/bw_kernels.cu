@@ -380,12 +380,16 @@ __device__ void compact_image(const uint8_t* lab, int b, int H, int W, int level
 
 // Labels and per-image counts. One CTA per image. With a single image
 // (fused != 0) the same CTA also writes cu_img and the packed rows, as
-// nothing depends on other images.
+// nothing depends on other images. granular != 0 is the window-granular
+// split: every pooling window takes the finest class of its members (an
+// aligned 2x2 window with a kept member is kept whole; with two levels an
+// aligned 4x4 block is pooled 4x4 only when all its members rank below the
+// k_mid cut, else its non-kept members are pooled 2x2).
 __global__ void __launch_bounds__(SPLIT_THREADS) split_select_kernel(
     const float* __restrict__ score, const uint8_t* __restrict__ mask,
     const int32_t* __restrict__ k_keep, const int32_t* __restrict__ k_mid, uint8_t* labels_out,
-    int32_t* counts, int H, int W, int levels, int fused, int32_t* cu_img, int32_t* row_src,
-    int32_t* tok_row) {
+    int32_t* counts, int H, int W, int levels, int granular, int fused, int32_t* cu_img,
+    int32_t* row_src, int32_t* tok_row) {
   pdl_trigger();
   pdl_wait();
   extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -413,11 +417,43 @@ __global__ void __launch_bounds__(SPLIT_THREADS) split_select_kernel(
     cand[i] = keep ? 0 : 1;
   }
   __syncthreads();
+  if (granular) {
+    // one thread per 2x2 window: a window with a kept member is kept whole
+    const int W2 = W >> 1, nw = (H >> 1) * W2;
+    for (int w = threadIdx.x; w < nw; w += blockDim.x) {
+      const int t = (2 * (w / W2)) * W + 2 * (w % W2);
+      if (lab[t] == HILO_LABEL_KEEP || lab[t + 1] == HILO_LABEL_KEEP || lab[t + W] == HILO_LABEL_KEEP ||
+          lab[t + W + 1] == HILO_LABEL_KEEP) {
+        lab[t] = lab[t + 1] = lab[t + W] = lab[t + W + 1] = HILO_LABEL_KEEP;
+        cand[t] = cand[t + 1] = cand[t + W] = cand[t + W + 1] = 0;
+      }
+    }
+    __syncthreads();
+  }
   if (levels == 2) {
     mark_topk(keys, cand, sel, N, km, sh);
     for (int i = threadIdx.x; i < N; i += blockDim.x)
       if (cand[i]) lab[i] = sel[i] ? HILO_LABEL_POOL2 : HILO_LABEL_POOL4;
     __syncthreads();
+    if (granular) {
+      // one thread per 4x4 block: pooled 4x4 only when every member is
+      const int W4 = W >> 2, nb = (H >> 2) * W4;
+      for (int v = threadIdx.x; v < nb; v += blockDim.x) {
+        const int t = (4 * (v / W4)) * W + 4 * (v % W4);
+        bool all4 = true;
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+          for (int j = 0; j < 4; ++j) all4 &= lab[t + i * W + j] == HILO_LABEL_POOL4;
+        if (all4) continue;
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (lab[t + i * W + j] == HILO_LABEL_POOL4) lab[t + i * W + j] = HILO_LABEL_POOL2;
+      }
+      __syncthreads();
+    }
   }
   // Per thread, a contiguous chunk of tokens, of 2x2 windows and of 4x4
   // windows: kept tokens, and windows holding at least one member of their
@@ -634,6 +670,45 @@ __global__ void __launch_bounds__(256) unpack_kernel(const float* __restrict__ o
   }
 }
 
+// Delta unpool: a kept token copies its output row; a pooled member keeps
+// its own value plus its window's update, y = x + (out - packed), one fp32
+// subtract then one fp32 add (x and packed widened from bf16).
+__global__ void __launch_bounds__(256) unpack_delta_kernel(const float* __restrict__ out_img,
+                                                           const __nv_bfloat16* __restrict__ packed,
+                                                           const __nv_bfloat16* __restrict__ x,
+                                                           const uint8_t* __restrict__ labels,
+                                                           const int32_t* __restrict__ tok_row,
+                                                           float* __restrict__ y, long long ntok, int d) {
+  pdl_trigger();
+  pdl_wait();
+  const int lane = threadIdx.x & 31;
+  const long long wstep = static_cast<long long>(gridDim.x) * (blockDim.x >> 5);
+  for (long long t = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+       t < ntok; t += wstep) {
+    const int r = __ldg(tok_row + t);
+    const float4* s = reinterpret_cast<const float4*>(out_img + static_cast<long long>(r) * d);
+    float4* o = reinterpret_cast<float4*>(y + t * d);
+    if (__ldg(labels + t) == HILO_LABEL_KEEP) {
+      for (int c = lane; c < (d >> 2); c += 32) __stcs(o + c, __ldg(s + c));
+      continue;
+    }
+    const uint4* xr = reinterpret_cast<const uint4*>(x + t * d);
+    const uint4* pr = reinterpret_cast<const uint4*>(packed + static_cast<long long>(r) * d);
+    for (int c = lane; c < (d >> 3); c += 32) {
+      float xf[8], pf[8];
+      bf16x8_to_f32(__ldg(xr + c), xf);
+      bf16x8_to_f32(__ldg(pr + c), pf);
+      const float4 o0 = __ldg(s + 2 * c), o1 = __ldg(s + 2 * c + 1);
+      const float ov[8] = {o0.x, o0.y, o0.z, o0.w, o1.x, o1.y, o1.z, o1.w};
+      float v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = __fadd_rn(xf[u], __fsub_rn(ov[u], pf[u]));
+      __stcs(o + 2 * c, make_float4(v[0], v[1], v[2], v[3]));
+      __stcs(o + 2 * c + 1, make_float4(v[4], v[5], v[6], v[7]));
+    }
+  }
+}
+
 __global__ void __launch_bounds__(256) unpack_update_kernel(const float* __restrict__ out_img,
                                                             const int32_t* __restrict__ tok_row,
                                                             __nv_bfloat16* __restrict__ x,
@@ -801,7 +876,7 @@ size_t split_compact_smem(int N) { return static_cast<size_t>(N); }
 cudaError_t launch_split(const float* score, const uint8_t* mask, const int32_t* k_keep,
                          const int32_t* k_mid, uint8_t* labels, int32_t* row_src, int32_t* counts,
                          int32_t* cu_img, int32_t* tok_row, int B, int H, int W, int levels,
-                         cudaStream_t st) {
+                         int granular, cudaStream_t st) {
   const int N = H * W;
   const size_t sm1 = split_select_smem(N), sm2 = split_compact_smem(N);
   cudaError_t e = cudaFuncSetAttribute(split_select_kernel,
@@ -813,7 +888,7 @@ cudaError_t launch_split(const float* score, const uint8_t* mask, const int32_t*
   if (e != cudaSuccess) return e;
   const int fused = B == 1 ? 1 : 0;
   e = launch_pdl(split_select_kernel, dim3(B), dim3(SPLIT_THREADS), sm1, st, score, mask, k_keep,
-                 k_mid, labels, counts, H, W, levels, fused, cu_img, row_src, tok_row);
+                 k_mid, labels, counts, H, W, levels, granular, fused, cu_img, row_src, tok_row);
   if (e != cudaSuccess || fused) return e;
   return launch_pdl(split_compact_kernel, dim3(B), dim3(SPLIT_THREADS), sm2, st,
                     static_cast<const uint8_t*>(labels), static_cast<const int32_t*>(counts), cu_img,
@@ -832,6 +907,14 @@ cudaError_t launch_pack(const void* x, const uint8_t* labels, const int32_t* row
 cudaError_t launch_unpack(const float* out_img, const int32_t* tok_row, float* y, long long ntok,
                           int d, int num_sms, cudaStream_t st) {
   return launch_pdl(unpack_kernel, dim3(grid_for(ntok, 8, num_sms, 8)), dim3(256), 0, st, out_img,
+                    tok_row, y, ntok, d);
+}
+
+cudaError_t launch_unpack_delta(const float* out_img, const void* packed, const void* x,
+                                const uint8_t* labels, const int32_t* tok_row, float* y, long long ntok,
+                                int d, int num_sms, cudaStream_t st) {
+  return launch_pdl(unpack_delta_kernel, dim3(grid_for(ntok, 8, num_sms, 8)), dim3(256), 0, st, out_img,
+                    static_cast<const __nv_bfloat16*>(packed), static_cast<const __nv_bfloat16*>(x), labels,
                     tok_row, y, ntok, d);
 }
 

@@ -50,7 +50,8 @@ EXPORTS = ("hilo_status_string", "hilo_last_error", "hilo_sync_status", "hilo_de
            "hilo_score", "hilo_split_workspace_bytes", "hilo_split", "hilo_pack",
            "hilo_block_workspace_bytes", "hilo_block_forward", "hilo_unpack", "hilo_unpack_update",
            "hilo_convert_bf16_to_f16", "hilo_set_stage_events", "hilo_launch_count",
-           "hilo_block_forward_static_ws", "hilo_sobel_workspace_bytes", "hilo_sobel_select")
+           "hilo_block_forward_static_ws", "hilo_sobel_workspace_bytes", "hilo_sobel_select",
+           "hilo_split_regions", "hilo_unpack_delta")
 
 _lib = None
 
@@ -92,6 +93,8 @@ def lib() -> ctypes.CDLL:
         "hilo_launch_count": (ctypes.c_ulonglong, []),
         "hilo_sobel_workspace_bytes": (S, [shp]),
         "hilo_sobel_select": (I, [shp, P, I, I, P, I, F, P, P, S, P]),
+        "hilo_split_regions": (I, [shp, P, P, P, P, spo, P, S, P]),
+        "hilo_unpack_delta": (I, [shp, P, P, P, spo, P, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -243,6 +246,15 @@ def hilo_split(shape: Shape, score, mask, k_keep, k_mid, out: SplitBuffers, ws=N
                                           ctypes.byref(o), _ptr(ws), ws_bytes, _stream(stream)))
 
 
+def hilo_split_regions(shape: Shape, score, mask, k_keep, k_mid, out: SplitBuffers, ws=None, ws_bytes=0,
+                       stream=None) -> None:
+    s = shape.c()
+    o = out.c()
+    _check("hilo_split_regions", lib().hilo_split_regions(ctypes.byref(s), _ptr(score), _ptr(mask), _ptr(k_keep),
+                                                          _ptr(k_mid), ctypes.byref(o), _ptr(ws), ws_bytes,
+                                                          _stream(stream)))
+
+
 def hilo_sobel_workspace_bytes(shape: Shape) -> int:
     s = shape.c()
     return int(lib().hilo_sobel_workspace_bytes(ctypes.byref(s)))
@@ -292,6 +304,13 @@ def hilo_unpack(shape: Shape, out_img, split: SplitBuffers, y, stream=None) -> N
     o = split.c()
     _check("hilo_unpack", lib().hilo_unpack(ctypes.byref(s), _ptr(out_img), ctypes.byref(o), _ptr(y),
                                             _stream(stream)))
+
+
+def hilo_unpack_delta(shape: Shape, out_img, packed, x, split: SplitBuffers, y, stream=None) -> None:
+    s = shape.c()
+    o = split.c()
+    _check("hilo_unpack_delta", lib().hilo_unpack_delta(ctypes.byref(s), _ptr(out_img), _ptr(packed), _ptr(x),
+                                                        ctypes.byref(o), _ptr(y), _stream(stream)))
 
 
 def hilo_unpack_update(shape: Shape, out_img, split: SplitBuffers, x, alpha: float, stream=None) -> None:
@@ -346,14 +365,21 @@ class HotPath:
     def out_img(self) -> torch.Tensor:
         return self.out[self.shape.B * self.shape.T:]
 
-    def run(self, x, text, mask, k_keep, k_mid, stream=None, unpack: bool = True) -> None:
+    def run(self, x, text, mask, k_keep, k_mid, stream=None, unpack: bool = True, regions: bool = False) -> None:
+        """One pass. regions=True takes the window-granular split and the
+        delta unpool instead of the token-granular split and the nearest
+        unpool."""
         sh = self.shape
         hilo_score(sh, x, self.score, stream)
-        hilo_split(sh, self.score, mask, k_keep, k_mid, self.split, None, 0, stream)
+        (hilo_split_regions if regions else hilo_split)(sh, self.score, mask, k_keep, k_mid, self.split, None, 0,
+                                                        stream)
         hilo_pack(sh, x, self.split, self.packed, self.cap, stream)
         self.blocks(text, self.packed, HILO_BF16, stream)
         if unpack:
-            hilo_unpack(sh, self.out_img, self.split, self.y, stream)
+            if regions:
+                hilo_unpack_delta(sh, self.out_img, self.packed, x, self.split, self.y, stream)
+            else:
+                hilo_unpack(sh, self.out_img, self.split, self.y, stream)
 
     def blocks(self, in_txt, in_img, in_dtype, stream=None) -> None:
         sh = self.shape

@@ -82,6 +82,24 @@ def test_null_pointers_rejected(H):
     assert L.hilo_block_forward(ctypes.byref(s), ctypes.byref(w), 1, 64, 1, 1, 0, 1, 1, 1 << 30, None) == -1
 
 
+def test_regions_entry_points_check_arguments(H):
+    """hilo_split_regions validates like hilo_split; hilo_unpack_delta rejects
+    NULL and unaligned pointers before any launch."""
+    s = H.hilo_shape(1, 8, 8, 128, 4, 1, 1, 1)
+    L = H.lib()
+    sp = H.hilo_split_out()
+    assert L.hilo_split_regions(ctypes.byref(s), 1, 1, 1, 1, ctypes.byref(sp), None, 0, None) == -1
+    bad = H.hilo_shape(1, 7, 8, 128, 4, 1, 1, 1)
+    for f in ("labels", "row_src", "counts", "cu_img", "tok_row"):
+        setattr(sp, f, 256)
+    assert L.hilo_split_regions(ctypes.byref(bad), 1, 1, 1, 1, ctypes.byref(sp), None, 0, None) == -2
+    s2 = H.hilo_shape(1, 8, 8, 128, 4, 1, 1, 2)
+    assert L.hilo_split_regions(ctypes.byref(s2), 1, 1, 1, None, ctypes.byref(sp), None, 0, None) == -1
+    assert L.hilo_unpack_delta(ctypes.byref(s), 256, None, 256, ctypes.byref(sp), 256, None) == -1
+    assert L.hilo_unpack_delta(ctypes.byref(s), 260, 256, 256, ctypes.byref(sp), 256, None) == -1
+    assert L.hilo_unpack_delta(ctypes.byref(s), 256, 256, 264, ctypes.byref(sp), 256, None) == -1
+
+
 def test_workspace_size_and_check(H):
     s = H.hilo_shape(2, 64, 64, 3072, 512, 24, 1, 1)
     cap = 2 * 4096
