@@ -26,6 +26,11 @@ the DiT it feeds; the concrete variant -- token-space score, top-k split,
           softmax attention, tanh-GELU 4x MLP, residual adds.
   unpack  every grid token reads the output row of its kept token or of its
           window (nearest broadcast).
+  row_sizes, block(n_img=...)  proportional attention for pooled tokens:
+          a packed row standing for n grid tokens adds ln(n) to its logits as
+          a key, i.e. it draws the attention of n identical copies (the
+          paper is silent on how pooled tokens attend; this is the reading
+          that keeps the attention mass of the uncompressed sequence).
   split(granular=True), unpack_delta  the window-granular (regionalised)
           split -- each pooling window takes the finest class of any member,
           so kept regions are whole 2x2 windows and every pooled window is
@@ -265,9 +270,15 @@ def gelu_tanh(z: np.ndarray) -> np.ndarray:
     return 0.5 * z * (1.0 + np.tanh(math.sqrt(2.0 / math.pi) * (z + 0.044715 * z ** 3)))
 
 
-def softmax_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray) -> np.ndarray:
-    """Non-causal softmax attention of one head, scale 1/sqrt(head_dim)."""
+def softmax_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, key_n=None) -> np.ndarray:
+    """Non-causal softmax attention of one head, scale 1/sqrt(head_dim).
+
+    key_n (optional, one positive weight per key) is proportional attention:
+    ln(key_n[j]) is added to every logit of key j, so a key standing for n
+    tokens receives the attention mass of n identical copies of itself."""
     sc = (q @ k.T) / math.sqrt(q.shape[-1])
+    if key_n is not None:
+        sc = sc + np.log(np.asarray(key_n, dtype=np.float64))[None, :]
     sc = sc - sc.max(axis=-1, keepdims=True)
     p = np.exp(sc)
     p = p / p.sum(axis=-1, keepdims=True)
@@ -300,13 +311,15 @@ def _as_f64(u) -> np.ndarray:
     return bf16_to_f32(u).astype(np.float64) if u.dtype == np.uint16 else np.asarray(u, np.float64)
 
 
-def block(u_txt, u_img, cu_img, T: int, weights, heads: int, mlp: bool):
+def block(u_txt, u_img, cu_img, T: int, weights, heads: int, mlp: bool, n_img=None):
     """One MMDiT block on the joint sequence of each image.
 
     u_txt: [B*T, d] text rows (image b owns rows b*T .. b*T+T-1);
     u_img: [rows, d] packed image rows (image b owns cu_img[b] .. cu_img[b+1]-1).
     Either may be bf16 bits (uint16) or floats. Returns fp64 (txt, img).
     ``weights`` has ``.txt`` and ``.img`` with PyTorch-layout [out, in] arrays.
+    n_img (optional): proportional attention, the number of grid tokens each
+    packed image row stands for (text keys count 1), see softmax_attention.
     """
     ut = _as_f64(u_txt)
     ui = _as_f64(u_img)
@@ -320,10 +333,11 @@ def block(u_txt, u_img, cu_img, T: int, weights, heads: int, mlp: bool):
         t0, t1 = b * T, (b + 1) * T
         i0, i1 = int(cu_img[b]), int(cu_img[b + 1])
         joint = np.concatenate([qkv[0][t0:t1], qkv[1][i0:i1]], axis=0)
+        kn = None if n_img is None else np.concatenate([np.ones(T), np.asarray(n_img[i0:i1], np.float64)])
         o = np.empty((joint.shape[0], d))
         for h in range(heads):
             c = slice(h * hd, (h + 1) * hd)
-            o[:, c] = softmax_attention(joint[:, c], joint[:, d:][:, c], joint[:, 2 * d:][:, c])
+            o[:, c] = softmax_attention(joint[:, c], joint[:, d:][:, c], joint[:, 2 * d:][:, c], kn)
         att[0][t0:t1] = o[:T]
         att[1][i0:i1] = o[T:]
     out = []
@@ -336,7 +350,7 @@ def block(u_txt, u_img, cu_img, T: int, weights, heads: int, mlp: bool):
 
 
 def block_rows(u_txt, u_img, cu_img, T: int, weights, heads: int, mlp: bool, b: int,
-               txt_rows, img_rows):
+               txt_rows, img_rows, n_img=None):
     """The block's outputs for selected rows of image ``b`` only.
 
     Same arithmetic as ``block``; keys and values of the whole joint sequence
@@ -354,6 +368,7 @@ def block_rows(u_txt, u_img, cu_img, T: int, weights, heads: int, mlp: bool, b: 
     ln_i = layer_norm(ui[i0:i1])
     kv = np.concatenate([ln_t @ _w(wt.w_qkv[d:]).T + _w(wt.b_qkv[d:]),
                          ln_i @ _w(wi.w_qkv[d:]).T + _w(wi.b_qkv[d:])], axis=0)
+    kn = None if n_img is None else np.concatenate([np.ones(t1 - t0), np.asarray(n_img[i0:i1], np.float64)])
     res = []
     for rows, u_all, w in ((np.asarray(txt_rows, int), ut, wt), (np.asarray(img_rows, int), ui, wi)):
         if rows.size == 0:
@@ -364,7 +379,7 @@ def block_rows(u_txt, u_img, cu_img, T: int, weights, heads: int, mlp: bool, b: 
         o = np.empty((len(rows), d))
         for h in range(heads):
             c = slice(h * hd, (h + 1) * hd)
-            o[:, c] = softmax_attention(q[:, c], kv[:, :d][:, c], kv[:, d:][:, c])
+            o[:, c] = softmax_attention(q[:, c], kv[:, :d][:, c], kv[:, d:][:, c], kn)
         u = u + o @ _w(w.w_o).T + _w(w.b_o)
         if mlp:
             u = u + gelu_tanh(layer_norm(u) @ _w(w.w_1).T + _w(w.b_1)) @ _w(w.w_2).T + _w(w.b_2)
@@ -383,6 +398,15 @@ def block_dense(x_bits, text_bits, weights, heads: int, mlp: bool):
 # ---------------------------------------------------------------------------
 # Step 5: unpack, and the denoising-loop update
 # ---------------------------------------------------------------------------
+
+
+def row_sizes(sp: Split) -> np.ndarray:
+    """Number of grid tokens each packed image row stands for: 1 for a kept
+    token, the number of its class members for a pooled window (fp32)."""
+    n = np.zeros(int(sp.cu_img[-1]), dtype=np.float32)
+    for b in range(sp.labels.shape[0]):
+        np.add.at(n, sp.tok_row[b], np.float32(1.0))
+    return n
 
 
 def unpack(out_img: np.ndarray, sp: Split) -> np.ndarray:
@@ -479,9 +503,11 @@ def sobel_select(img: np.ndarray, mask: np.ndarray, H: int, W: int, patch: int, 
     return (hf | (dilate_mask(mask, H, W, radius) != 0)).astype(np.uint8)
 
 
-def hot_path(x_bits, text_bits, mask, k_keep, k_mid, levels, weights_list, heads, mlp, regions=False):
+def hot_path(x_bits, text_bits, mask, k_keep, k_mid, levels, weights_list, heads, mlp, regions=False,
+             prop=False):
     """score -> split -> pack -> blocks -> unpack for one batch; regions=True
-    takes the window-granular split and the delta unpool.
+    takes the window-granular split and the delta unpool, prop=True
+    proportional attention (each packed row weighted by its row size).
 
     Returns (split, packed, (txt_out, img_out), y) with the block outputs in fp64.
     """
@@ -490,7 +516,8 @@ def hot_path(x_bits, text_bits, mask, k_keep, k_mid, levels, weights_list, heads
     sp = split(score(x_bits), mask, k_keep, k_mid, H, W, levels, granular=regions)
     packed = pack(x_bits, sp)
     ut, ui = text_bits.reshape(B * T, d), packed
+    n_img = row_sizes(sp) if prop else None
     for wts in weights_list:
-        ut, ui = block(ut, ui, sp.cu_img, T, wts, heads, mlp)
+        ut, ui = block(ut, ui, sp.cu_img, T, wts, heads, mlp, n_img)
     y = unpack_delta(ui, packed, x_bits, sp) if regions else unpack(ui, sp)
     return sp, packed, (ut, ui), y

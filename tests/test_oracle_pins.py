@@ -548,6 +548,81 @@ def test_block_permutation_equivariance():
     assert np.allclose(op, oi[perm], rtol=0, atol=1e-10)
 
 
+def test_proportional_attention_equals_duplicated_keys():
+    """A key with weight n attends exactly like n identical copies of it."""
+    rng = np.random.default_rng(30)
+    q = rng.standard_normal((7, 16))
+    k = rng.standard_normal((9, 16)) * 2
+    v = rng.standard_normal((9, 16))
+    n = rng.integers(1, 6, size=9)
+    got = O.softmax_attention(q, k, v, n)
+    ref = O.softmax_attention(q, np.repeat(k, n, axis=0), np.repeat(v, n, axis=0))
+    assert np.allclose(got, ref, rtol=0, atol=1e-12)
+    # two keys, equal logits: the weights split n0 : n1
+    q2 = np.zeros((1, 4))
+    k2 = rng.standard_normal((2, 4))
+    v2 = np.array([[1.0, 0, 0, 0], [0, 1.0, 0, 0]])
+    o = O.softmax_attention(q2, k2, v2, [3, 1])
+    assert np.allclose(o[0, :2], [0.75, 0.25], rtol=0, atol=1e-15)
+
+
+def test_block_proportional_ones_is_plain_block():
+    rng = np.random.default_rng(31)
+    d, heads, T = 32, 2, 4
+    w = _rand_weights(rng, d, mlp=True)
+    ut = bits(rng.standard_normal((2 * T, d)))
+    ui = bits(rng.standard_normal((13, d)))
+    cu = [0, 6, 13]
+    a = O.block(ut, ui, cu, T, w, heads, True)
+    b = O.block(ut, ui, cu, T, w, heads, True, n_img=np.ones(13, np.float32))
+    assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
+
+
+def test_block_proportional_equals_block_on_duplicated_rows():
+    """The whole block with row weights n equals the plain block on the
+    sequence where image row r appears n_r times (its first copy's output,
+    and every text output, agree), for two images of one batch."""
+    rng = np.random.default_rng(32)
+    d, heads, T = 32, 2, 3
+    w = _rand_weights(rng, d, mlp=True)
+    ut = bits(rng.standard_normal((2 * T, d)))
+    ui = bits(rng.standard_normal((9, d)))
+    cu = [0, 5, 9]
+    n = np.array([1, 3, 1, 2, 4, 2, 1, 1, 3], dtype=np.float32)
+    pt, pi = O.block(ut, ui, cu, T, w, heads, True, n_img=n)
+    rep = np.repeat(np.arange(9), n.astype(int))
+    cu_dup = [0, int(n[:5].sum()), int(n.sum())]
+    dt, di = O.block(ut, ui[rep], cu_dup, T, w, heads, True)
+    first = np.searchsorted(rep, np.arange(9))
+    assert np.allclose(pt, dt, rtol=0, atol=1e-10)
+    assert np.allclose(pi, di[first], rtol=0, atol=1e-10)
+    # the sampled-rows form agrees with the whole block
+    rt, ri = O.block_rows(ut, ui, cu, T, w, heads, True, 1, [3, 5], [6, 8], n_img=n)
+    assert np.allclose(rt, pt[[3, 5]], rtol=0, atol=1e-12) and np.allclose(ri, pi[[6, 8]], rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("granular", [False, True])
+def test_row_sizes_count_the_grid(granular):
+    rng = np.random.default_rng(33)
+    H, W, B = 8, 12, 2
+    N = H * W
+    s = rng.random((B, N)).astype(np.float32)
+    m = (rng.random((B, N)) < 0.1).astype(np.uint8)
+    sp = O.split(s, m, [10, 30], [20, 10], H, W, 2, granular=granular)
+    n = O.row_sizes(sp)
+    for b in range(B):
+        r0, r1 = int(sp.cu_img[b]), int(sp.cu_img[b + 1])
+        assert n[r0:r1].sum() == N
+        nk, n2, n4 = (int(c) for c in sp.counts[b])
+        assert np.all(n[r0:r0 + nk] == 1)
+        for r in range(r0 + nk, r1):
+            size, cls = (2, O.POOL2) if r < r0 + nk + n2 else (4, O.POOL4)
+            mem = O.window_members(int(sp.row_src[r]), size, W)
+            assert n[r] == sum(1 for t in mem if sp.labels[b, t] == cls)
+            if granular:
+                assert n[r] == size * size
+
+
 def test_keep_ratio_one_is_dense_block():
     wl = I.tiny_layer(keep_ratio=1024, H=16, W=16, d=64, heads=2, T=8)
     b = I.make_batch(wl)
