@@ -350,6 +350,35 @@ def time_regions(H, torch, stream, wl, hp, inputs, hbm_peak: float, steps: int) 
             "unpack_nearest_ms_same_split": nearest_ms}
 
 
+def time_prop(H, torch, stream, wl, hp, dw, inputs, steps: int) -> dict:
+    """Proportional attention on the timed workload: the hot path with it,
+    and the block alone with and without it on the same packed rows."""
+    x, text, mask, kk, km = inputs
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for _ in range(steps):
+            fn()
+        s1.record(stream)
+        torch.cuda.synchronize()
+        return s0.elapsed_time(s1) / steps
+
+    path_ms = timed(lambda: hp.run(x, text, mask, kk, km, prop=True))
+    H.hilo_sync_status()
+    sh, cu = hp.shape, hp.split.cu_img
+    plain = timed(lambda: H.hilo_block_forward(sh, dw, cu, hp.cap, text, hp.packed, H.HILO_BF16, hp.out, hp.ws,
+                                               hp.ws_bytes, stream))
+    prop = timed(lambda: H.hilo_block_forward_prop(sh, dw, cu, hp.cap, text, hp.packed, H.HILO_BF16, hp.n_img,
+                                                   hp.out, hp.ws, hp.ws_bytes, stream))
+    H.hilo_sync_status()
+    return {"hot_path_ms": path_ms, "image_tokens_per_s": wl.B * wl.N / (path_ms * 1e-3),
+            "block_ms_prop": prop, "block_ms_plain_same_rows": plain, "block_overhead": prop / plain - 1.0}
+
+
 def time_configs(H, I, torch, stream, steps: int):
     """Hot path, compressed block and dense block of each workload configuration.
 
@@ -654,6 +683,7 @@ def run_hilo(args):
         extras["sweep"] = sweep
         extras["sobel_selector"] = time_sobel_selector(H, I, torch, stream, wl, batch, hp, hbm_peak, Ks)
         extras["regions"] = time_regions(H, torch, stream, wl, hp, (x, text, mask, kk, km), hbm_peak, Ks)
+        extras["proportional_attention"] = time_prop(H, torch, stream, wl, hp, dw, (x, text, mask, kk, km), Ks)
         if world == 1:
             extras["configs"] = time_configs(H, I, torch, stream, steps=20)
         # dense block: every grid token is its own row, no score/split/pack/unpack

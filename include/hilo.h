@@ -269,6 +269,34 @@ int hilo_block_forward(const hilo_shape* shape, const hilo_block_weights* weight
                        size_t ws_bytes, void* stream);
 
 /*
+ * hilo_row_sizes -- the number of grid tokens each packed image row stands
+ * for: 1 for a kept token, the number of its class members for a pooled
+ * window. These are the weights of proportional attention.
+ *   split  outputs of hilo_split or hilo_split_regions
+ *   n_img  fp32 [cap] device; rows [0, cu_img[B]) are written
+ */
+int hilo_row_sizes(const hilo_shape* shape, const hilo_split_out* split, float* n_img, int32_t cap,
+                   void* stream);
+
+/*
+ * hilo_block_forward_prop -- hilo_block_forward with proportional attention
+ * for pooled tokens: as a key, packed image row r adds ln(n_img[r]) to its
+ * logits (text keys add 0), so a row standing for n grid tokens draws the
+ * attention of n identical copies of itself:
+ *     softmax_j(s_ij + ln n_j) = n_j e^(s_ij) / sum_k n_k e^(s_ik).
+ * The paper does not say how pooled tokens attend; this weighting keeps the
+ * attention mass of the uncompressed sequence. The kernel multiplies each
+ * probability by n_j before the row sum and the bf16 rounding of P.
+ *   n_img  fp32 [cap] device, 4-byte aligned, positive; e.g. hilo_row_sizes
+ * Other arguments, layouts and errors as hilo_block_forward (HILO_ERR_ARG
+ * for a NULL or unaligned n_img).
+ */
+int hilo_block_forward_prop(const hilo_shape* shape, const hilo_block_weights* weights,
+                            const int32_t* cu_img, int32_t cap, const void* in_txt,
+                            const void* in_img, int in_dtype, const float* n_img, float* out,
+                            void* ws, size_t ws_bytes, void* stream);
+
+/*
  * hilo_unpack -- back to the full grid (nearest broadcast): every token reads
  * the block output of its kept row or of its window's row.
  *   out_img  fp32 [cap, d]  image rows of the block output (out + B*T*d)

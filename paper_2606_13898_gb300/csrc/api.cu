@@ -314,9 +314,11 @@ size_t hilo_block_workspace_bytes(const hilo_shape* shape, int32_t cap) {
   return block_ws_layout(shape, cap).total;
 }
 
-int hilo_block_forward(const hilo_shape* shape, const hilo_block_weights* w, const int32_t* cu_img,
-                       int32_t cap, const void* in_txt, const void* in_img, int in_dtype,
-                       float* out, void* ws, size_t ws_bytes, void* stream) {
+// The block of hilo_block_forward; n_img != NULL selects proportional
+// attention (hilo_block_forward_prop).
+static int block_forward_impl(const hilo_shape* shape, const hilo_block_weights* w, const int32_t* cu_img,
+                              int32_t cap, const void* in_txt, const void* in_img, int in_dtype,
+                              const float* n_img, float* out, void* ws, size_t ws_bytes, void* stream) {
   int st = check_shape(shape, true);
   if (st) return st;
   if (!w || !cu_img || !in_img || !out) return fail(HILO_ERR_ARG, "hilo_block_forward: NULL pointer");
@@ -388,6 +390,7 @@ int hilo_block_forward(const hilo_shape* shape, const hilo_block_weights* w, con
   aa.qkv = qkv;
   aa.out = attn;
   aa.cu_img = cu_img;
+  aa.n_img = n_img;
   aa.B = B;
   aa.T = T;
   aa.heads = shape->heads;
@@ -417,6 +420,39 @@ int hilo_block_forward(const hilo_shape* shape, const hilo_block_weights* w, con
     stage_mark(7, s);
   }
   return HILO_OK;
+}
+
+int hilo_block_forward(const hilo_shape* shape, const hilo_block_weights* w, const int32_t* cu_img,
+                       int32_t cap, const void* in_txt, const void* in_img, int in_dtype,
+                       float* out, void* ws, size_t ws_bytes, void* stream) {
+  return block_forward_impl(shape, w, cu_img, cap, in_txt, in_img, in_dtype, nullptr, out, ws, ws_bytes,
+                            stream);
+}
+
+int hilo_block_forward_prop(const hilo_shape* shape, const hilo_block_weights* w, const int32_t* cu_img,
+                            int32_t cap, const void* in_txt, const void* in_img, int in_dtype,
+                            const float* n_img, float* out, void* ws, size_t ws_bytes, void* stream) {
+  if (!n_img) return fail(HILO_ERR_ARG, "hilo_block_forward_prop: n_img is NULL");
+  if (reinterpret_cast<uintptr_t>(n_img) & 3)
+    return fail(HILO_ERR_ARG, "hilo_block_forward_prop: n_img must be 4-byte aligned");
+  return block_forward_impl(shape, w, cu_img, cap, in_txt, in_img, in_dtype, n_img, out, ws, ws_bytes,
+                            stream);
+}
+
+int hilo_row_sizes(const hilo_shape* shape, const hilo_split_out* split, float* n_img, int32_t cap,
+                   void* stream) {
+  int st = check_shape(shape, false);
+  if (st) return st;
+  if ((st = check_split(split))) return st;
+  if (!n_img) return fail(HILO_ERR_ARG, "hilo_row_sizes: NULL pointer");
+  if (cap < 0) return fail(HILO_ERR_ARG, "hilo_row_sizes: cap=%d", cap);
+  DevInfo* dev;
+  if ((st = current_device(&dev))) return st;
+  cudaError_t e = hilo::launch_row_sizes(split->labels, split->row_src, split->counts, split->cu_img, n_img,
+                                         shape->B, shape->H, shape->W, cap, dev->num_sms,
+                                         static_cast<cudaStream_t>(stream));
+  if (e == cudaSuccess && cap > 0) count(1);
+  return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_row_sizes");
 }
 
 int hilo_unpack(const hilo_shape* shape, const float* out_img, const hilo_split_out* split, float* y,

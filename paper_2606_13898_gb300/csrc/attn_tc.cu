@@ -27,6 +27,15 @@
 // row's running maximum grows by more than 2^8 (until then the
 // probabilities are formed against the older, smaller maximum, so they stay
 // <= 256, well inside bf16 range).
+// With proportional attention (PROP) every key j carries a weight n_j (the
+// number of grid tokens a packed image row stands for; text keys weigh 1):
+// softmax(s + ln n) = n e^s / sum(n e^s), so each probability is multiplied
+// by its key's weight before the row sum and the bf16 packing, and the row
+// maxima (the stabiliser) stay those of the raw logits. Each softmax warp
+// fetches the next key tile's 128 weights with asynchronous 4-byte copies
+// (zero-filled past the ragged end) into its own double-buffered shared slot
+// while it works on the current tile, and reads them back as 16-byte
+// broadcasts; no barrier spans warps.
 // Every mbarrier wait is bounded (error latched, TMEM freed, CTA returns).
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -55,7 +64,7 @@ constexpr uint32_t ATTN_TMEM_COLS = 512;  // S0 | S1 | O0 | O1
 constexpr int BOX_BYTES = 128 * 128;       // 128 rows x 64 16-bit elements
 constexpr float RESCALE_LOG2 = 8.0f;
 
-template <int HD>
+template <int HD, bool PROP>
 struct Cfg {
   static constexpr int NBOX = HD / 64;
   static constexpr int TILE_BYTES = NBOX * BOX_BYTES;  // 128 rows x HD
@@ -64,15 +73,56 @@ struct Cfg {
   static constexpr int OFF_K = 2 * TILE_BYTES;
   static constexpr int OFF_V = 4 * TILE_BYTES;
   static constexpr int DATA_BYTES = 6 * TILE_BYTES;
-  static constexpr int SMEM_BYTES = DATA_BYTES + 1024 + 256;
+  // barriers (256 B) and, with PROP, 8 softmax warps x 2 slots x 128 weights
+  static constexpr int OFF_W = DATA_BYTES + 256;
+  static constexpr int SMEM_BYTES = DATA_BYTES + 1024 + 256 + (PROP ? 8 * 2 * BKV * 4 : 0);
 };
 
 struct AttnParams {
   const int32_t* cu_img;
+  const float* n_img;  // PROP: weight of each packed image row
   __nv_bfloat16* out;
   int B, T, heads, d, qt_txt, pairs_max;
   float scale_log2;  // log2(e) / sqrt(head_dim)
 };
+
+// 4-byte asynchronous global -> shared copy; bytes past src_bytes (0 or 4)
+// are zero-filled
+__device__ __forceinline__ void cp_async4(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// Pairs of fp32 values in one 64-bit register pair: Blackwell's paired fp32
+// instructions (fma/mul/add .f32x2) apply the same IEEE operation to both
+// halves at one issue slot per pair.
+__device__ __forceinline__ uint64_t f2(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_split(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
 
 __device__ __forceinline__ float ex2(float x) {
   float y;
@@ -94,10 +144,10 @@ __device__ __forceinline__ void seq_tile(const AttnParams& p, int b, int L, int 
   }
 }
 
-template <int HD>
+template <int HD, bool PROP>
 __global__ void __launch_bounds__(ATTN_THREADS, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm, const __grid_constant__ AttnParams p) {
-  using C = Cfg<HD>;
+  using C = Cfg<HD, PROP>;
   pdl_trigger();
   pdl_wait();  // cu_img and q/k/v are written by the previous kernels
   // ---- work item: (image, head, query-tile pair)
@@ -316,23 +366,90 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
     const bool active = i == 0 || has1;
     float m = -INFINITY, l = 0.f;
     bool ok = active;
+    // PROP: key weights of tile tt into the warp's slot tt & 1 (text tiles
+    // weigh 1; columns past the ragged end 0), one commit group per call
+    float* wslots = reinterpret_cast<float*>(smem + C::OFF_W) + warp * 2 * BKV;
+    auto fetch_weights = [&](int tt) {
+      if (tt < nkv) {
+        float* wb = wslots + (tt & 1) * BKV;
+        if (tt < p.qt_txt) {
+#pragma unroll
+          for (int u = 0; u < 4; ++u) wb[lane + 32 * u] = 1.0f;
+        } else {
+          int r0, v;
+          seq_tile(p, b, L, tt, r0, v);
+          const float* src = p.n_img + (p.cu_img[b] + (tt - p.qt_txt) * BKV);
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int col = lane + 32 * u;
+            cp_async4(smem_u32(wb + col), col < v ? src + col : p.n_img, col < v ? 4u : 0u);
+          }
+        }
+      }
+      cp_async_commit();
+    };
+    // ragged key tile: rows past `valid` hold other tokens (or stale data);
+    // zero them in V so that the zero-probability columns add exactly 0.
+    // Returns false when the wait for V gave up.
+    auto zero_v_tail = [&](int t, int valid) -> bool {
+      if (i == 0 && valid < BKV) {
+        if (!mbar_wait_warp(&v_full[t & 1], static_cast<uint32_t>((t >> 1) & 1), abort_flag, err,
+                            DEV_TIMEOUT_ATTN + 256 * 11))
+          return false;
+        if (row >= valid) {
+          unsigned char* vr = sV(t & 1) + row * 128;
+#pragma unroll
+          for (int j = 0; j < C::NBOX; ++j)
+#pragma unroll
+            for (int c16 = 0; c16 < 8; ++c16)
+              *reinterpret_cast<uint4*>(vr + j * BOX_BYTES + c16 * 16) = make_uint4(0, 0, 0, 0);
+        }
+      }
+      return true;
+    };
+    // S_i(t) complete means every earlier MMA is too (PV_i(t-1) included),
+    // so O_i can be rescaled and P_i written over S_i without another wait.
+    // tcgen05.ld / tcgen05.st are warp-collective: the whole warp rescales
+    // when any of its rows needs it (rows that do not use alpha = 1)
+    auto rescale_o = [&](bool rescale, float m_use) {
+      if (__any_sync(0xffffffffu, rescale)) {
+        const float alpha = rescale ? ex2(m - m_use) : 1.0f;
+#pragma unroll 1
+        for (int c = 0; c < HD / 32; ++c) {
+          float o[32];
+          tmem_ld32(tO + c * 32, o);
+          tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < 32; ++j) o[j] *= alpha;
+          tmem_st32(tO + c * 32, o);
+        }
+        l *= alpha;
+      }
+    };
+    if (PROP && active) fetch_weights(0);
     for (int t = 0; t < nkv && ok; ++t) {
       int row0, valid;
       seq_tile(p, b, L, t, row0, valid);
       const uint32_t tp = static_cast<uint32_t>(t & 1);
+      if (PROP) {
+        // every lane is done with slot (t + 1) & 1 (read for tile t - 1)
+        // before the next tile's weights are fetched into it
+        __syncwarp();
+        fetch_weights(t + 1);
+      }
       if (!mbar_wait_warp(&s_full[i], tp, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 10)) {
         ok = false;
         break;
       }
       tc_fence_after();
+      // row max and row sum with 8 independent partials combined by a tree,
+      // so the reductions do not form one 128-long dependent chain; only the
+      // last key tile of a segment is ragged and needs masking
+      const bool full_tile = valid == BKV;
       float s[BKV];
 #pragma unroll
       for (int c = 0; c < BKV / 32; ++c) tmem_ld32(tS + c * 32, s + c * 32);
       tmem_ld_wait();
-      // row max and (below) row sum with 8 independent partials combined by
-      // a tree, so the reductions do not form one 128-long dependent chain;
-      // only the last key tile of a segment is ragged and needs masking
-      const bool full_tile = valid == BKV;
       float mx8[8];
 #pragma unroll
       for (int u = 0; u < 8; ++u) mx8[u] = -INFINITY;
@@ -356,58 +473,58 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
         rescale = true;
       }
       float ls8[8];
+      if (PROP) {
+        // probabilities by key pairs: exponent argument s*scale - m as one
+        // paired fma, two exp2, times the pair's weights (one paired mul);
+        // the row sum's partials (2u, 2u+1) for pair c with u = c mod 4 are
+        // the same partition and order as key j into partial j mod 8.
+        // Masked columns are 0, selected, never computed from their stale
+        // logits. First: this tile's weights have landed (all groups but the
+        // newest) and are visible to the whole warp.
+        cp_async_wait<1>();
+        __syncwarp();
+        const uint64_t* w2 = reinterpret_cast<const uint64_t*>(wslots + (t & 1) * BKV);
+        const uint64_t sc2 = f2(p.scale_log2, p.scale_log2), nm2 = f2(-m_use, -m_use);
+        uint64_t ls4[4];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) ls8[u] = 0.f;
-      if (full_tile) {
+        for (int u = 0; u < 4; ++u) ls4[u] = 0ull;
 #pragma unroll
-        for (int j = 0; j < BKV; ++j) {
-          const float pj = ex2(fmaf(s[j], p.scale_log2, -m_use));
-          s[j] = pj;
-          ls8[j & 7] += pj;
+        for (int c = 0; c < BKV / 2; ++c) {
+          float a, a1;
+          f2_split(f2_fma(f2(s[2 * c], s[2 * c + 1]), sc2, nm2), a, a1);
+          a = (full_tile || 2 * c < valid) ? ex2(a) : 0.f;
+          a1 = (full_tile || 2 * c + 1 < valid) ? ex2(a1) : 0.f;
+          const uint64_t pr = f2_mul(f2(a, a1), w2[c]);
+          f2_split(pr, s[2 * c], s[2 * c + 1]);
+          ls4[c & 3] = f2_add(ls4[c & 3], pr);
         }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) f2_split(ls4[u], ls8[2 * u], ls8[2 * u + 1]);
       } else {
 #pragma unroll
-        for (int j = 0; j < BKV; ++j) {
-          const float pj = j < valid ? ex2(fmaf(s[j], p.scale_log2, -m_use)) : 0.f;
-          s[j] = pj;
-          ls8[j & 7] += pj;
+        for (int u = 0; u < 8; ++u) ls8[u] = 0.f;
+        if (full_tile) {
+#pragma unroll
+          for (int j = 0; j < BKV; ++j) {
+            const float pj = ex2(fmaf(s[j], p.scale_log2, -m_use));
+            s[j] = pj;
+            ls8[j & 7] += pj;
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < BKV; ++j) {
+            const float pj = j < valid ? ex2(fmaf(s[j], p.scale_log2, -m_use)) : 0.f;
+            s[j] = pj;
+            ls8[j & 7] += pj;
+          }
         }
       }
       const float lsum = ((ls8[0] + ls8[1]) + (ls8[2] + ls8[3])) + ((ls8[4] + ls8[5]) + (ls8[6] + ls8[7]));
-      // ragged key tile: rows past `valid` hold other tokens (or stale data);
-      // zero them in V so that the zero-probability columns add exactly 0
-      if (i == 0 && valid < BKV) {
-        if (!mbar_wait_warp(&v_full[t & 1], static_cast<uint32_t>((t >> 1) & 1), abort_flag, err,
-                       DEV_TIMEOUT_ATTN + 256 * 11)) {
-          ok = false;
-          break;
-        }
-        if (row >= valid) {
-          unsigned char* vr = sV(t & 1) + row * 128;
-#pragma unroll
-          for (int j = 0; j < C::NBOX; ++j)
-#pragma unroll
-            for (int c16 = 0; c16 < 8; ++c16)
-              *reinterpret_cast<uint4*>(vr + j * BOX_BYTES + c16 * 16) = make_uint4(0, 0, 0, 0);
-        }
+      if (!zero_v_tail(t, valid)) {
+        ok = false;
+        break;
       }
-      // S_i(t) complete means every earlier MMA is too (PV_i(t-1) included),
-      // so O_i can be rescaled and P_i written over S_i without another wait.
-      // tcgen05.ld / tcgen05.st are warp-collective: the whole warp rescales
-      // when any of its rows needs it (rows that do not use alpha = 1)
-      if (__any_sync(0xffffffffu, rescale)) {
-        const float alpha = rescale ? ex2(m - m_use) : 1.0f;
-#pragma unroll 1
-        for (int c = 0; c < HD / 32; ++c) {
-          float o[32];
-          tmem_ld32(tO + c * 32, o);
-          tmem_ld_wait();
-#pragma unroll
-          for (int j = 0; j < 32; ++j) o[j] *= alpha;
-          tmem_st32(tO + c * 32, o);
-        }
-        l *= alpha;
-      }
+      rescale_o(rescale, m_use);
       m = m_use;
       l += lsum;
       // P_i as bf16 pairs (keys 2c, 2c+1 in column c) over the first 64
@@ -425,6 +542,7 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
       tc_fence_before();
       mbar_arrive(&p_full[i]);
     }
+    if (PROP) cp_async_wait<0>();  // no copy in flight when the CTA leaves
     if (ok && mbar_wait_warp(&o_done[i], static_cast<uint32_t>((nkv - 1) & 1), abort_flag, err,
                         DEV_TIMEOUT_ATTN + 256 * 14)) {
       tc_fence_after();
@@ -459,26 +577,27 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
   }
 }
 
-template <int HD>
+template <int HD, bool PROP>
 cudaError_t launch_hd(const AttnArgs& a, const AttnParams& p, int grid, cudaStream_t st) {
   CUtensorMap tm;
   if (!encode_tmap_bf16_2d(&tm, a.qkv, 3ull * a.d, a.R, 3ull * a.d, 64, 128))
     return cudaErrorInvalidValue;
-  cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       Cfg<HD>::SMEM_BYTES);
+  cudaError_t e = cudaFuncSetAttribute(attn_kernel<HD, PROP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       Cfg<HD, PROP>::SMEM_BYTES);
   if (e != cudaSuccess) return e;
   // the register split must fit what the CTA is launched with, or the
   // softmax warpgroups' setmaxnreg.inc would wait for registers forever
   static int regs = -1;
   if (regs < 0) {
     cudaFuncAttributes fa;
-    e = cudaFuncGetAttributes(&fa, attn_kernel<HD>);
+    e = cudaFuncGetAttributes(&fa, attn_kernel<HD, PROP>);
     if (e != cudaSuccess) return e;
     regs = fa.numRegs;
   }
   if (static_cast<long long>(regs) * ATTN_THREADS < 256LL * SOFTMAX_REGS + 128LL * CONTROL_REGS)
     return cudaErrorInvalidConfiguration;
-  return launch_pdl(attn_kernel<HD>, dim3(grid), dim3(ATTN_THREADS), Cfg<HD>::SMEM_BYTES, st, tm, p);
+  return launch_pdl(attn_kernel<HD, PROP>, dim3(grid), dim3(ATTN_THREADS), Cfg<HD, PROP>::SMEM_BYTES, st, tm,
+                    p);
 }
 
 }  // namespace
@@ -487,6 +606,7 @@ cudaError_t launch_attention(const AttnArgs& a, int num_sms, cudaStream_t st) {
   (void)num_sms;
   AttnParams p;
   p.cu_img = a.cu_img;
+  p.n_img = a.n_img;
   p.out = static_cast<__nv_bfloat16*>(a.out);
   p.B = a.B;
   p.T = a.T;
@@ -499,8 +619,13 @@ cudaError_t launch_attention(const AttnArgs& a, int num_sms, cudaStream_t st) {
   const long long items = static_cast<long long>(a.B) * a.heads * p.pairs_max;
   if (items <= 0) return cudaSuccess;
   if (items > 0x7fffffffLL) return cudaErrorInvalidValue;
-  if (a.head_dim == 128) return launch_hd<128>(a, p, static_cast<int>(items), st);
-  if (a.head_dim == 64) return launch_hd<64>(a, p, static_cast<int>(items), st);
+  if (a.n_img) {
+    if (a.head_dim == 128) return launch_hd<128, true>(a, p, static_cast<int>(items), st);
+    if (a.head_dim == 64) return launch_hd<64, true>(a, p, static_cast<int>(items), st);
+    return cudaErrorInvalidValue;
+  }
+  if (a.head_dim == 128) return launch_hd<128, false>(a, p, static_cast<int>(items), st);
+  if (a.head_dim == 64) return launch_hd<64, false>(a, p, static_cast<int>(items), st);
   return cudaErrorInvalidValue;
 }
 

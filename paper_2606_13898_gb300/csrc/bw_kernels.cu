@@ -651,6 +651,40 @@ __global__ void __launch_bounds__(256) pack_kernel(const __nv_bfloat16* __restri
   }
 }
 
+// Number of grid tokens each packed image row stands for: 1 for a kept
+// token, the count of its class members for a pooled window (the weights of
+// proportional attention). One thread per row of the capacity.
+__global__ void __launch_bounds__(256) row_sizes_kernel(const uint8_t* __restrict__ labels,
+                                                        const int32_t* __restrict__ row_src,
+                                                        const int32_t* __restrict__ counts,
+                                                        const int32_t* __restrict__ cu_img,
+                                                        float* __restrict__ n_img, int B, int H, int W,
+                                                        int cap) {
+  pdl_trigger();
+  pdl_wait();
+  const int N = H * W;
+  const int total = min(cu_img[B], cap);
+  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < total; r += gridDim.x * blockDim.x) {
+    int b = 0;
+    while (b + 1 < B && cu_img[b + 1] <= r) ++b;
+    const int local = r - cu_img[b];
+    const int nk = counts[3 * b], n2 = counts[3 * b + 1];
+    if (local < nk) {
+      n_img[r] = 1.0f;
+      continue;
+    }
+    const int size = local < nk + n2 ? 2 : 4;
+    const uint8_t cls = size == 2 ? HILO_LABEL_POOL2 : HILO_LABEL_POOL4;
+    const int src = row_src[r];
+    const int Wn = W / size;
+    const uint8_t* lab = labels + static_cast<long long>(b) * N + (size * (src / Wn)) * W + size * (src % Wn);
+    int c = 0;
+    for (int i = 0; i < size; ++i)
+      for (int j = 0; j < size; ++j) c += lab[i * W + j] == cls ? 1 : 0;
+    n_img[r] = static_cast<float>(c);
+  }
+}
+
 // ============================================================= unpack =====
 
 __global__ void __launch_bounds__(256) unpack_kernel(const float* __restrict__ out_img,
@@ -908,6 +942,14 @@ cudaError_t launch_unpack(const float* out_img, const int32_t* tok_row, float* y
                           int d, int num_sms, cudaStream_t st) {
   return launch_pdl(unpack_kernel, dim3(grid_for(ntok, 8, num_sms, 8)), dim3(256), 0, st, out_img,
                     tok_row, y, ntok, d);
+}
+
+cudaError_t launch_row_sizes(const uint8_t* labels, const int32_t* row_src, const int32_t* counts,
+                             const int32_t* cu_img, float* n_img, int B, int H, int W, int cap, int num_sms,
+                             cudaStream_t st) {
+  if (cap <= 0) return cudaSuccess;
+  return launch_pdl(row_sizes_kernel, dim3(grid_for(cap, 256, num_sms, 4)), dim3(256), 0, st, labels, row_src,
+                    counts, cu_img, n_img, B, H, W, cap);
 }
 
 cudaError_t launch_unpack_delta(const float* out_img, const void* packed, const void* x,

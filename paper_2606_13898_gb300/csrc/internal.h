@@ -26,6 +26,9 @@ cudaError_t launch_pack(const void* x, const uint8_t* labels, const int32_t* row
                         int W, int d, int cap, int num_sms, cudaStream_t st);
 cudaError_t launch_unpack(const float* out_img, const int32_t* tok_row, float* y, long long ntok,
                           int d, int num_sms, cudaStream_t st);
+cudaError_t launch_row_sizes(const uint8_t* labels, const int32_t* row_src, const int32_t* counts,
+                             const int32_t* cu_img, float* n_img, int B, int H, int W, int cap, int num_sms,
+                             cudaStream_t st);
 cudaError_t launch_unpack_delta(const float* out_img, const void* packed, const void* x,
                                 const uint8_t* labels, const int32_t* tok_row, float* y, long long ntok,
                                 int d, int num_sms, cudaStream_t st);
@@ -91,6 +94,7 @@ struct AttnArgs {
   const void* qkv;  // bf16 [R, 3d]
   void* out;        // bf16 [R, d]
   const int32_t* cu_img;
+  const float* n_img = nullptr;  // proportional attention: weight per packed image row
   int B, T, heads, head_dim, d, R, max_img_rows;
 };
 cudaError_t launch_attention(const AttnArgs& a, int num_sms, cudaStream_t st);

@@ -51,7 +51,7 @@ EXPORTS = ("hilo_status_string", "hilo_last_error", "hilo_sync_status", "hilo_de
            "hilo_block_workspace_bytes", "hilo_block_forward", "hilo_unpack", "hilo_unpack_update",
            "hilo_convert_bf16_to_f16", "hilo_set_stage_events", "hilo_launch_count",
            "hilo_block_forward_static_ws", "hilo_sobel_workspace_bytes", "hilo_sobel_select",
-           "hilo_split_regions", "hilo_unpack_delta")
+           "hilo_split_regions", "hilo_unpack_delta", "hilo_row_sizes", "hilo_block_forward_prop")
 
 _lib = None
 
@@ -95,6 +95,9 @@ def lib() -> ctypes.CDLL:
         "hilo_sobel_select": (I, [shp, P, I, I, P, I, F, P, P, S, P]),
         "hilo_split_regions": (I, [shp, P, P, P, P, spo, P, S, P]),
         "hilo_unpack_delta": (I, [shp, P, P, P, spo, P, P]),
+        "hilo_row_sizes": (I, [shp, spo, P, ctypes.c_int32, P]),
+        "hilo_block_forward_prop": (I, [shp, ctypes.POINTER(hilo_block_weights), P, ctypes.c_int32, P, P, I,
+                                        P, P, P, S, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -289,6 +292,22 @@ def hilo_block_forward(shape: Shape, weights: DeviceWeights, cu_img, cap: int, i
         _ptr(ws), ws_bytes, _stream(stream)))
 
 
+def hilo_block_forward_prop(shape: Shape, weights: DeviceWeights, cu_img, cap: int, in_txt, in_img, in_dtype: int,
+                            n_img, out, ws, ws_bytes: int, stream=None) -> None:
+    s = shape.c()
+    w = weights.c()
+    _check("hilo_block_forward_prop", lib().hilo_block_forward_prop(
+        ctypes.byref(s), ctypes.byref(w), _ptr(cu_img), cap, _ptr(in_txt), _ptr(in_img), in_dtype, _ptr(n_img),
+        _ptr(out), _ptr(ws), ws_bytes, _stream(stream)))
+
+
+def hilo_row_sizes(shape: Shape, split: SplitBuffers, n_img, cap: int, stream=None) -> None:
+    s = shape.c()
+    o = split.c()
+    _check("hilo_row_sizes", lib().hilo_row_sizes(ctypes.byref(s), ctypes.byref(o), _ptr(n_img), cap,
+                                                  _stream(stream)))
+
+
 def hilo_block_forward_static_ws(shape: Shape, weights: DeviceWeights, cu_img, cap: int, in_txt, in_img,
                                  in_dtype: int, out, stream=None) -> None:
     """hilo_block_forward with the library's built-in scratch (no workspace argument)."""
@@ -358,6 +377,7 @@ class HotPath:
         self.packed = torch.empty(self.cap, d, dtype=torch.bfloat16, device=device)
         self.out = torch.empty(B * T + self.cap, d, dtype=torch.float32, device=device)
         self.y = torch.empty(B, shape.H, shape.W, d, dtype=torch.float32, device=device)
+        self.n_img = torch.empty(self.cap, dtype=torch.float32, device=device)
         self.ws_bytes = hilo_block_workspace_bytes(shape, self.cap)
         self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=device)
 
@@ -365,31 +385,36 @@ class HotPath:
     def out_img(self) -> torch.Tensor:
         return self.out[self.shape.B * self.shape.T:]
 
-    def run(self, x, text, mask, k_keep, k_mid, stream=None, unpack: bool = True, regions: bool = False) -> None:
+    def run(self, x, text, mask, k_keep, k_mid, stream=None, unpack: bool = True, regions: bool = False,
+            prop: bool = False) -> None:
         """One pass. regions=True takes the window-granular split and the
         delta unpool instead of the token-granular split and the nearest
-        unpool."""
+        unpool; prop=True weights each packed row's attention by its row size
+        (proportional attention)."""
         sh = self.shape
         hilo_score(sh, x, self.score, stream)
         (hilo_split_regions if regions else hilo_split)(sh, self.score, mask, k_keep, k_mid, self.split, None, 0,
                                                         stream)
         hilo_pack(sh, x, self.split, self.packed, self.cap, stream)
-        self.blocks(text, self.packed, HILO_BF16, stream)
+        if prop:
+            hilo_row_sizes(sh, self.split, self.n_img, self.cap, stream)
+        self.blocks(text, self.packed, HILO_BF16, stream, self.n_img if prop else None)
         if unpack:
             if regions:
                 hilo_unpack_delta(sh, self.out_img, self.packed, x, self.split, self.y, stream)
             else:
                 hilo_unpack(sh, self.out_img, self.split, self.y, stream)
 
-    def blocks(self, in_txt, in_img, in_dtype, stream=None) -> None:
+    def blocks(self, in_txt, in_img, in_dtype, stream=None, n_img=None) -> None:
         sh = self.shape
         for i, w in enumerate(self.weights):
-            if i == 0:
-                hilo_block_forward(sh, w, self.split.cu_img, self.cap, in_txt, in_img, in_dtype, self.out,
-                                   self.ws, self.ws_bytes, stream)
+            args = (in_txt, in_img, in_dtype) if i == 0 else (self.out, self.out_img, HILO_F32)
+            if n_img is None:
+                hilo_block_forward(sh, w, self.split.cu_img, self.cap, *args, self.out, self.ws, self.ws_bytes,
+                                   stream)
             else:
-                hilo_block_forward(sh, w, self.split.cu_img, self.cap, self.out, self.out_img, HILO_F32,
-                                   self.out, self.ws, self.ws_bytes, stream)
+                hilo_block_forward_prop(sh, w, self.split.cu_img, self.cap, *args, n_img, self.out, self.ws,
+                                        self.ws_bytes, stream)
 
 
 # ---------------------------------------------------------------------------

@@ -100,6 +100,26 @@ def test_regions_entry_points_check_arguments(H):
     assert L.hilo_unpack_delta(ctypes.byref(s), 256, 256, 264, ctypes.byref(sp), 256, None) == -1
 
 
+def test_prop_entry_points_check_arguments(H):
+    s = H.hilo_shape(1, 8, 8, 128, 4, 1, 1, 1)
+    L = H.lib()
+    w = H.hilo_block_weights()
+    for f in ("txt", "img"):
+        sw = getattr(w, f)
+        for n in ("w_qkv", "b_qkv", "w_o", "b_o", "w_1", "b_1", "w_2", "b_2"):
+            setattr(sw, n, 256)
+    assert L.hilo_block_forward_prop(ctypes.byref(s), ctypes.byref(w), 256, 64, 256, 256, 0, None, 256, 256,
+                                     1 << 30, None) == -1
+    assert L.hilo_block_forward_prop(ctypes.byref(s), ctypes.byref(w), 256, 64, 256, 256, 0, 258, 256, 256,
+                                     1 << 30, None) == -1
+    sp = H.hilo_split_out()
+    assert L.hilo_row_sizes(ctypes.byref(s), ctypes.byref(sp), 256, 64, None) == -1
+    for f in ("labels", "row_src", "counts", "cu_img", "tok_row"):
+        setattr(sp, f, 256)
+    assert L.hilo_row_sizes(ctypes.byref(s), ctypes.byref(sp), None, 64, None) == -1
+    assert L.hilo_row_sizes(ctypes.byref(s), ctypes.byref(sp), 256, -1, None) == -1
+
+
 def test_workspace_size_and_check(H):
     s = H.hilo_shape(2, 64, 64, 3072, 512, 24, 1, 1)
     cap = 2 * 4096
