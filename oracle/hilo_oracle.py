@@ -26,6 +26,10 @@ the DiT it feeds; the concrete variant -- token-space score, top-k split,
           softmax attention, tanh-GELU 4x MLP, residual adds.
   unpack  every grid token reads the output row of its kept token or of its
           window (nearest broadcast).
+  split(lf=f), pack(lf=f)  the separate low-frequency token set (Sec. 2.3:
+          the kept tokens are concatenated with all tokens of a downsampled
+          image, here the grid average-pooled f-fold per side, without the
+          VAE); the other tokens read their window's row back (delta unpool).
   row_sizes, block(n_img=...)  proportional attention for pooled tokens:
           a packed row standing for n grid tokens adds ln(n) to its logits as
           a key, i.e. it draws the attention of n identical copies (the
@@ -81,6 +85,7 @@ import numpy as np
 KEEP = 0
 POOL2 = 1
 POOL4 = 2
+LF = 3
 
 # ---------------------------------------------------------------------------
 # bf16 conversion (own implementation; pinned against torch in the tests)
@@ -163,7 +168,7 @@ def ranking(s: np.ndarray) -> np.ndarray:
 
 
 def split(s: np.ndarray, mask: np.ndarray, k_keep, k_mid, H: int, W: int, levels: int,
-          granular: bool = False) -> Split:
+          granular: bool = False, lf: int = 0) -> Split:
     """Deterministic keep/pool split of each image (see module docstring).
 
     granular=True is the window-granular (regionalised) variant, the token-
@@ -172,7 +177,16 @@ def split(s: np.ndarray, mask: np.ndarray, k_keep, k_mid, H: int, W: int, levels
     2x2 window with a member in top-k_keep or the mask is kept whole; with two
     levels, an aligned 4x4 block is pooled 4x4 only when all 16 of its members
     rank below the k_mid cut, otherwise its (whole, non-kept) 2x2 windows are
-    pooled 2x2. Every pooled window is then full."""
+    pooled 2x2. Every pooled window is then full.
+
+    lf > 0 is the separate low-frequency token set of Sec. 2.3 in token
+    space: the kept tokens (top-k_keep united with the mask) are followed by
+    one row per aligned lf x lf window of the whole grid (every window, kept
+    members included: the grid downsampled lf-fold per side); the other
+    tokens are labelled LF and read their output from their window's row.
+    counts = (kept, windows, 0); levels must be 1."""
+    if lf:
+        return _split_lf(s, mask, k_keep, H, W, lf)
     B, N = s.shape
     assert N == H * W and levels in (1, 2)
     labels = np.empty((B, N), dtype=np.uint8)
@@ -224,14 +238,43 @@ def split(s: np.ndarray, mask: np.ndarray, k_keep, k_mid, H: int, W: int, levels
 # ---------------------------------------------------------------------------
 
 
+def _split_lf(s, mask, k_keep, H: int, W: int, lf: int) -> Split:
+    B, N = s.shape
+    assert H % lf == 0 and W % lf == 0
+    nlf = (H // lf) * (W // lf)
+    p = np.arange(N) // W
+    q = np.arange(N) % W
+    win_of = (p // lf) * (W // lf) + (q // lf)
+    labels = np.empty((B, N), dtype=np.uint8)
+    counts = np.zeros((B, 3), dtype=np.int32)
+    cu = np.zeros(B + 1, dtype=np.int32)
+    tok_row = np.empty((B, N), dtype=np.int32)
+    rows = []
+    for b in range(B):
+        keep = mask[b].astype(bool).copy()
+        keep[ranking(s[b])[:int(k_keep[b])]] = True
+        labels[b] = np.where(keep, KEEP, LF)
+        kept = np.nonzero(keep)[0]
+        counts[b] = (len(kept), nlf, 0)
+        cu[b + 1] = cu[b] + len(kept) + nlf
+        base = int(cu[b])
+        tok_row[b, kept] = base + np.arange(len(kept))
+        tok_row[b, ~keep] = base + len(kept) + win_of[~keep]
+        rows += [kept, np.arange(nlf)]
+    row_src = np.concatenate([np.asarray(r, dtype=np.int64) for r in rows]).astype(np.int32)
+    return Split(labels, row_src, counts, cu, tok_row)
+
+
 def window_members(w: int, size: int, W: int) -> list[int]:
     """Token ids of aligned size x size window ``w`` in raster order."""
     wp, wq = divmod(w, W // size)
     return [(size * wp + i) * W + size * wq + j for i in range(size) for j in range(size)]
 
 
-def pack(x_bits: np.ndarray, sp: Split) -> np.ndarray:
-    """Packed image rows, uint16 [rows, d] (bf16)."""
+def pack(x_bits: np.ndarray, sp: Split, lf: int = 0) -> np.ndarray:
+    """Packed image rows, uint16 [rows, d] (bf16). With lf > 0 (a split made
+    with the same lf) the rows after the kept tokens are the lf x lf window
+    means over all members."""
     B, H, W, d = x_bits.shape
     x = bf16_to_f32(x_bits).reshape(B, H * W, d)
     out = np.empty((int(sp.cu_img[-1]), d), dtype=np.uint16)
@@ -243,8 +286,11 @@ def pack(x_bits: np.ndarray, sp: Split) -> np.ndarray:
             if r < nk:
                 out[base + r] = x_bits.reshape(B, H * W, d)[b, src]
                 continue
-            size, cls = (2, POOL2) if r < nk + n2 else (4, POOL4)
-            members = [t for t in window_members(src, size, W) if sp.labels[b, t] == cls]
+            if lf:
+                members = window_members(src, lf, W)
+            else:
+                size, cls = (2, POOL2) if r < nk + n2 else (4, POOL4)
+                members = [t for t in window_members(src, size, W) if sp.labels[b, t] == cls]
             acc = x[b, members[0]].copy()
             for t in members[1:]:
                 acc = acc + x[b, t]
@@ -504,7 +550,7 @@ def sobel_select(img: np.ndarray, mask: np.ndarray, H: int, W: int, patch: int, 
 
 
 def hot_path(x_bits, text_bits, mask, k_keep, k_mid, levels, weights_list, heads, mlp, regions=False,
-             prop=False):
+             prop=False, lf=0):
     """score -> split -> pack -> blocks -> unpack for one batch; regions=True
     takes the window-granular split and the delta unpool, prop=True
     proportional attention (each packed row weighted by its row size).
@@ -513,11 +559,11 @@ def hot_path(x_bits, text_bits, mask, k_keep, k_mid, levels, weights_list, heads
     """
     B, H, W, d = x_bits.shape
     T = text_bits.shape[1]
-    sp = split(score(x_bits), mask, k_keep, k_mid, H, W, levels, granular=regions)
-    packed = pack(x_bits, sp)
+    sp = split(score(x_bits), mask, k_keep, k_mid, H, W, levels, granular=regions, lf=lf)
+    packed = pack(x_bits, sp, lf)
     ut, ui = text_bits.reshape(B * T, d), packed
     n_img = row_sizes(sp) if prop else None
     for wts in weights_list:
         ut, ui = block(ut, ui, sp.cu_img, T, wts, heads, mlp, n_img)
-    y = unpack_delta(ui, packed, x_bits, sp) if regions else unpack(ui, sp)
+    y = unpack_delta(ui, packed, x_bits, sp) if (regions or lf) else unpack(ui, sp)
     return sp, packed, (ut, ui), y

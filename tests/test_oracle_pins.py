@@ -292,7 +292,78 @@ def test_split_granular_brute_force_and_invariants(seed, levels):
     assert np.all(spN.labels == O.KEEP)
 
 
+def test_split_lf_hand_worked():
+    """4 x 4 grid, lf = 2, k_keep = 1 (token 5 ranks first), mask token 15:
+    kept [5, 15], then all four 2 x 2 windows of the grid; every other token
+    reads its window's row."""
+    s = np.zeros((1, 16), dtype=np.float32)
+    s[0, 5] = 1.0
+    m = np.zeros((1, 16), np.uint8)
+    m[0, 15] = 1
+    sp = O.split(s, m, [1], [0], 4, 4, 1, lf=2)
+    assert sp.counts[0].tolist() == [2, 4, 0]
+    assert sp.row_src.tolist() == [5, 15, 0, 1, 2, 3]
+    assert sp.tok_row[0].tolist() == [2, 2, 3, 3, 2, 0, 3, 3, 4, 4, 5, 5, 4, 4, 5, 1]
+    assert sp.labels[0].tolist() == [O.LF] * 5 + [O.KEEP] + [O.LF] * 9 + [O.KEEP]
+
+
+@pytest.mark.parametrize("lf", [2, 4, 8])
+def test_split_lf_count_law_and_rows(lf):
+    rng = np.random.default_rng(50 + lf)
+    H, W, B = 16, 24, 2
+    N = H * W
+    s = rng.random((B, N)).astype(np.float32)
+    m = (rng.random((B, N)) < 0.1).astype(np.uint8)
+    kk = [N // 5, 0]
+    sp = O.split(s, m, kk, [0, 0], H, W, 1, lf=lf)
+    nlf = (H // lf) * (W // lf)
+    for b in range(B):
+        top = set(O.ranking(s[b])[:kk[b]].tolist()) | set(np.nonzero(m[b])[0].tolist())
+        base = int(sp.cu_img[b])
+        assert sp.counts[b].tolist() == [len(top), nlf, 0]
+        assert sp.row_src[base:base + len(top)].tolist() == sorted(top)
+        assert sp.row_src[base + len(top):int(sp.cu_img[b + 1])].tolist() == list(range(nlf))
+        for i in range(N):
+            r = int(sp.tok_row[b, i]) - base
+            if i in top:
+                assert sp.labels[b, i] == O.KEEP and int(sp.row_src[base + r]) == i
+            else:
+                assert sp.labels[b, i] == O.LF
+                assert r - len(top) == (i // W // lf) * (W // lf) + (i % W) // lf
+
+
+@pytest.mark.parametrize("lf", [2, 4])
+def test_pack_lf_is_the_downsampled_grid(lf):
+    """LF rows are the grid average-pooled lf-fold per side (all members,
+    kept ones included): the fp64 reshape-mean within one bf16 rounding and
+    the fp32 summation; constant windows pool exactly and the delta unpool of
+    an unchanged block returns every token."""
+    rng = np.random.default_rng(60 + lf)
+    H, W, d = 8, 16, 32
+    x = rng.standard_normal((1, H, W, d)).astype(np.float32)
+    xb = bits(x)
+    xf = O.bf16_to_f32(xb)[0].astype(np.float64)
+    s = O.score(xb)
+    m = (rng.random((1, H * W)) < 0.2).astype(np.uint8)
+    sp = O.split(s, m, [H * W // 4], [0], H, W, 1, lf=lf)
+    packed = O.pack(xb, sp, lf)
+    nk = int(sp.counts[0, 0])
+    ref = xf.reshape(H // lf, lf, W // lf, lf, d).mean(axis=(1, 3)).reshape(-1, d)
+    got = O.bf16_to_f32(packed[nk:]).astype(np.float64)
+    assert np.all(np.abs(got - ref) <= np.abs(ref) * 2 ** -8 + 1e-6)
+    # kept rows are the tokens themselves
+    assert np.array_equal(packed[:nk], xb.reshape(-1, d)[sp.row_src[:nk]])
+    # constant windows: exact pooling, and y = x through the delta unpool
+    blk = rng.standard_normal((H // lf, W // lf, d)).astype(np.float32)
+    xc = bits(np.repeat(np.repeat(blk, lf, axis=0), lf, axis=1)[None])
+    pc = O.pack(xc, sp, lf)
+    assert np.array_equal(pc[nk:], bits(blk).reshape(-1, d))
+    y = O.unpack_delta(O.bf16_to_f32(pc), pc, xc, sp)
+    assert np.array_equal(y, O.bf16_to_f32(xc))
+
+
 # ---------------------------------------------------------- pack/unpack ----
+
 
 
 def test_pack_constant_windows_lossless():
