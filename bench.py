@@ -379,6 +379,35 @@ def time_prop(H, torch, stream, wl, hp, dw, inputs, steps: int) -> dict:
             "block_ms_prop": prop, "block_ms_plain_same_rows": plain, "block_overhead": prop / plain - 1.0}
 
 
+def time_lf(H, torch, stream, wl, dw, inputs, steps: int, lf: int = 4) -> dict:
+    """The separate low-frequency token set on the timed workload: kept
+    tokens (top-k united with the mask) followed by every lf x lf window mean
+    of the grid, delta unpool; with and without proportional attention."""
+    x, text, mask, kk, km = inputs
+    sh = H.Shape(B=wl.B, H=wl.H, W=wl.W, d=wl.d, T=wl.T, heads=wl.heads, mlp=int(wl.mlp), levels=1, lf=lf)
+    hp = H.HotPath(sh, [dw])
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for _ in range(steps):
+            fn()
+        s1.record(stream)
+        torch.cuda.synchronize()
+        return s0.elapsed_time(s1) / steps
+
+    ms = timed(lambda: hp.run(x, text, mask, kk, km))
+    ms_prop = timed(lambda: hp.run(x, text, mask, kk, km, prop=True))
+    H.hilo_sync_status()
+    counts = hp.split.counts.view(-1, 3).sum(0).tolist()
+    return {"lf": lf, "hot_path_ms": ms, "image_tokens_per_s": wl.B * wl.N / (ms * 1e-3),
+            "hot_path_ms_proportional_attention": ms_prop, "kept_tokens": int(counts[0]),
+            "low_frequency_tokens": int(counts[1]), "packed_image_rows": int(hp.split.cu_img[-1].item())}
+
+
 def time_configs(H, I, torch, stream, steps: int):
     """Hot path, compressed block and dense block of each workload configuration.
 
@@ -684,6 +713,7 @@ def run_hilo(args):
         extras["sobel_selector"] = time_sobel_selector(H, I, torch, stream, wl, batch, hp, hbm_peak, Ks)
         extras["regions"] = time_regions(H, torch, stream, wl, hp, (x, text, mask, kk, km), hbm_peak, Ks)
         extras["proportional_attention"] = time_prop(H, torch, stream, wl, hp, dw, (x, text, mask, kk, km), Ks)
+        extras["low_frequency_set"] = time_lf(H, torch, stream, wl, dw, (x, text, mask, kk, km), Ks)
         if world == 1:
             extras["configs"] = time_configs(H, I, torch, stream, steps=20)
         # dense block: every grid token is its own row, no score/split/pack/unpack

@@ -57,8 +57,9 @@ enum {
   HILO_ERR_UNSUPPORTED = -6  /* no sm_103a device, or a feature not built */
 };
 
-/* Per-token labels written by hilo_split. */
-enum { HILO_KEEP = 0, HILO_POOL2 = 1, HILO_POOL4 = 2 };
+/* Per-token labels written by hilo_split (HILO_LF: a non-kept token of the
+ * separate low-frequency mode, shape.lf > 0). */
+enum { HILO_KEEP = 0, HILO_POOL2 = 1, HILO_POOL4 = 2, HILO_LF = 3 };
 
 /* Input dtypes of hilo_block_forward. */
 enum { HILO_BF16 = 0, HILO_F32 = 1 };
@@ -72,16 +73,31 @@ enum { HILO_BF16 = 0, HILO_F32 = 1 };
  *   heads   attention heads; head_dim = d / heads must be 64 or 128
  *   mlp     1: attention + 4x GELU MLP (a full MMDiT block); 0: attention only
  *   levels  1: every non-kept token is pooled 2x2; 2: 2x2 and 4x4 pooling
+ *   lf      0: the in-grid pooling above; 2, 4 or 8: the separate
+ *           low-frequency token set (paper Sec. 2.3: the kept tokens are
+ *           concatenated with every token of a downsampled image; here the
+ *           grid average-pooled lf-fold per side, all members included).
+ *           Needs levels == 1 and H, W multiples of lf.
  * Any other combination returns HILO_ERR_SHAPE.
  */
 typedef struct {
-  int32_t B, H, W, d, T, heads, mlp, levels;
+  int32_t B, H, W, d, T, heads, mlp, levels, lf;
 } hilo_shape;
+
+/*
+ * The most packed image rows a split of this shape can produce over the
+ * batch: B*N, or B*(N + N/lf^2) with the separate low-frequency set (every
+ * token kept and every window added). Size row_src, the packed rows, the
+ * block's image rows (cap) and the unpack inputs to at least this; 0 for an
+ * invalid shape.
+ */
+size_t hilo_row_capacity(const hilo_shape* shape);
 
 /*
  * Outputs of hilo_split (device pointers, caller-allocated), N = H*W:
  *   labels   uint8 [B*N]  HILO_KEEP / HILO_POOL2 / HILO_POOL4 per token
- *   row_src  int32 [B*N]  for packed image row r (0 <= r < cu_img[B]): the
+ *   row_src  int32 [hilo_row_capacity]  for packed image row r
+ *                         (0 <= r < cu_img[B]): the
  *                         token id of a kept row, else the window id of a
  *                         pooled row (2x2 window id (p/2)*(W/2) + q/2, 4x4
  *                         window id (p/4)*(W/4) + q/4)
@@ -91,6 +107,10 @@ typedef struct {
  *                         offset) each grid token reads its output from
  * Per image the packed rows are: kept tokens in raster order, then 2x2
  * windows in window-raster order, then 4x4 windows in window-raster order.
+ * With shape.lf > 0: kept tokens, then every lf x lf window of the grid in
+ * window-raster order (counts = kept, windows, 0; row_src of window rows =
+ * the window id (p/lf)*(W/lf) + q/lf; tok_row of an HILO_LF token = its
+ * window's row).
  */
 typedef struct {
   uint8_t* labels;

@@ -324,7 +324,10 @@ def softmax_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, key_n=None) -
     tokens receives the attention mass of n identical copies of itself."""
     sc = (q @ k.T) / math.sqrt(q.shape[-1])
     if key_n is not None:
-        sc = sc + np.log(np.asarray(key_n, dtype=np.float64))[None, :]
+        # a weight of 0 (a low-frequency row all of whose members are kept)
+        # removes the key: ln 0 = -inf
+        with np.errstate(divide="ignore"):
+            sc = sc + np.log(np.asarray(key_n, dtype=np.float64))[None, :]
     sc = sc - sc.max(axis=-1, keepdims=True)
     p = np.exp(sc)
     p = p / p.sum(axis=-1, keepdims=True)

@@ -74,6 +74,10 @@ int check_shape(const hilo_shape* s, bool need_block) {
   if (s->levels != 1 && s->levels != 2) return fail(HILO_ERR_SHAPE, "levels=%d must be 1 or 2", s->levels);
   if (s->levels == 2 && ((s->H & 3) || (s->W & 3)))
     return fail(HILO_ERR_SHAPE, "H=%d, W=%d must be multiples of 4 for two-level pooling", s->H, s->W);
+  if (s->lf != 0 && s->lf != 2 && s->lf != 4 && s->lf != 8)
+    return fail(HILO_ERR_SHAPE, "lf=%d must be 0, 2, 4 or 8", s->lf);
+  if (s->lf && (s->levels != 1 || s->H % s->lf || s->W % s->lf))
+    return fail(HILO_ERR_SHAPE, "lf=%d needs levels=1 and H=%d, W=%d multiples of lf", s->lf, s->H, s->W);
   if (static_cast<long long>(s->H) * s->W > 32768)
     return fail(HILO_ERR_SHAPE, "H*W=%lld exceeds 32768 tokens per image",
                 static_cast<long long>(s->H) * s->W);
@@ -242,7 +246,7 @@ static int split_common(const char* name, const hilo_shape* shape, const float* 
   cudaError_t e = hilo::launch_split(score, mask, k_keep, shape->levels == 2 ? k_mid : k_keep,
                                      out->labels, out->row_src, out->counts, out->cu_img,
                                      out->tok_row, shape->B, shape->H, shape->W, shape->levels, granular,
-                                     static_cast<cudaStream_t>(stream));
+                                     shape->lf, static_cast<cudaStream_t>(stream));
   if (e == cudaSuccess) count(shape->B == 1 ? 1 : 2);  // one image: the select kernel also compacts
   return e == cudaSuccess ? HILO_OK : cuda_fail(e, name);
 }
@@ -260,6 +264,8 @@ int hilo_split_regions(const hilo_shape* shape, const float* score, const uint8_
                        size_t ws_bytes, void* stream) {
   (void)ws;
   (void)ws_bytes;
+  if (shape && shape->lf)
+    return fail(HILO_ERR_ARG, "hilo_split_regions: the window-granular split has no low-frequency mode");
   return split_common("hilo_split_regions", shape, score, mask, k_keep, k_mid, out, 1, stream);
 }
 
@@ -303,10 +309,16 @@ int hilo_pack(const hilo_shape* shape, const void* x, const hilo_split_out* spli
   DevInfo* dev;
   if ((st = current_device(&dev))) return st;
   cudaError_t e = hilo::launch_pack(x, split->labels, split->row_src, split->counts, split->cu_img,
-                                    packed, shape->B, shape->H, shape->W, shape->d, cap,
+                                    packed, shape->B, shape->H, shape->W, shape->d, cap, shape->lf,
                                     dev->num_sms, static_cast<cudaStream_t>(stream));
   if (e == cudaSuccess) count(1);
   return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_pack");
+}
+
+size_t hilo_row_capacity(const hilo_shape* shape) {
+  if (check_shape(shape, false)) return 0;
+  const size_t N = static_cast<size_t>(shape->H) * shape->W;
+  return static_cast<size_t>(shape->B) * (N + (shape->lf ? N / (shape->lf * shape->lf) : 0));
 }
 
 size_t hilo_block_workspace_bytes(const hilo_shape* shape, int32_t cap) {
@@ -397,7 +409,7 @@ static int block_forward_impl(const hilo_shape* shape, const hilo_block_weights*
   aa.head_dim = d / shape->heads;
   aa.d = d;
   aa.R = R;
-  aa.max_img_rows = shape->H * shape->W;
+  aa.max_img_rows = static_cast<int>(hilo_row_capacity(shape) / shape->B);
   e = hilo::launch_attention(aa, dev->num_sms, s);
   if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: attention");
   count(1);
@@ -449,7 +461,7 @@ int hilo_row_sizes(const hilo_shape* shape, const hilo_split_out* split, float* 
   DevInfo* dev;
   if ((st = current_device(&dev))) return st;
   cudaError_t e = hilo::launch_row_sizes(split->labels, split->row_src, split->counts, split->cu_img, n_img,
-                                         shape->B, shape->H, shape->W, cap, dev->num_sms,
+                                         shape->B, shape->H, shape->W, cap, shape->lf, dev->num_sms,
                                          static_cast<cudaStream_t>(stream));
   if (e == cudaSuccess && cap > 0) count(1);
   return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_row_sizes");

@@ -83,6 +83,7 @@ struct AttnParams {
   const float* n_img;  // PROP: weight of each packed image row
   __nv_bfloat16* out;
   int B, T, heads, d, qt_txt, pairs_max;
+  int cap;           // image-row capacity: row offsets are clamped to it
   float scale_log2;  // log2(e) / sqrt(head_dim)
 };
 
@@ -139,7 +140,7 @@ __device__ __forceinline__ void seq_tile(const AttnParams& p, int b, int L, int 
     valid = min(BKV, p.T - j * BKV);
   } else {
     const int k = j - p.qt_txt;
-    row0 = p.B * p.T + p.cu_img[b] + k * BKV;
+    row0 = p.B * p.T + min(p.cu_img[b], p.cap) + k * BKV;
     valid = min(BKV, L - k * BKV);
   }
 }
@@ -155,7 +156,8 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
   const int b = item / (p.heads * p.pairs_max);
   const int h = (item / p.pairs_max) % p.heads;
   const int pair = item % p.pairs_max;
-  const int L = p.cu_img[b + 1] - p.cu_img[b];
+  // image rows [cu_img[b], cu_img[b+1]) within the capacity
+  const int L = min(p.cu_img[b + 1], p.cap) - min(p.cu_img[b], p.cap);
   const int nkv = p.qt_txt + (L + BKV - 1) / BKV;  // also the number of query tiles
   if (2 * pair >= nkv) return;                     // beyond this image's compressed length
   const bool has1 = 2 * pair + 1 < nkv;
@@ -378,7 +380,7 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
         } else {
           int r0, v;
           seq_tile(p, b, L, tt, r0, v);
-          const float* src = p.n_img + (p.cu_img[b] + (tt - p.qt_txt) * BKV);
+          const float* src = p.n_img + (min(p.cu_img[b], p.cap) + (tt - p.qt_txt) * BKV);
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
             const int col = lane + 32 * u;
@@ -613,6 +615,7 @@ cudaError_t launch_attention(const AttnArgs& a, int num_sms, cudaStream_t st) {
   p.heads = a.heads;
   p.d = a.d;
   p.qt_txt = (a.T + BQ - 1) / BQ;
+  p.cap = a.R - a.B * a.T;
   const int qt_img_max = (a.max_img_rows + BQ - 1) / BQ;
   p.pairs_max = (p.qt_txt + qt_img_max + 1) / 2;
   p.scale_log2 = static_cast<float>(1.4426950408889634 / sqrt(static_cast<double>(a.head_dim)));

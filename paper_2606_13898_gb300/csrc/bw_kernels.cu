@@ -304,7 +304,7 @@ __device__ void mark_topk(const uint32_t* keys, const uint8_t* cand, uint8_t* se
 // the token -> row map, kept tokens first (raster order), then 2x2 windows,
 // then 4x4 windows (window-raster order). `base` is the image's first packed
 // row. Called by all threads of the CTA.
-__device__ void compact_image(const uint8_t* lab, int b, int H, int W, int levels, int base, int nk,
+__device__ void compact_image(const uint8_t* lab, int b, int H, int W, int levels, int lf, int base, int nk,
                               int n2, int32_t* row_src, int32_t* tok_row, int* warp_tot) {
   const int N = H * W;
   int32_t* trow = tok_row + static_cast<long long>(b) * N;
@@ -321,6 +321,20 @@ __device__ void compact_image(const uint8_t* lab, int b, int H, int W, int level
         trow[i] = r;
         ++r;
       }
+  }
+  // low-frequency mode: every lf x lf window of the grid, in window-raster
+  // order; its non-kept members read it back
+  if (lf) {
+    const int Wl = W / lf, nw = (H / lf) * Wl;
+    for (int w = threadIdx.x; w < nw; w += blockDim.x) {
+      const int r = base + nk + w;
+      row_src[r] = w;
+      const int t0 = (lf * (w / Wl)) * W + lf * (w % Wl);
+      for (int i = 0; i < lf; ++i)
+        for (int j = 0; j < lf; ++j)
+          if (lab[t0 + i * W + j] != HILO_LABEL_KEEP) trow[t0 + i * W + j] = r;
+    }
+    return;
   }
   // 2x2 windows in window-raster order
   {
@@ -385,11 +399,16 @@ __device__ void compact_image(const uint8_t* lab, int b, int H, int W, int level
 // aligned 2x2 window with a kept member is kept whole; with two levels an
 // aligned 4x4 block is pooled 4x4 only when all its members rank below the
 // k_mid cut, else its non-kept members are pooled 2x2).
+template <bool GRANULAR, bool LFMODE>
 __global__ void __launch_bounds__(SPLIT_THREADS) split_select_kernel(
     const float* __restrict__ score, const uint8_t* __restrict__ mask,
     const int32_t* __restrict__ k_keep, const int32_t* __restrict__ k_mid, uint8_t* labels_out,
-    int32_t* counts, int H, int W, int levels, int granular, int fused, int32_t* cu_img,
+    int32_t* counts, int H, int W, int levels, int lf_arg, int fused, int32_t* cu_img,
     int32_t* row_src, int32_t* tok_row) {
+  // the modes are template parameters, so the plain split carries none of
+  // their code (this CTA has 1024 threads and at most 64 registers each)
+  constexpr bool granular = GRANULAR;
+  const int lf = LFMODE ? lf_arg : 0;
   pdl_trigger();
   pdl_wait();
   extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -413,7 +432,7 @@ __global__ void __launch_bounds__(SPLIT_THREADS) split_select_kernel(
   mark_topk(keys, nullptr, sel, N, k, sh);
   for (int i = threadIdx.x; i < N; i += blockDim.x) {
     const bool keep = sel[i] || cand[i];
-    lab[i] = keep ? HILO_LABEL_KEEP : HILO_LABEL_POOL2;
+    lab[i] = keep ? HILO_LABEL_KEEP : (lf ? HILO_LABEL_LF : HILO_LABEL_POOL2);
     cand[i] = keep ? 0 : 1;
   }
   __syncthreads();
@@ -461,13 +480,16 @@ __global__ void __launch_bounds__(SPLIT_THREADS) split_select_kernel(
   // counts and each thread's first packed row.
   const int tch = (N + blockDim.x - 1) / blockDim.x;
   const int i0 = min(N, static_cast<int>(threadIdx.x) * tch), i1 = min(N, i0 + tch);
-  const int W2 = W >> 1, nw2 = (H >> 1) * W2;
+  // (low-frequency mode: the "2x2 windows" below are the lf x lf windows,
+  // every one of which has a row)
+  const int W2 = lf ? W / lf : W >> 1, nw2 = (lf ? H / lf : H >> 1) * W2;
   const int wch = (nw2 + blockDim.x - 1) / blockDim.x;
   const int w0 = min(nw2, static_cast<int>(threadIdx.x) * wch), w1 = min(nw2, w0 + wch);
   const int W4 = W >> 2, nw4 = levels == 2 ? (H >> 2) * W4 : 0;
   const int vch = (nw4 + blockDim.x - 1) / blockDim.x;
   const int v0 = min(nw4, static_cast<int>(threadIdx.x) * vch), v1 = min(nw4, v0 + vch);
   auto has2 = [&](int w) {
+    if (lf) return true;
     const int t = (2 * (w / W2)) * W + 2 * (w % W2);
     return lab[t] == HILO_LABEL_POOL2 || lab[t + 1] == HILO_LABEL_POOL2 || lab[t + W] == HILO_LABEL_POOL2 ||
            lab[t + W + 1] == HILO_LABEL_POOL2;
@@ -511,8 +533,16 @@ __global__ void __launch_bounds__(SPLIT_THREADS) split_select_kernel(
   r2 += nk;
   for (int w = w0; w < w1; ++w) {
     if (!has2(w)) continue;
-    const int t = (2 * (w / W2)) * W + 2 * (w % W2);
     row_src[r2] = w;
+    if (lf) {
+      const int t0 = (lf * (w / W2)) * W + lf * (w % W2);
+      for (int i = 0; i < lf; ++i)
+        for (int j = 0; j < lf; ++j)
+          if (lab[t0 + i * W + j] != HILO_LABEL_KEEP) trow[t0 + i * W + j] = r2;
+      ++r2;
+      continue;
+    }
+    const int t = (2 * (w / W2)) * W + 2 * (w % W2);
     const int mem[4] = {t, t + 1, t + W, t + W + 1};
 #pragma unroll
     for (int j = 0; j < 4; ++j)
@@ -536,7 +566,7 @@ __global__ void __launch_bounds__(SPLIT_THREADS) split_select_kernel(
 // Packed offsets, row sources and token -> row map. One CTA per image.
 __global__ void __launch_bounds__(SPLIT_THREADS) split_compact_kernel(
     const uint8_t* __restrict__ labels, const int32_t* __restrict__ counts, int32_t* cu_img,
-    int32_t* row_src, int32_t* tok_row, int H, int W, int levels) {
+    int32_t* row_src, int32_t* tok_row, int H, int W, int levels, int lf) {
   pdl_trigger();
   pdl_wait();
   extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -553,7 +583,7 @@ __global__ void __launch_bounds__(SPLIT_THREADS) split_compact_kernel(
     cu_img[b + 1] = base + nk + n2 + n4;
   }
   __syncthreads();
-  compact_image(lab, b, H, W, levels, base, nk, n2, row_src, tok_row, warp_tot);
+  compact_image(lab, b, H, W, levels, lf, base, nk, n2, row_src, tok_row, warp_tot);
 }
 
 // =============================================================== pack =====
@@ -565,6 +595,42 @@ __global__ void __launch_bounds__(SPLIT_THREADS) split_compact_kernel(
 // correct rounding and rounds to bf16 (nearest even).
 
 constexpr int PACK_WARPS_PER_ROW = 4;
+
+// A low-frequency row: the mean of all LF x LF members of the window whose
+// first member is w0 (raster order, the first initialising the sum), one
+// correctly rounded division; this lane's 8-channel chunks c0, c0 + cstep, ...
+template <int LF>
+__device__ __forceinline__ void pack_lf_row(const __nv_bfloat16* __restrict__ w0, int W, int d, int c0, int G,
+                                            int cstep, uint4* __restrict__ dst) {
+  constexpr int NM = LF * LF;
+  const float cnt = static_cast<float>(NM);
+#pragma unroll 1
+  for (int c = c0; c < G; c += cstep) {
+    float acc[8];
+#pragma unroll 1
+    for (int g = 0; g < NM; g += 4) {
+      uint4 v[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int m = g + q;
+        v[q] = __ldg(reinterpret_cast<const uint4*>(w0 + static_cast<long long>((m / LF) * W + (m % LF)) * d) + c);
+      }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        float f[8];
+        bf16x8_to_f32(v[q], f);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) acc[u] = (g == 0 && q == 0) ? f[u] : __fadd_rn(acc[u], f[u]);
+      }
+    }
+    uint4 o;
+    o.x = pack_bf16x2(__fdiv_rn(acc[0], cnt), __fdiv_rn(acc[1], cnt));
+    o.y = pack_bf16x2(__fdiv_rn(acc[2], cnt), __fdiv_rn(acc[3], cnt));
+    o.z = pack_bf16x2(__fdiv_rn(acc[4], cnt), __fdiv_rn(acc[5], cnt));
+    o.w = pack_bf16x2(__fdiv_rn(acc[6], cnt), __fdiv_rn(acc[7], cnt));
+    dst[c] = o;
+  }
+}
 
 __global__ void __launch_bounds__(256) pack_kernel(const __nv_bfloat16* __restrict__ x,
                                                    const uint8_t* __restrict__ labels,
@@ -651,6 +717,45 @@ __global__ void __launch_bounds__(256) pack_kernel(const __nv_bfloat16* __restri
   }
 }
 
+// Low-frequency mode: per image, the kept rows (copies) and then one row per
+// LF x LF window of the grid (the mean of all its members). Same row
+// assignment as pack_kernel: four warps per packed row.
+template <int LF>
+__global__ void __launch_bounds__(256) pack_lf_kernel(const __nv_bfloat16* __restrict__ x,
+                                                      const int32_t* __restrict__ row_src,
+                                                      const int32_t* __restrict__ counts,
+                                                      const int32_t* __restrict__ cu_img,
+                                                      __nv_bfloat16* __restrict__ packed, int B, int H, int W,
+                                                      int d, int cap) {
+  pdl_trigger();
+  pdl_wait();
+  const int lane = threadIdx.x & 31;
+  const int N = H * W;
+  const int G = d >> 3;
+  const int total = min(cu_img[B], cap);
+  const long long nwarps = static_cast<long long>(gridDim.x) * (blockDim.x >> 5);
+  constexpr int CSTEP = 32 * PACK_WARPS_PER_ROW;
+  for (long long gw = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+       gw < static_cast<long long>(total) * PACK_WARPS_PER_ROW; gw += nwarps) {
+    const int r = static_cast<int>(gw / PACK_WARPS_PER_ROW);
+    const int c0 = lane + 32 * static_cast<int>(gw % PACK_WARPS_PER_ROW);
+    int b = 0;
+    while (b + 1 < B && cu_img[b + 1] <= r) ++b;
+    const int local = r - cu_img[b];
+    const int src = row_src[r];
+    const __nv_bfloat16* xb = x + static_cast<long long>(b) * N * d;
+    uint4* dst = reinterpret_cast<uint4*>(packed + static_cast<long long>(r) * d);
+    if (local < counts[3 * b]) {
+      const uint4* sp = reinterpret_cast<const uint4*>(xb + static_cast<long long>(src) * d);
+#pragma unroll 4
+      for (int c = c0; c < G; c += CSTEP) dst[c] = __ldg(sp + c);
+      continue;
+    }
+    const int t0 = (LF * (src / (W / LF))) * W + LF * (src % (W / LF));
+    pack_lf_row<LF>(xb + static_cast<long long>(t0) * d, W, d, c0, G, CSTEP, dst);
+  }
+}
+
 // Number of grid tokens each packed image row stands for: 1 for a kept
 // token, the count of its class members for a pooled window (the weights of
 // proportional attention). One thread per row of the capacity.
@@ -659,7 +764,7 @@ __global__ void __launch_bounds__(256) row_sizes_kernel(const uint8_t* __restric
                                                         const int32_t* __restrict__ counts,
                                                         const int32_t* __restrict__ cu_img,
                                                         float* __restrict__ n_img, int B, int H, int W,
-                                                        int cap) {
+                                                        int cap, int lf) {
   pdl_trigger();
   pdl_wait();
   const int N = H * W;
@@ -673,8 +778,8 @@ __global__ void __launch_bounds__(256) row_sizes_kernel(const uint8_t* __restric
       n_img[r] = 1.0f;
       continue;
     }
-    const int size = local < nk + n2 ? 2 : 4;
-    const uint8_t cls = size == 2 ? HILO_LABEL_POOL2 : HILO_LABEL_POOL4;
+    const int size = lf ? lf : (local < nk + n2 ? 2 : 4);
+    const uint8_t cls = lf ? HILO_LABEL_LF : (size == 2 ? HILO_LABEL_POOL2 : HILO_LABEL_POOL4);
     const int src = row_src[r];
     const int Wn = W / size;
     const uint8_t* lab = labels + static_cast<long long>(b) * N + (size * (src / Wn)) * W + size * (src % Wn);
@@ -800,11 +905,11 @@ __global__ void __launch_bounds__(LN_THREADS) layernorm_kernel(const void* __res
                                                                int in_f32, float* resid,
                                                                uint16_t* __restrict__ ln, int ln_f16,
                                                                const int32_t* __restrict__ cu_img,
-                                                               int B, int n_txt, int d) {
+                                                               int B, int n_txt, int cap, int d) {
   pdl_trigger();
   pdl_wait();
   __shared__ float red[LN_THREADS / 32];
-  const int rows = n_txt + cu_img[B];
+  const int rows = n_txt + min(cu_img[B], cap);
   const float inv_d = 1.0f / static_cast<float>(d);
   for (int r = blockIdx.x; r < rows; r += gridDim.x) {
     const long long off = static_cast<long long>(r < n_txt ? r : r - n_txt) * d;
@@ -910,28 +1015,35 @@ size_t split_compact_smem(int N) { return static_cast<size_t>(N); }
 cudaError_t launch_split(const float* score, const uint8_t* mask, const int32_t* k_keep,
                          const int32_t* k_mid, uint8_t* labels, int32_t* row_src, int32_t* counts,
                          int32_t* cu_img, int32_t* tok_row, int B, int H, int W, int levels,
-                         int granular, cudaStream_t st) {
+                         int granular, int lf, cudaStream_t st) {
   const int N = H * W;
   const size_t sm1 = split_select_smem(N), sm2 = split_compact_smem(N);
-  cudaError_t e = cudaFuncSetAttribute(split_select_kernel,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(sm1));
+  auto* kern = lf ? split_select_kernel<false, true>
+                  : (granular ? split_select_kernel<true, false> : split_select_kernel<false, false>);
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(sm1));
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(split_compact_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            static_cast<int>(sm2));
   if (e != cudaSuccess) return e;
   const int fused = B == 1 ? 1 : 0;
-  e = launch_pdl(split_select_kernel, dim3(B), dim3(SPLIT_THREADS), sm1, st, score, mask, k_keep,
-                 k_mid, labels, counts, H, W, levels, granular, fused, cu_img, row_src, tok_row);
+  e = launch_pdl(kern, dim3(B), dim3(SPLIT_THREADS), sm1, st, score, mask, k_keep, k_mid, labels, counts, H, W,
+                 levels, lf, fused, cu_img, row_src, tok_row);
   if (e != cudaSuccess || fused) return e;
   return launch_pdl(split_compact_kernel, dim3(B), dim3(SPLIT_THREADS), sm2, st,
                     static_cast<const uint8_t*>(labels), static_cast<const int32_t*>(counts), cu_img,
-                    row_src, tok_row, H, W, levels);
+                    row_src, tok_row, H, W, levels, lf);
 }
 
 cudaError_t launch_pack(const void* x, const uint8_t* labels, const int32_t* row_src,
                         const int32_t* counts, const int32_t* cu_img, void* packed, int B, int H,
-                        int W, int d, int cap, int num_sms, cudaStream_t st) {
+                        int W, int d, int cap, int lf, int num_sms, cudaStream_t st) {
+  const dim3 grid(grid_for(static_cast<long long>(cap) * PACK_WARPS_PER_ROW, 8, num_sms, 8));
+  const auto* xs = static_cast<const __nv_bfloat16*>(x);
+  auto* ps = static_cast<__nv_bfloat16*>(packed);
+  if (lf == 2) return launch_pdl(pack_lf_kernel<2>, grid, dim3(256), 0, st, xs, row_src, counts, cu_img, ps, B, H, W, d, cap);
+  if (lf == 4) return launch_pdl(pack_lf_kernel<4>, grid, dim3(256), 0, st, xs, row_src, counts, cu_img, ps, B, H, W, d, cap);
+  if (lf == 8) return launch_pdl(pack_lf_kernel<8>, grid, dim3(256), 0, st, xs, row_src, counts, cu_img, ps, B, H, W, d, cap);
+  if (lf) return cudaErrorInvalidValue;
   return launch_pdl(pack_kernel, dim3(grid_for(static_cast<long long>(cap) * PACK_WARPS_PER_ROW, 8, num_sms, 8)),
                     dim3(256), 0, st,
                     static_cast<const __nv_bfloat16*>(x), labels, row_src, counts, cu_img,
@@ -945,11 +1057,11 @@ cudaError_t launch_unpack(const float* out_img, const int32_t* tok_row, float* y
 }
 
 cudaError_t launch_row_sizes(const uint8_t* labels, const int32_t* row_src, const int32_t* counts,
-                             const int32_t* cu_img, float* n_img, int B, int H, int W, int cap, int num_sms,
-                             cudaStream_t st) {
+                             const int32_t* cu_img, float* n_img, int B, int H, int W, int cap, int lf,
+                             int num_sms, cudaStream_t st) {
   if (cap <= 0) return cudaSuccess;
   return launch_pdl(row_sizes_kernel, dim3(grid_for(cap, 256, num_sms, 4)), dim3(256), 0, st, labels, row_src,
-                    counts, cu_img, n_img, B, H, W, cap);
+                    counts, cu_img, n_img, B, H, W, cap, lf);
 }
 
 cudaError_t launch_unpack_delta(const float* out_img, const void* packed, const void* x,
@@ -984,7 +1096,7 @@ cudaError_t launch_layernorm(const void* in_txt, const void* in_img, int in_f32,
 #define HILO_LN_CASE(NC)                                                                      \
   case NC:                                                                                    \
     return launch_pdl(layernorm_kernel<NC>, grid, dim3(LN_THREADS), 0, st, in_txt, in_img, in_f32, \
-                      resid, lo, ln_f16, cu_img, B, n_txt, d);
+                      resid, lo, ln_f16, cu_img, B, n_txt, cap, d);
     HILO_LN_CASE(1)
     HILO_LN_CASE(2)
     HILO_LN_CASE(3)

@@ -63,8 +63,9 @@ struct Sched {
   int mt0, mt1, rows0, rows1, nt, total;
   __device__ void init(const Params& p) {
     nt = (p.N + PN - 1) / PN;
-    rows0 = p.rows_dev[0] ? *p.rows_dev[0] : p.rows_static[0];
-    rows1 = p.rows_dev[1] ? *p.rows_dev[1] : p.rows_static[1];
+    // a device row count is bounded by the group's capacity (rows_static)
+    rows0 = p.rows_dev[0] ? min(*p.rows_dev[0], p.rows_static[0]) : p.rows_static[0];
+    rows1 = p.rows_dev[1] ? min(*p.rows_dev[1], p.rows_static[1]) : p.rows_static[1];
     mt0 = (rows0 + PM - 1) / PM;
     mt1 = (rows1 + PM - 1) / PM;
     total = (mt0 + mt1) * nt;
@@ -371,7 +372,7 @@ cudaError_t launch_gemm_pair(const GemmArgs& a, int num_sms, cudaStream_t st) {
   long long upper = 0;
   for (int g = 0; g < 2; ++g) {
     p.row_base[g] = a.g[g].row_base;
-    p.rows_static[g] = a.g[g].rows_static;
+    p.rows_static[g] = a.g[g].rows_dev ? a.g[g].rows_cap : a.g[g].rows_static;
     p.rows_dev[g] = a.g[g].rows_dev;
     p.bias[g] = static_cast<const __nv_bfloat16*>(a.g[g].bias);
     upper += (a.g[g].rows_cap + PM - 1) / PM;

@@ -66,8 +66,9 @@ struct Sched {
   int mt0, mt1, rows0, rows1, nt, total;
   __device__ void init(const GemmParams& p) {
     nt = (p.N + BN - 1) / BN;
-    rows0 = p.rows_dev[0] ? *p.rows_dev[0] : p.rows_static[0];
-    rows1 = p.rows_dev[1] ? *p.rows_dev[1] : p.rows_static[1];
+    // a device row count is bounded by the group's capacity (rows_static)
+    rows0 = p.rows_dev[0] ? min(*p.rows_dev[0], p.rows_static[0]) : p.rows_static[0];
+    rows1 = p.rows_dev[1] ? min(*p.rows_dev[1], p.rows_static[1]) : p.rows_static[1];
     mt0 = (rows0 + BM - 1) / BM;
     mt1 = (rows1 + BM - 1) / BM;
     total = (mt0 + mt1) * nt;
@@ -289,7 +290,7 @@ cudaError_t launch_bn(const GemmArgs& a, int num_sms, cudaStream_t st) {
   long long upper = 0;
   for (int g = 0; g < 2; ++g) {
     p.row_base[g] = a.g[g].row_base;
-    p.rows_static[g] = a.g[g].rows_static;
+    p.rows_static[g] = a.g[g].rows_dev ? a.g[g].rows_cap : a.g[g].rows_static;
     p.rows_dev[g] = a.g[g].rows_dev;
     p.bias[g] = static_cast<const __nv_bfloat16*>(a.g[g].bias);
     upper += (a.g[g].rows_cap + BM - 1) / BM;

@@ -9,6 +9,7 @@
 #define HILO_LABEL_KEEP 0
 #define HILO_LABEL_POOL2 1
 #define HILO_LABEL_POOL4 2
+#define HILO_LABEL_LF 3
 
 namespace hilo {
 
@@ -20,15 +21,15 @@ size_t split_compact_smem(int N);
 cudaError_t launch_split(const float* score, const uint8_t* mask, const int32_t* k_keep,
                          const int32_t* k_mid, uint8_t* labels, int32_t* row_src, int32_t* counts,
                          int32_t* cu_img, int32_t* tok_row, int B, int H, int W, int levels,
-                         int granular, cudaStream_t st);
+                         int granular, int lf, cudaStream_t st);
 cudaError_t launch_pack(const void* x, const uint8_t* labels, const int32_t* row_src,
                         const int32_t* counts, const int32_t* cu_img, void* packed, int B, int H,
-                        int W, int d, int cap, int num_sms, cudaStream_t st);
+                        int W, int d, int cap, int lf, int num_sms, cudaStream_t st);
 cudaError_t launch_unpack(const float* out_img, const int32_t* tok_row, float* y, long long ntok,
                           int d, int num_sms, cudaStream_t st);
 cudaError_t launch_row_sizes(const uint8_t* labels, const int32_t* row_src, const int32_t* counts,
-                             const int32_t* cu_img, float* n_img, int B, int H, int W, int cap, int num_sms,
-                             cudaStream_t st);
+                             const int32_t* cu_img, float* n_img, int B, int H, int W, int cap, int lf,
+                             int num_sms, cudaStream_t st);
 cudaError_t launch_unpack_delta(const float* out_img, const void* packed, const void* x,
                                 const uint8_t* labels, const int32_t* tok_row, float* y, long long ntok,
                                 int d, int num_sms, cudaStream_t st);

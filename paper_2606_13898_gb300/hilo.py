@@ -20,6 +20,7 @@ import torch
 from . import build as _build
 
 HILO_OK = 0
+HILO_ERR_SHAPE = -2
 HILO_KEEP, HILO_POOL2, HILO_POOL4 = 0, 1, 2
 HILO_BF16, HILO_F32 = 0, 1
 
@@ -31,7 +32,7 @@ class HiloError(RuntimeError):
 
 
 class hilo_shape(ctypes.Structure):
-    _fields_ = [(n, ctypes.c_int32) for n in ("B", "H", "W", "d", "T", "heads", "mlp", "levels")]
+    _fields_ = [(n, ctypes.c_int32) for n in ("B", "H", "W", "d", "T", "heads", "mlp", "levels", "lf")]
 
 
 class hilo_split_out(ctypes.Structure):
@@ -51,7 +52,8 @@ EXPORTS = ("hilo_status_string", "hilo_last_error", "hilo_sync_status", "hilo_de
            "hilo_block_workspace_bytes", "hilo_block_forward", "hilo_unpack", "hilo_unpack_update",
            "hilo_convert_bf16_to_f16", "hilo_set_stage_events", "hilo_launch_count",
            "hilo_block_forward_static_ws", "hilo_sobel_workspace_bytes", "hilo_sobel_select",
-           "hilo_split_regions", "hilo_unpack_delta", "hilo_row_sizes", "hilo_block_forward_prop")
+           "hilo_split_regions", "hilo_unpack_delta", "hilo_row_sizes", "hilo_block_forward_prop",
+           "hilo_row_capacity")
 
 _lib = None
 
@@ -96,6 +98,7 @@ def lib() -> ctypes.CDLL:
         "hilo_split_regions": (I, [shp, P, P, P, P, spo, P, S, P]),
         "hilo_unpack_delta": (I, [shp, P, P, P, spo, P, P]),
         "hilo_row_sizes": (I, [shp, spo, P, ctypes.c_int32, P]),
+        "hilo_row_capacity": (S, [shp]),
         "hilo_block_forward_prop": (I, [shp, ctypes.POINTER(hilo_block_weights), P, ctypes.c_int32, P, P, I,
                                         P, P, P, S, P]),
     }
@@ -139,13 +142,14 @@ class Shape:
     heads: int = 1
     mlp: int = 1
     levels: int = 1
+    lf: int = 0
 
     @property
     def N(self) -> int:
         return self.H * self.W
 
     def c(self) -> hilo_shape:
-        return hilo_shape(self.B, self.H, self.W, self.d, self.T, self.heads, int(self.mlp), self.levels)
+        return hilo_shape(self.B, self.H, self.W, self.d, self.T, self.heads, int(self.mlp), self.levels, self.lf)
 
 
 @dataclasses.dataclass
@@ -163,7 +167,7 @@ class SplitBuffers:
         n = shape.B * shape.N
         return SplitBuffers(
             labels=torch.empty(n, dtype=torch.uint8, device=device),
-            row_src=torch.empty(n, dtype=torch.int32, device=device),
+            row_src=torch.empty(hilo_row_capacity(shape), dtype=torch.int32, device=device),
             counts=torch.empty(3 * shape.B, dtype=torch.int32, device=device),
             cu_img=torch.empty(shape.B + 1, dtype=torch.int32, device=device),
             tok_row=torch.empty(n, dtype=torch.int32, device=device))
@@ -234,6 +238,14 @@ def hilo_sync_status(stream=None) -> None:
 def hilo_score(shape: Shape, x, score, stream=None) -> None:
     s = shape.c()
     _check("hilo_score", lib().hilo_score(ctypes.byref(s), _ptr(x), _ptr(score), _stream(stream)))
+
+
+def hilo_row_capacity(shape: Shape) -> int:
+    s = shape.c()
+    n = int(lib().hilo_row_capacity(ctypes.byref(s)))
+    if n == 0:
+        raise HiloError("hilo_row_capacity", HILO_ERR_SHAPE, lib().hilo_last_error().decode())
+    return n
 
 
 def hilo_split_workspace_bytes(shape: Shape) -> int:
@@ -369,7 +381,7 @@ class HotPath:
 
     def __init__(self, shape: Shape, weights: list, device="cuda"):
         self.shape = shape
-        self.cap = shape.B * shape.N
+        self.cap = hilo_row_capacity(shape)
         self.weights = weights
         B, N, d, T = shape.B, shape.N, shape.d, shape.T
         self.score = torch.empty(B * N, dtype=torch.float32, device=device)
@@ -390,7 +402,8 @@ class HotPath:
         """One pass. regions=True takes the window-granular split and the
         delta unpool instead of the token-granular split and the nearest
         unpool; prop=True weights each packed row's attention by its row size
-        (proportional attention)."""
+        (proportional attention). A shape with lf > 0 runs the separate
+        low-frequency token set (with the delta unpool)."""
         sh = self.shape
         hilo_score(sh, x, self.score, stream)
         (hilo_split_regions if regions else hilo_split)(sh, self.score, mask, k_keep, k_mid, self.split, None, 0,
@@ -400,7 +413,9 @@ class HotPath:
             hilo_row_sizes(sh, self.split, self.n_img, self.cap, stream)
         self.blocks(text, self.packed, HILO_BF16, stream, self.n_img if prop else None)
         if unpack:
-            if regions:
+            # pooled or low-frequency tokens keep their own detail in the
+            # window-granular and low-frequency modes (delta unpool)
+            if regions or sh.lf:
                 hilo_unpack_delta(sh, self.out_img, self.packed, x, self.split, self.y, stream)
             else:
                 hilo_unpack(sh, self.out_img, self.split, self.y, stream)

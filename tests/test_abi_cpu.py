@@ -120,6 +120,21 @@ def test_prop_entry_points_check_arguments(H):
     assert L.hilo_row_sizes(ctypes.byref(s), ctypes.byref(sp), 256, -1, None) == -1
 
 
+def test_lf_shape_checks_and_row_capacity(H):
+    L = H.lib()
+    ok = H.hilo_shape(2, 8, 12, 128, 4, 1, 1, 1, 4)
+    assert L.hilo_row_capacity(ctypes.byref(ok)) == 2 * (96 + 96 // 16)
+    assert L.hilo_row_capacity(ctypes.byref(H.hilo_shape(2, 8, 12, 128, 4, 1, 1, 1, 0))) == 2 * 96
+    for bad in (H.hilo_shape(1, 8, 12, 128, 4, 1, 1, 1, 3), H.hilo_shape(1, 8, 12, 128, 4, 1, 1, 2, 4),
+                H.hilo_shape(1, 8, 12, 128, 4, 1, 1, 1, 8)):
+        assert L.hilo_row_capacity(ctypes.byref(bad)) == 0
+        assert L.hilo_score(ctypes.byref(bad), 256, 256, None) == -2
+    sp = H.hilo_split_out()
+    for f in ("labels", "row_src", "counts", "cu_img", "tok_row"):
+        setattr(sp, f, 256)
+    assert L.hilo_split_regions(ctypes.byref(ok), 256, 256, 256, 256, ctypes.byref(sp), None, 0, None) == -1
+
+
 def test_workspace_size_and_check(H):
     s = H.hilo_shape(2, 64, 64, 3072, 512, 24, 1, 1)
     cap = 2 * 4096
