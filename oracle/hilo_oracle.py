@@ -30,6 +30,10 @@ the DiT it feeds; the concrete variant -- token-space score, top-k split,
           the kept tokens are concatenated with all tokens of a downsampled
           image, here the grid average-pooled f-fold per side, without the
           VAE); the other tokens read their window's row back (delta unpool).
+  e4m3_encode, quantize_rows, block_fp8  FP8 GEMM operands (Sec. 3.3 reports
+          FP8 on top of HiLo-Token without a scheme): per-row e4m3 scaling
+          of activations and weights, fp32 accumulation, the activations
+          rounded where the kernels round them.
   row_sizes, block(n_img=...)  proportional attention for pooled tokens:
           a packed row standing for n grid tokens adds ln(n) to its logits as
           a key, i.e. it draws the attention of n identical copies (the
@@ -490,6 +494,162 @@ def update(x_bits: np.ndarray, y: np.ndarray, alpha: float) -> np.ndarray:
     x = bf16_to_f32(x_bits)
     t = np.float32(alpha) * np.asarray(y, dtype=np.float32)
     return f32_to_bf16(x - t)
+
+
+# ---------------------------------------------------------------------------
+# FP8 (e4m3) GEMM operands (Sec. 3.3 reports FP8 on top of HiLo-Token; the
+# scheme below is this implementation's: per-row scaling of every GEMM
+# operand, fp32 accumulation)
+# ---------------------------------------------------------------------------
+
+E4M3_MAX = 448.0
+
+
+def e4m3_encode(t: np.ndarray) -> np.ndarray:
+    """fp32 values -> e4m3 codes (uint8): 1 sign bit, 4 exponent bits (bias
+    7), 3 mantissa bits; round to nearest, ties to even; values beyond the
+    largest finite magnitude 448 saturate to +-448 (NaN is not expected)."""
+    t = np.asarray(t, dtype=np.float32).astype(np.float64)
+    sign = (np.signbit(t)).astype(np.uint8) << 7
+    a = np.abs(t)
+    # quantum of the binade holding a: 2^(e-3) for e >= -6, 2^-9 below
+    # (subnormals); frexp gives a = m 2^x with m in [0.5, 1)
+    _, x = np.frexp(np.where(a > 0, a, 1.0))
+    e = np.maximum(x - 1, -6)
+    q = np.ldexp(1.0, e - 3)
+    m = a / q                       # exact: q is a power of two
+    r = np.floor(m)
+    frac = m - r
+    up = (frac > 0.5) | ((frac == 0.5) & (np.mod(r, 2) == 1))
+    v = (r + up) * q                # rounded magnitude (may step to the next binade)
+    v = np.minimum(v, E4M3_MAX)
+    # bits of the rounded magnitude
+    _, xv = np.frexp(np.where(v > 0, v, 1.0))
+    ev = xv - 1
+    sub = v < 2.0 ** -6
+    exp_field = np.where(sub, 0, ev + 7)
+    mant = np.where(sub, v / 2.0 ** -9, v / np.ldexp(1.0, ev) * 8 - 8)
+    code = (exp_field.astype(np.int64) << 3) | mant.astype(np.int64)
+    return (sign | code.astype(np.uint8)).astype(np.uint8)
+
+
+def e4m3_decode(c: np.ndarray) -> np.ndarray:
+    """e4m3 codes -> values (fp64; 0x7f / 0xff are NaN)."""
+    c = np.asarray(c, dtype=np.uint8).astype(np.int64)
+    s = np.where(c & 0x80, -1.0, 1.0)
+    ef = (c >> 3) & 0xF
+    mf = c & 0x7
+    v = np.where(ef == 0, mf * 2.0 ** -9, (1 + mf / 8.0) * np.ldexp(1.0, ef - 7))
+    v = np.where((c & 0x7F) == 0x7F, np.nan, v)
+    return s * v
+
+
+def quantize_rows(x) -> tuple[np.ndarray, np.ndarray]:
+    """Per-row e4m3 quantisation of an fp32 matrix [R, C]: amax = max |x| of
+    the row, inv = 448 / amax and scale = amax / 448 (each one correctly
+    rounded fp32 division; 1 for an all-zero row), code = e4m3(x * inv) with
+    the product rounded to fp32 first. Returns (codes uint8 [R, C], scale
+    fp32 [R]); code value times scale approximates x."""
+    x = np.asarray(x, dtype=np.float32)
+    amax = np.abs(x).max(axis=1) if x.shape[1] else np.zeros(x.shape[0], np.float32)
+    pos = amax > 0
+    inv = np.where(pos, np.float32(E4M3_MAX) / np.where(pos, amax, 1).astype(np.float32), 1).astype(np.float32)
+    scale = np.where(pos, amax.astype(np.float32) / np.float32(E4M3_MAX), 1).astype(np.float32)
+    codes = e4m3_encode((x * inv[:, None]).astype(np.float32))
+    return codes, scale
+
+
+def dequant(codes, scale) -> np.ndarray:
+    return e4m3_decode(codes) * np.asarray(scale, np.float64)[:, None]
+
+
+def gemm_e4m3(a64, wq, bias=None) -> np.ndarray:
+    """One FP8 GEMM as the kernels take it: the activations a [R, K] rounded
+    to fp32 and quantised per row, the weights wq = (codes [N, K], scale [N])
+    quantised per output channel; out = (codes_A codes_W^T) * scale_A[r] *
+    scale_W[o] (+ bias), in fp64."""
+    ca, sa = quantize_rows(np.asarray(a64, dtype=np.float32))
+    cw, sw = wq
+    acc = e4m3_decode(ca) @ e4m3_decode(cw).T
+    out = acc * sa.astype(np.float64)[:, None] * np.asarray(sw, np.float64)[None, :]
+    return out if bias is None else out + _w(bias)
+
+
+def f32_to_f16_sat(a) -> np.ndarray:
+    """fp32 -> fp16 (round to nearest even, saturating at +-65504), as fp64."""
+    a = np.clip(np.asarray(a, dtype=np.float64), -65504.0, 65504.0)
+    return a.astype(np.float32).astype(np.float16).astype(np.float64)
+
+
+def block_fp8(u_txt, u_img, cu_img, T: int, weights_q, heads: int, mlp: bool):
+    """The MMDiT block of ``block`` with e4m3 GEMM operands, in the order the
+    kernels take: LayerNorm -> fp32 -> per-row e4m3; QKV = (codes_A codes_W^T)
+    * scale_A[r] * scale_W[o] + b, rounded to bf16; attention (fp64) rounded
+    to bf16 -> per-row e4m3 -> out-projection; LayerNorm-2 -> per-row e4m3 ->
+    MLP1 -> GELU rounded to fp16 -> per-row e4m3 -> MLP2. The residual stream
+    stays fp64 here (fp32 in the kernels). ``weights_q`` per stream holds
+    (codes, scale) for w_qkv, w_o, w_1, w_2 (see quantize_weights) and the
+    bf16 biases. Returns fp64 (txt, img)."""
+    ut = _as_f64(u_txt)
+    ui = _as_f64(u_img)
+    d = ut.shape[1] if ut.size else ui.shape[1]
+    hd = d // heads
+    B = len(cu_img) - 1
+
+    q_gemm = gemm_e4m3
+    streams = ((ut, weights_q.txt), (ui, weights_q.img))
+    qkv = [bf16_to_f32(f32_to_bf16(q_gemm(layer_norm(u), w.w_qkv, w.b_qkv))).astype(np.float64) if u.size else
+           np.zeros((0, 3 * d)) for u, w in streams]
+    att = [np.zeros_like(ut), np.zeros_like(ui)]
+    for b in range(B):
+        t0, t1 = b * T, (b + 1) * T
+        i0, i1 = int(cu_img[b]), int(cu_img[b + 1])
+        joint = np.concatenate([qkv[0][t0:t1], qkv[1][i0:i1]], axis=0)
+        o = np.empty((joint.shape[0], d))
+        for h in range(heads):
+            c = slice(h * hd, (h + 1) * hd)
+            o[:, c] = softmax_attention(joint[:, c], joint[:, d:][:, c], joint[:, 2 * d:][:, c])
+        att[0][t0:t1] = o[:T]
+        att[1][i0:i1] = o[T:]
+    out = []
+    for (u, w), a in zip(streams, att):
+        if u.size == 0:
+            out.append(u)
+            continue
+        a16 = bf16_to_f32(f32_to_bf16(a)).astype(np.float64)
+        u = u + q_gemm(a16, w.w_o, w.b_o)
+        if mlp:
+            hid = f32_to_f16_sat(gelu_tanh(q_gemm(layer_norm(u), w.w_1, w.b_1)))
+            u = u + q_gemm(hid, w.w_2, w.b_2)
+        out.append(u)
+    return out[0], out[1]
+
+
+@dataclasses.dataclass
+class StreamWeightsQ:
+    w_qkv: tuple
+    b_qkv: np.ndarray
+    w_o: tuple
+    b_o: np.ndarray
+    w_1: tuple = None
+    b_1: np.ndarray = None
+    w_2: tuple = None
+    b_2: np.ndarray = None
+
+
+@dataclasses.dataclass
+class BlockWeightsQ:
+    txt: StreamWeightsQ
+    img: StreamWeightsQ
+
+
+def quantize_weights(w) -> BlockWeightsQ:
+    """Per-output-channel e4m3 weights (each row of W[out, in] quantised as
+    in quantize_rows, from the bf16 values); biases stay bf16."""
+    def one(s):
+        q = lambda m: quantize_rows(bf16_to_f32(m)) if m is not None else None
+        return StreamWeightsQ(q(s.w_qkv), s.b_qkv, q(s.w_o), s.b_o, q(s.w_1), s.b_1, q(s.w_2), s.b_2)
+    return BlockWeightsQ(one(w.txt), one(w.img))
 
 
 # ---------------------------------------------------------------------------

@@ -694,6 +694,102 @@ def test_row_sizes_count_the_grid(granular):
                 assert n[r] == size * size
 
 
+# ------------------------------------------------------------------- FP8 --
+
+def test_e4m3_codes_roundtrip_and_match_torch():
+    """Every finite e4m3 code decodes and re-encodes to itself (both zeros
+    keep their sign); in-range fp32 values round like torch's float8_e4m3fn
+    cast (round to nearest, ties to even)."""
+    codes = np.arange(256, dtype=np.uint8)
+    vals = O.e4m3_decode(codes)
+    fin = ~np.isnan(vals)
+    assert fin.sum() == 254 and np.nanmax(vals) == 448.0 and np.nanmin(vals) == -448.0
+    assert np.array_equal(O.e4m3_encode(vals[fin].astype(np.float32)), codes[fin])
+    x = (np.random.default_rng(7).standard_normal(200000) * 40).astype(np.float32)
+    x = np.concatenate([x[np.abs(x) <= 448], (np.random.default_rng(8).random(20000) * 0.03).astype(np.float32)])
+    ref = torch.from_numpy(x).to(torch.float8_e4m3fn).view(torch.uint8).numpy()
+    assert np.array_equal(O.e4m3_encode(x), ref)
+
+
+def test_e4m3_ties_saturation_subnormals():
+    t = np.array([1.0625, 1.1875, 1.0625 + 2 ** -20, 464.0, 1000.0, -1e30, 2 ** -10, 3 * 2 ** -10, 2 ** -6,
+                  0.9375 + 2 ** -5], dtype=np.float32)
+    got = O.e4m3_decode(O.e4m3_encode(t))
+    # 1.0625 is halfway between 1 and 1.125: to the even mantissa (1);
+    # 1.1875 halfway between 1.125 and 1.25: to 1.25; just above halfway
+    # rounds up; beyond 448 saturates; 2^-10 is half the smallest
+    # subnormal 2^-9 (ties to 0); 3 * 2^-10 rounds to 2 * 2^-9; 2^-6 is
+    # the smallest normal; 0.96875 sits halfway between 0.9375 and 1.0
+    assert got.tolist() == [1.0, 1.25, 1.125, 448.0, 448.0, -448.0, 0.0, 2 ** -8, 2 ** -6, 1.0]
+
+
+def test_quantize_rows_error_bound():
+    rng = np.random.default_rng(9)
+    x = (rng.standard_normal((64, 300)) * np.exp(rng.uniform(-8, 8, (64, 1)))).astype(np.float32)
+    x[3] = 0.0
+    codes, scale = O.quantize_rows(x)
+    deq = O.dequant(codes, scale)
+    assert scale[3] == 1.0 and np.all(deq[3] == 0)
+    amax = np.abs(x).max(axis=1)
+    # the row maximum maps to the largest code
+    assert np.all(np.abs(O.e4m3_decode(codes[np.arange(64), np.abs(x).argmax(axis=1)]))[amax > 0] == 448.0)
+    # half a quantum of the binade (2^-4 relative), or half the subnormal
+    # quantum 2^-10 of the scaled value, plus fp32 rounding of x * inv
+    bound = np.maximum(2.0 ** -4 * np.abs(x), 2.0 ** -10 * scale[:, None]) * (1 + 2.0 ** -20)
+    assert np.all(np.abs(deq - x) <= bound)
+
+
+def test_gemm_e4m3_exact_on_representable_operands_and_scale_invariance():
+    rng = np.random.default_rng(10)
+    # rows whose maximum is 448 * 2^k and all entries e4m3 values times 2^k:
+    # quantisation is exact, so the GEMM is the exact product
+    grid = O.e4m3_decode(np.arange(0, 126, dtype=np.uint8))
+    def rep(shape, k):
+        m = rng.choice(grid, size=shape) * rng.choice([-1, 1], size=shape)
+        m[:, 0] = 448.0
+        return (m * 2.0 ** k).astype(np.float32)
+    a = rep((5, 64), -7)
+    w = rep((7, 64), -9)
+    wq = O.quantize_rows(w)
+    assert np.array_equal(O.dequant(*wq), w.astype(np.float64))
+    assert np.array_equal(O.gemm_e4m3(a, wq), a.astype(np.float64) @ w.astype(np.float64).T)
+    # a power-of-two factor on one weight row moves into its scale only
+    w2 = w.copy()
+    w2[2] *= 8
+    out1, out2 = O.gemm_e4m3(a, wq), O.gemm_e4m3(a, O.quantize_rows(w2))
+    assert np.array_equal(out2[:, 2], 8 * out1[:, 2]) and np.array_equal(np.delete(out2, 2, 1), np.delete(out1, 2, 1))
+
+
+def test_block_fp8_error_follows_the_e4m3_model():
+    """Against the exact block, the FP8 block's error is a few percent of the
+    block's update (e4m3 keeps 3 mantissa bits: at most 2^-4 relative per
+    operand, about 3.6% RMS, so about 5% per GEMM output): between 1% and
+    10% of ||out - u||. A swapped or missing scale is off by orders of
+    magnitude."""
+    rng = np.random.default_rng(11)
+    d, heads, T = 256, 2, 16
+    std = 1 / np.sqrt(d)   # logits of order one: attention does not amplify q/k errors
+
+    def one():
+        s = I.StreamWeights(w_qkv=bits(rng.normal(0, std, (3 * d, d))), b_qkv=bits(rng.normal(0, std, 3 * d)),
+                            w_o=bits(rng.normal(0, std, (d, d))), b_o=bits(rng.normal(0, std, d)))
+        s.w_1, s.b_1 = bits(rng.normal(0, std, (4 * d, d))), bits(rng.normal(0, std, 4 * d))
+        s.w_2, s.b_2 = bits(rng.normal(0, std / 2, (d, 4 * d))), bits(rng.normal(0, std, d))
+        return s
+    w = I.BlockWeights(txt=one(), img=one())
+    ut = bits(rng.standard_normal((T, d)))
+    ui = bits(rng.standard_normal((40, d)))
+    et, ei = O.block(ut, ui, [0, 40], T, w, heads, True)
+    qt, qi = O.block_fp8(ut, ui, [0, 40], T, O.quantize_weights(w), heads, True)
+    for got, ref, u in ((qi, ei, ui), (qt, et, ut)):
+        delta = ref - O.bf16_to_f32(u).astype(np.float64)
+        r = np.linalg.norm(got - ref) / np.linalg.norm(delta)
+        assert 0.01 < r < 0.1, r
+    # a block with no image rows leaves the text stream's FP8 result alone
+    qt0, _ = O.block_fp8(ut, ui[:0], [0, 0], T, O.quantize_weights(w), heads, True)
+    assert qt0.shape == qt.shape
+
+
 def test_keep_ratio_one_is_dense_block():
     wl = I.tiny_layer(keep_ratio=1024, H=16, W=16, d=64, heads=2, T=8)
     b = I.make_batch(wl)
