@@ -408,6 +408,60 @@ def time_lf(H, torch, stream, wl, dw, inputs, steps: int, lf: int = 4) -> dict:
             "low_frequency_tokens": int(counts[1]), "packed_image_rows": int(hp.split.cu_img[-1].item())}
 
 
+def time_fp8(H, I, torch, stream, wl, hp, inputs, bf16_peak: float, steps: int) -> dict:
+    """FP8 (e4m3) GEMM operands on the timed workload: the block with and
+    without them on the same packed rows, the hot path with them, and the FP8
+    GEMMs' throughput (24 M d^2 FLOP per block, from the per-stage events)."""
+    x, text, mask, kk, km = inputs
+    w8 = H.DeviceWeightsFP8.from_host(I.make_weights(wl.d, wl.mlp, seed=I.weight_seed(wl)))
+    hp.enable_fp8([w8])
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for _ in range(steps):
+            fn()
+        s1.record(stream)
+        torch.cuda.synchronize()
+        return s0.elapsed_time(s1) / steps
+
+    path_ms = timed(lambda: hp.run(x, text, mask, kk, km, fp8=True))
+    H.hilo_sync_status()
+    sh, cu = hp.shape, hp.split.cu_img
+    b8 = timed(lambda: H.hilo_block_forward_fp8(sh, w8, cu, hp.cap, text, hp.packed, H.HILO_BF16, hp.out, hp.ws,
+                                                hp.ws_bytes, stream))
+    b16 = timed(lambda: H.hilo_block_forward(sh, hp.weights[0], cu, hp.cap, text, hp.packed, H.HILO_BF16, hp.out,
+                                             hp.ws, hp.ws_bytes, stream))
+    # per-stage times of the FP8 block (the bf16 block's stage marks)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(8)]
+    for e in ev:
+        e.record(stream)
+    H.hilo_set_stage_events(ev)
+    for _ in range(3):
+        H.hilo_block_forward_fp8(sh, w8, cu, hp.cap, text, hp.packed, H.HILO_BF16, hp.out, hp.ws, hp.ws_bytes,
+                                 stream)
+    torch.cuda.synchronize()
+    H.hilo_set_stage_events([])
+    st = [ev[i].elapsed_time(ev[i + 1]) for i in range(7)]
+    H.hilo_sync_status()
+    M = wl.B * wl.T + int(cu[-1].item())
+    d = wl.d
+    # stages: 1 QKV, 2 attention + its quantisation, 3 out-projection, 4 LN2,
+    # 5 MLP1 + hidden quantisation, 6 MLP2
+    gemm_ms = st[1] + st[3] + st[5] + st[6]
+    tflops = 24.0 * M * d * d / (gemm_ms * 1e-3) / 1e12
+    return {"block_ms_fp8": b8, "block_ms_bf16_same_rows": b16, "block_speedup": b16 / b8,
+            "hot_path_ms": path_ms, "image_tokens_per_s": wl.B * wl.N / (path_ms * 1e-3),
+            "stage_ms": {"ln1": st[0], "qkv": st[1], "attention_and_quant": st[2], "out_proj": st[3],
+                         "ln2": st[4], "mlp1_and_quant": st[5], "mlp2": st[6]},
+            "gemm_TFLOP/s_incl_hidden_quant": tflops,
+            "frac_fp8_peak": tflops / (2 * bf16_peak),
+            "fp8_peak_note": "2 x measured bf16 dense (the nominal fp8 : bf16 ratio)"}
+
+
 def time_configs(H, I, torch, stream, steps: int):
     """Hot path, compressed block and dense block of each workload configuration.
 
@@ -714,6 +768,7 @@ def run_hilo(args):
         extras["regions"] = time_regions(H, torch, stream, wl, hp, (x, text, mask, kk, km), hbm_peak, Ks)
         extras["proportional_attention"] = time_prop(H, torch, stream, wl, hp, dw, (x, text, mask, kk, km), Ks)
         extras["low_frequency_set"] = time_lf(H, torch, stream, wl, dw, (x, text, mask, kk, km), Ks)
+        extras["fp8"] = time_fp8(H, I, torch, stream, wl, hp, (x, text, mask, kk, km), bf16_peak, Ks)
         if world == 1:
             extras["configs"] = time_configs(H, I, torch, stream, steps=20)
         # dense block: every grid token is its own row, no score/split/pack/unpack

@@ -61,8 +61,8 @@ enum {
  * separate low-frequency mode, shape.lf > 0). */
 enum { HILO_KEEP = 0, HILO_POOL2 = 1, HILO_POOL4 = 2, HILO_LF = 3 };
 
-/* Input dtypes of hilo_block_forward. */
-enum { HILO_BF16 = 0, HILO_F32 = 1 };
+/* Input dtypes of hilo_block_forward (HILO_F16: hilo_quantize_rows_e4m3). */
+enum { HILO_BF16 = 0, HILO_F32 = 1, HILO_F16 = 2 };
 
 /*
  * Problem shape.
@@ -141,6 +141,23 @@ typedef struct {
 typedef struct {
   hilo_stream_weights txt, img;
 } hilo_block_weights;
+
+/*
+ * FP8 weights of one stream for hilo_block_forward_fp8: each matrix W[out, in]
+ * as e4m3 codes with one fp32 dequantisation scale per output channel (row),
+ * e.g. from hilo_quantize_rows_e4m3 of the bf16 matrix; biases bf16.
+ *   w_*  uint8 e4m3 [out, in], 16-byte aligned
+ *   s_*  fp32 [out], 16-byte aligned: W[o, i] ~ e4m3(w[o, i]) * s[o]
+ */
+typedef struct {
+  const void *w_qkv, *w_o, *w_1, *w_2;
+  const float *s_qkv, *s_o, *s_1, *s_2;
+  const void *b_qkv, *b_o, *b_1, *b_2;
+} hilo_stream_weights_fp8;
+
+typedef struct {
+  hilo_stream_weights_fp8 txt, img;
+} hilo_block_weights_fp8;
 
 /* Readable name of a status code. */
 const char* hilo_status_string(int status);
@@ -349,6 +366,40 @@ int hilo_unpack_delta(const hilo_shape* shape, const float* out_img, const void*
  */
 int hilo_unpack_update(const hilo_shape* shape, const float* out_img,
                        const hilo_split_out* split, void* x, float alpha, void* stream);
+
+/*
+ * hilo_quantize_rows_e4m3 -- per-row e4m3 quantisation: for each row, amax =
+ * the largest magnitude, inv = 448 / amax and scale = amax / 448 (correctly
+ * rounded fp32 divisions; 1 and 1 for an all-zero row), dst = e4m3(src * inv)
+ * with the product rounded to fp32, then round to nearest even and saturate
+ * at +-448. Used for the weights of hilo_block_forward_fp8 (once, at load)
+ * and, inside it, for the attention output and the MLP hidden rows.
+ *   src    [rows, cols] device, HILO_BF16, HILO_F16 or HILO_F32, 16-byte aligned
+ *   dst    uint8 e4m3 [rows, cols] device, 16-byte aligned; cols a multiple of 8
+ *   scale  fp32 [rows] device
+ */
+int hilo_quantize_rows_e4m3(const void* src, int src_dtype, int64_t rows, int32_t cols, uint8_t* dst,
+                            float* scale, void* stream);
+
+/* Workspace bytes hilo_block_forward_fp8 needs for `cap` image-row capacity. */
+size_t hilo_block_fp8_workspace_bytes(const hilo_shape* shape, int32_t cap);
+
+/*
+ * hilo_block_forward_fp8 -- the block of hilo_block_forward with e4m3 GEMM
+ * operands and fp32 accumulation (paper Sec. 3.3 reports FP8 on top of
+ * HiLo-Token; this scaling scheme is the library's): every GEMM input row is
+ * quantised per row (the LayerNorm outputs inside the LayerNorm kernel, the
+ * attention output and the MLP hidden rows by a row pass), the weights per
+ * output channel; each output is acc * row scale * column scale + bias. The
+ * q|k|v rows, the attention and the residual stream are as in
+ * hilo_block_forward (bf16 / fp32); the MLP hidden rows are fp16 before
+ * their quantisation. Needs d a multiple of 256 and at least 1024 (else
+ * HILO_ERR_SHAPE). Other arguments, layouts, in-place use and errors as
+ * hilo_block_forward, with hilo_block_fp8_workspace_bytes of workspace.
+ */
+int hilo_block_forward_fp8(const hilo_shape* shape, const hilo_block_weights_fp8* weights,
+                           const int32_t* cu_img, int32_t cap, const void* in_txt, const void* in_img,
+                           int in_dtype, float* out, void* ws, size_t ws_bytes, void* stream);
 
 /*
  * hilo_block_forward_static_ws -- hilo_block_forward without a workspace

@@ -117,6 +117,27 @@ BlockWs block_ws_layout(const hilo_shape* s, int32_t cap) {
   return w;
 }
 
+// FP8 block: one e4m3 buffer for the A operand of every GEMM (LayerNorm
+// outputs, attention output, MLP hidden; each used before the next is
+// written, in stream order) with its per-row scales, then bf16 q|k|v and
+// attention rows and the fp16 MLP hidden rows.
+struct BlockWs8 {
+  size_t q8, qs, qkv, attn, hid, total;
+};
+
+BlockWs8 block_fp8_ws_layout(const hilo_shape* s, int32_t cap) {
+  const size_t R = static_cast<size_t>(s->B) * s->T + static_cast<size_t>(cap);
+  const size_t d = static_cast<size_t>(s->d);
+  BlockWs8 w;
+  w.q8 = 0;
+  w.qs = w.q8 + align256(R * (s->mlp ? 4 * d : d));
+  w.qkv = w.qs + align256(R * 4);
+  w.attn = w.qkv + align256(R * 3 * d * 2);
+  w.hid = w.attn + align256(R * d * 2);
+  w.total = w.hid + (s->mlp ? align256(R * 4 * d * 2) : 0);
+  return w;
+}
+
 }  // namespace
 
 namespace hilo {
@@ -151,6 +172,10 @@ bool encode_tmap_2d(CUtensorMap* map, TmapType type, const void* base, uint64_t 
   if (type == TMAP_F32) {
     dt = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
     esize = 4;
+  }
+  if (type == TMAP_U8) {
+    dt = CU_TENSOR_MAP_DATA_TYPE_UINT8;
+    esize = 1;
   }
   cuuint64_t dims[2] = {inner, outer};
   cuuint64_t strides[1] = {row_stride_elems * esize};
@@ -367,7 +392,7 @@ static int block_forward_impl(const hilo_shape* shape, const hilo_block_weights*
   stage_mark(0, s);
   // the residual is read from the input by the out-projection epilogue (no
   // fp32 copy of it is made) unless the input already is the output buffer
-  cudaError_t e = hilo::launch_layernorm(in_txt, in_img, in_f32, nullptr, ln, 0, cu_img, B, BT, cap, d,
+  cudaError_t e = hilo::launch_layernorm(in_txt, in_img, in_f32, nullptr, ln, 0, nullptr, cu_img, B, BT, cap, d,
                                          dev->num_sms, s);
   if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: layernorm 1");
   count(1);
@@ -419,7 +444,7 @@ static int block_forward_impl(const hilo_shape* shape, const hilo_block_weights*
   if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: out-projection gemm");
   stage_mark(4, s);
   if (shape->mlp) {
-    e = hilo::launch_layernorm(out, out + static_cast<size_t>(BT) * d, 1, nullptr, ln, 1, cu_img, B, BT,
+    e = hilo::launch_layernorm(out, out + static_cast<size_t>(BT) * d, 1, nullptr, ln, 1, nullptr, cu_img, B, BT,
                                cap, d, dev->num_sms, s);
     if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: layernorm 2");
     count(1);
@@ -449,6 +474,150 @@ int hilo_block_forward_prop(const hilo_shape* shape, const hilo_block_weights* w
     return fail(HILO_ERR_ARG, "hilo_block_forward_prop: n_img must be 4-byte aligned");
   return block_forward_impl(shape, w, cu_img, cap, in_txt, in_img, in_dtype, n_img, out, ws, ws_bytes,
                             stream);
+}
+
+int hilo_quantize_rows_e4m3(const void* src, int src_dtype, int64_t rows, int32_t cols, uint8_t* dst,
+                            float* scale, void* stream) {
+  if (!src || !dst || !scale) return fail(HILO_ERR_ARG, "hilo_quantize_rows_e4m3: NULL pointer");
+  if (src_dtype != HILO_BF16 && src_dtype != HILO_F16 && src_dtype != HILO_F32)
+    return fail(HILO_ERR_ARG, "hilo_quantize_rows_e4m3: src_dtype=%d", src_dtype);
+  if (rows < 0 || rows > 0x7fffffff || cols < 0 || cols % 8)
+    return fail(HILO_ERR_ARG, "hilo_quantize_rows_e4m3: rows=%lld, cols=%d (a multiple of 8)",
+                static_cast<long long>(rows), cols);
+  if ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15)
+    return fail(HILO_ERR_ARG, "hilo_quantize_rows_e4m3: src and dst must be 16-byte aligned");
+  DevInfo* dev;
+  int st;
+  if ((st = current_device(&dev))) return st;
+  if (rows == 0 || cols == 0) return HILO_OK;
+  const int type = src_dtype == HILO_BF16 ? 0 : (src_dtype == HILO_F16 ? 1 : 2);
+  cudaError_t e = hilo::launch_quant_rows(src, type, cols, static_cast<int>(rows), nullptr, 0, 0, 0, dst, scale,
+                                          dev->num_sms, static_cast<cudaStream_t>(stream));
+  if (e == cudaSuccess) count(1);
+  return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_quantize_rows_e4m3");
+}
+
+size_t hilo_block_fp8_workspace_bytes(const hilo_shape* shape, int32_t cap) {
+  if (!shape || cap < 0) return 0;
+  return block_fp8_ws_layout(shape, cap).total;
+}
+
+int hilo_block_forward_fp8(const hilo_shape* shape, const hilo_block_weights_fp8* w, const int32_t* cu_img,
+                           int32_t cap, const void* in_txt, const void* in_img, int in_dtype, float* out,
+                           void* ws, size_t ws_bytes, void* stream) {
+  int st = check_shape(shape, true);
+  if (st) return st;
+  if (shape->d < 1024 || shape->d % 256)
+    return fail(HILO_ERR_SHAPE, "hilo_block_forward_fp8: d=%d must be a multiple of 256, at least 1024",
+                shape->d);
+  if (!w || !cu_img || !in_img || !out) return fail(HILO_ERR_ARG, "hilo_block_forward_fp8: NULL pointer");
+  if (shape->T > 0 && !in_txt) return fail(HILO_ERR_ARG, "hilo_block_forward_fp8: in_txt is NULL with T>0");
+  if (in_dtype != HILO_BF16 && in_dtype != HILO_F32)
+    return fail(HILO_ERR_ARG, "hilo_block_forward_fp8: in_dtype=%d", in_dtype);
+  if (cap < 0) return fail(HILO_ERR_ARG, "hilo_block_forward_fp8: cap=%d", cap);
+  const hilo_stream_weights_fp8* sw[2] = {&w->txt, &w->img};
+  for (int i = 0; i < 2; ++i) {
+    if (i == 0 && shape->T == 0) continue;
+    const hilo_stream_weights_fp8& x = *sw[i];
+    if (!x.w_qkv || !x.s_qkv || !x.b_qkv || !x.w_o || !x.s_o || !x.b_o)
+      return fail(HILO_ERR_ARG, "hilo_block_forward_fp8: %s attention weight is NULL", i ? "image" : "text");
+    if (shape->mlp && (!x.w_1 || !x.s_1 || !x.b_1 || !x.w_2 || !x.s_2 || !x.b_2))
+      return fail(HILO_ERR_ARG, "hilo_block_forward_fp8: %s MLP weight is NULL", i ? "image" : "text");
+    if ((reinterpret_cast<uintptr_t>(x.s_qkv) | reinterpret_cast<uintptr_t>(x.s_o) |
+         reinterpret_cast<uintptr_t>(x.s_1) | reinterpret_cast<uintptr_t>(x.s_2)) & 15)
+      return fail(HILO_ERR_ARG, "hilo_block_forward_fp8: weight scales must be 16-byte aligned");
+  }
+  const BlockWs8 L = block_fp8_ws_layout(shape, cap);
+  if (!ws || ws_bytes < L.total)
+    return fail(HILO_ERR_WORKSPACE, "hilo_block_forward_fp8: workspace %zu < %zu bytes", ws_bytes, L.total);
+  DevInfo* dev;
+  if ((st = current_device(&dev))) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const int B = shape->B, T = shape->T, d = shape->d;
+  const int BT = B * T;
+  const int R = BT + cap;
+  char* base = static_cast<char*>(ws);
+  uint8_t* q8 = reinterpret_cast<uint8_t*>(base + L.q8);
+  float* qs = reinterpret_cast<float*>(base + L.qs);
+  void* qkv = base + L.qkv;
+  void* attn = base + L.attn;
+  void* hid = base + L.hid;
+  const int in_f32 = in_dtype == HILO_F32;
+  const bool in_place = in_f32 && in_txt == out && in_img == out + static_cast<size_t>(BT) * d;
+  const bool in_place_img = in_f32 && BT == 0 && in_img == out;
+
+  stage_mark(0, s);
+  cudaError_t e = hilo::launch_layernorm(in_txt, in_img, in_f32, nullptr, q8, 2, qs, cu_img, B, BT, cap, d,
+                                         dev->num_sms, s);
+  if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward_fp8: layernorm 1");
+  count(1);
+  stage_mark(1, s);
+  auto gemm = [&](int N, int K, int epi, void* o, const void* wt, const float* st_, const void* bt,
+                  const void* wi, const float* si, const void* bi) {
+    hilo::GemmArgs g;
+    if (epi == hilo::EPI_BIAS_RESIDIN_F32) {
+      g.resid_src[0] = in_txt;
+      g.resid_src[1] = in_img;
+      g.resid_f32 = in_f32;
+    }
+    g.A = q8;
+    g.op_f16 = 0;
+    g.fp8 = 1;
+    g.a_scale = qs;
+    g.R = R;
+    g.N = N;
+    g.K = K;
+    g.epilogue = epi;
+    g.out = o;
+    g.g[0] = {0, BT, nullptr, wt, bt, BT, st_};
+    g.g[1] = {BT, 0, cu_img + B, wi, bi, cap, si};
+    cudaError_t ge = hilo::launch_gemm(g, dev->num_sms, s);
+    if (ge == cudaSuccess) count(1);
+    return ge;
+  };
+  const hilo_stream_weights_fp8 &wt = w->txt, &wi = w->img;
+  e = gemm(3 * d, d, hilo::EPI_BIAS_BF16, qkv, wt.w_qkv, wt.s_qkv, wt.b_qkv, wi.w_qkv, wi.s_qkv, wi.b_qkv);
+  if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward_fp8: qkv gemm");
+  stage_mark(2, s);
+  hilo::AttnArgs aa;
+  aa.qkv = qkv;
+  aa.out = attn;
+  aa.cu_img = cu_img;
+  aa.B = B;
+  aa.T = T;
+  aa.heads = shape->heads;
+  aa.head_dim = d / shape->heads;
+  aa.d = d;
+  aa.R = R;
+  aa.max_img_rows = static_cast<int>(hilo_row_capacity(shape) / shape->B);
+  e = hilo::launch_attention(aa, dev->num_sms, s);
+  if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward_fp8: attention");
+  count(1);
+  e = hilo::launch_quant_rows(attn, 0, d, 0, cu_img, B, BT, cap, q8, qs, dev->num_sms, s);
+  if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward_fp8: attention quantisation");
+  count(1);
+  stage_mark(3, s);
+  e = gemm(d, d, (in_place || in_place_img) ? hilo::EPI_BIAS_RESID_F32 : hilo::EPI_BIAS_RESIDIN_F32, out, wt.w_o,
+           wt.s_o, wt.b_o, wi.w_o, wi.s_o, wi.b_o);
+  if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward_fp8: out-projection gemm");
+  stage_mark(4, s);
+  if (shape->mlp) {
+    e = hilo::launch_layernorm(out, out + static_cast<size_t>(BT) * d, 1, nullptr, q8, 2, qs, cu_img, B, BT, cap,
+                               d, dev->num_sms, s);
+    if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward_fp8: layernorm 2");
+    count(1);
+    stage_mark(5, s);
+    e = gemm(4 * d, d, hilo::EPI_BIAS_GELU_F16, hid, wt.w_1, wt.s_1, wt.b_1, wi.w_1, wi.s_1, wi.b_1);
+    if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward_fp8: mlp1 gemm");
+    e = hilo::launch_quant_rows(hid, 1, 4 * d, 0, cu_img, B, BT, cap, q8, qs, dev->num_sms, s);
+    if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward_fp8: hidden quantisation");
+    count(1);
+    stage_mark(6, s);
+    e = gemm(d, 4 * d, hilo::EPI_BIAS_RESID_F32, out, wt.w_2, wt.s_2, wt.b_2, wi.w_2, wi.s_2, wi.b_2);
+    if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward_fp8: mlp2 gemm");
+    stage_mark(7, s);
+  }
+  return HILO_OK;
 }
 
 int hilo_row_sizes(const hilo_shape* shape, const hilo_split_out* split, float* n_img, int32_t cap,

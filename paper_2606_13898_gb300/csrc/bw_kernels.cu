@@ -899,11 +899,32 @@ __device__ __forceinline__ float ln_block_sum(float v, float* red) {
   return t;
 }
 
+__device__ __forceinline__ float ln_block_max(float v, float* red) {
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  const float t = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
+  __syncthreads();
+  return t;
+}
+
+// e4m3 row quantisation constants from the row's largest magnitude: inv =
+// 448 / amax and scale = amax / 448, each one correctly rounded division
+// (1 and 1 for an all-zero row)
+__device__ __forceinline__ void e4m3_row_scale(float amax, float& inv, float& scale) {
+  inv = amax > 0.f ? __fdiv_rn(448.0f, amax) : 1.0f;
+  scale = amax > 0.f ? __fdiv_rn(amax, 448.0f) : 1.0f;
+}
+
+// ln_mode: 0 bf16, 1 fp16 (saturating), 2 e4m3 per row (ln_scale[r] = the
+// row's dequantisation scale)
 template <int NCH>
 __global__ void __launch_bounds__(LN_THREADS) layernorm_kernel(const void* __restrict__ in_txt,
                                                                const void* __restrict__ in_img,
                                                                int in_f32, float* resid,
-                                                               uint16_t* __restrict__ ln, int ln_f16,
+                                                               void* __restrict__ ln, int ln_mode,
+                                                               float* __restrict__ ln_scale,
                                                                const int32_t* __restrict__ cu_img,
                                                                int B, int n_txt, int cap, int d) {
   pdl_trigger();
@@ -950,7 +971,30 @@ __global__ void __launch_bounds__(LN_THREADS) layernorm_kernel(const void* __res
     }
     const float rstd = rsqrtf(ln_block_sum(sq, red) * inv_d + 1e-6f);
     float* rr = resid ? resid + static_cast<long long>(r) * d : nullptr;
-    uint16_t* lo = ln + static_cast<long long>(r) * d;
+    if (ln_mode == 2) {
+      float am = 0.f;
+#pragma unroll
+      for (int t = 0; t < NCH; ++t)
+        if (512 * t + 4 * static_cast<int>(threadIdx.x) < d) {
+#pragma unroll
+          for (int i = 0; i < 4; ++i) am = fmaxf(am, fabsf((v[4 * t + i] - mean) * rstd));
+        }
+      float inv, scale;
+      e4m3_row_scale(ln_block_max(am, red), inv, scale);
+      uint8_t* q = static_cast<uint8_t*>(ln) + static_cast<long long>(r) * d;
+#pragma unroll
+      for (int t = 0; t < NCH; ++t) {
+        const int c = 512 * t + 4 * threadIdx.x;
+        if (c >= d) continue;
+        if (rr) *reinterpret_cast<float4*>(rr + c) = make_float4(v[4 * t], v[4 * t + 1], v[4 * t + 2], v[4 * t + 3]);
+        *reinterpret_cast<uint32_t*>(q + c) =
+            pack_e4m3x4(__fmul_rn((v[4 * t] - mean) * rstd, inv), __fmul_rn((v[4 * t + 1] - mean) * rstd, inv),
+                        __fmul_rn((v[4 * t + 2] - mean) * rstd, inv), __fmul_rn((v[4 * t + 3] - mean) * rstd, inv));
+      }
+      if (threadIdx.x == 0) ln_scale[r] = scale;
+      continue;
+    }
+    uint16_t* lo = static_cast<uint16_t*>(ln) + static_cast<long long>(r) * d;
 #pragma unroll
     for (int t = 0; t < NCH; ++t) {
       const int c = 512 * t + 4 * threadIdx.x;
@@ -959,7 +1003,7 @@ __global__ void __launch_bounds__(LN_THREADS) layernorm_kernel(const void* __res
       const float y0 = (v[4 * t] - mean) * rstd, y1 = (v[4 * t + 1] - mean) * rstd;
       const float y2 = (v[4 * t + 2] - mean) * rstd, y3 = (v[4 * t + 3] - mean) * rstd;
       uint2 o;
-      if (ln_f16) {
+      if (ln_mode == 1) {
         o.x = pack_f16x2_sat(y0, y1);
         o.y = pack_f16x2_sat(y2, y3);
       } else {
@@ -968,6 +1012,79 @@ __global__ void __launch_bounds__(LN_THREADS) layernorm_kernel(const void* __res
       }
       *reinterpret_cast<uint2*>(lo + c) = o;
     }
+  }
+}
+
+// ==================================================== e4m3 rows =====
+// Per-row e4m3 quantisation: one 256-thread CTA per row. The row's largest
+// magnitude, then each element times 448 / amax (fp32) rounded to e4m3; the
+// dequantisation scale amax / 448 per row. src_type 0 bf16, 1 fp16, 2 fp32;
+// cols a multiple of 8. Rows: rows_static, or n_txt + min(cu_img[B], cap)
+// when cu_img is given (the row space of the block).
+
+constexpr int QR_THREADS = 256;
+
+__device__ __forceinline__ void load8(const void* src, int type, long long i8, float* f) {
+  if (type == 2) {
+    const float4* p = static_cast<const float4*>(src) + 2 * i8;
+    const float4 a = __ldg(p), b = __ldg(p + 1);
+    f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w; f[4] = b.x; f[5] = b.y; f[6] = b.z; f[7] = b.w;
+    return;
+  }
+  const uint4 u = __ldg(static_cast<const uint4*>(src) + i8);
+  if (type == 0) {
+    bf16x8_to_f32(u, f);
+    return;
+  }
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const __half2 h = *reinterpret_cast<const __half2*>(&w[j]);
+    const float2 t = __half22float2(h);
+    f[2 * j] = t.x;
+    f[2 * j + 1] = t.y;
+  }
+}
+
+__global__ void __launch_bounds__(QR_THREADS) quant_rows_kernel(const void* __restrict__ src, int type,
+                                                                int cols, int rows_static,
+                                                                const int32_t* __restrict__ cu_img, int B,
+                                                                int n_txt, int cap, uint8_t* __restrict__ dst,
+                                                                float* __restrict__ scale) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ float red[QR_THREADS / 32];
+  const int rows = cu_img ? n_txt + min(cu_img[B], cap) : rows_static;
+  const int g8 = cols >> 3;
+  for (int r = blockIdx.x; r < rows; r += gridDim.x) {
+    const long long base8 = static_cast<long long>(r) * g8;
+    float am = 0.f;
+    for (int g = threadIdx.x; g < g8; g += QR_THREADS) {
+      float f[8];
+      load8(src, type, base8 + g, f);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) am = fmaxf(am, fabsf(f[i]));
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, off));
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = am;
+    __syncthreads();
+    am = red[0];
+#pragma unroll
+    for (int w = 1; w < QR_THREADS / 32; ++w) am = fmaxf(am, red[w]);
+    __syncthreads();
+    float inv, sc;
+    e4m3_row_scale(am, inv, sc);
+    // second pass: the row is in L1 / L2 from the first
+    for (int g = threadIdx.x; g < g8; g += QR_THREADS) {
+      float f[8];
+      load8(src, type, base8 + g, f);
+      uint2 o;
+      o.x = pack_e4m3x4(__fmul_rn(f[0], inv), __fmul_rn(f[1], inv), __fmul_rn(f[2], inv), __fmul_rn(f[3], inv));
+      o.y = pack_e4m3x4(__fmul_rn(f[4], inv), __fmul_rn(f[5], inv), __fmul_rn(f[6], inv), __fmul_rn(f[7], inv));
+      reinterpret_cast<uint2*>(dst)[base8 + g] = o;
+    }
+    if (threadIdx.x == 0) scale[r] = sc;
   }
 }
 
@@ -1079,6 +1196,15 @@ cudaError_t launch_unpack_update(const float* out_img, const int32_t* tok_row, v
                     out_img, tok_row, static_cast<__nv_bfloat16*>(x), ntok, d, alpha);
 }
 
+cudaError_t launch_quant_rows(const void* src, int type, int cols, int rows_static, const int32_t* cu_img,
+                              int B, int n_txt, int cap, uint8_t* dst, float* scale, int num_sms,
+                              cudaStream_t st) {
+  const long long rmax = cu_img ? static_cast<long long>(n_txt) + cap : rows_static;
+  if (rmax <= 0) return cudaSuccess;
+  return launch_pdl(quant_rows_kernel, dim3(grid_for(rmax, 1, num_sms, 8)), dim3(QR_THREADS), 0, st, src, type,
+                    cols, rows_static, cu_img, B, n_txt, cap, dst, scale);
+}
+
 cudaError_t launch_bf16_to_f16(const void* src, void* dst, long long n, int num_sms,
                                cudaStream_t st) {
   if (n % 8) return cudaErrorInvalidValue;
@@ -1088,15 +1214,15 @@ cudaError_t launch_bf16_to_f16(const void* src, void* dst, long long n, int num_
 }
 
 cudaError_t launch_layernorm(const void* in_txt, const void* in_img, int in_f32, float* resid,
-                             void* ln, int ln_f16, const int32_t* cu_img, int B, int n_txt,
+                             void* ln, int ln_mode, float* ln_scale, const int32_t* cu_img, int B, int n_txt,
                              int cap, int d, int num_sms, cudaStream_t st) {
   const dim3 grid(grid_for(static_cast<long long>(n_txt) + cap, 1, num_sms, 16));
-  uint16_t* lo = static_cast<uint16_t*>(ln);
+  void* lo = ln;
   switch ((d + 511) / 512) {
 #define HILO_LN_CASE(NC)                                                                      \
   case NC:                                                                                    \
     return launch_pdl(layernorm_kernel<NC>, grid, dim3(LN_THREADS), 0, st, in_txt, in_img, in_f32, \
-                      resid, lo, ln_f16, cu_img, B, n_txt, cap, d);
+                      resid, lo, ln_mode, ln_scale, cu_img, B, n_txt, cap, d);
     HILO_LN_CASE(1)
     HILO_LN_CASE(2)
     HILO_LN_CASE(3)

@@ -16,6 +16,11 @@
 // "empty" and "accumulator ready" barriers are signalled in both CTAs by a
 // multicast commit; "accumulator free" collects 8 arrivals (4 epilogue warps
 // x 2 CTAs) in the even CTA. Every wait is bounded.
+//
+// FP8 (e4m3 A and W, kind::f8f6f4): a k-block is the same 128-byte swizzled
+// row of shared memory holding 128 elements instead of 64, and each MMA
+// consumes 32 of them; the epilogue multiplies each accumulator by its row's
+// A scale and its column's W scale before the bias.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -43,6 +48,8 @@ constexpr int SPLIT_MIN_KB = 16;            // shortest K piece of a tile cut al
 struct Params {
   int N, K;
   uint32_t idesc;
+  const float* a_scale;     // FP8: dequantisation scale per row of A (row space)
+  const float* b_scale[2];  // FP8: per output column, per weight group
   int row_base[2];
   int rows_static[2];
   const int32_t* rows_dev[2];
@@ -134,10 +141,13 @@ struct WorkIter {
   }
 };
 
+template <bool FP8>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     gemm2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                  const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmOut,
                  const __grid_constant__ Params p) {
+  // elements per k-block: one 128-byte swizzled row of A / W
+  constexpr int BKE = FP8 ? 128 : BK;
   extern __shared__ unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -186,7 +196,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
   cluster_sync();  // both CTAs' barriers are initialised before any remote use
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const int kblocks = p.K / BK;
+  const int kblocks = p.K / BKE;
   // The weights do not depend on the previous kernel: while it finishes,
   // pull the first k-blocks of this pair's first weight tile into L2. The
   // tile is exact when it lies in a group whose row count is static (the
@@ -205,7 +215,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       n = (cid - mt0 * nt) % nt;
     }
     const int y = n * PN + 128 * static_cast<int>(rank);
-    for (int kb = 0; kb < min(kblocks, STAGES); ++kb) tma_prefetch_l2_2d(tb, kb * BK, y);
+    for (int kb = 0; kb < min(kblocks, STAGES); ++kb) tma_prefetch_l2_2d(tb, kb * BKE, y);
   }
   pdl_wait();  // the row counts and A are written by the previous kernel
   sc.init(p);
@@ -231,8 +241,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
           unsigned char* sa = smem + stage * STAGE_BYTES;
           const uint32_t full_cl = mapa_shared(smem_u32(&full[stage]), 0);
           if (leader) mbar_arrive_expect_tx(&full[stage], 2 * STAGE_BYTES);
-          tma_load_2d_pair(sa, &tmA, full_cl, kb * BK, tl.m0 + 128 * static_cast<int>(rank));
-          tma_load_2d_pair(sa + HALF_BYTES, tb, full_cl, kb * BK, tl.n0 + 128 * static_cast<int>(rank));
+          tma_load_2d_pair(sa, &tmA, full_cl, kb * BKE, tl.m0 + 128 * static_cast<int>(rank));
+          tma_load_2d_pair(sa + HALF_BYTES, tb, full_cl, kb * BKE, tl.n0 + 128 * static_cast<int>(rank));
           armed |= 1u << stage;
           armed_par = (armed_par & ~(1u << stage)) | (phase << stage);
           if (++stage == STAGES) {
@@ -283,7 +293,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
           for (int k = 0; k < BK / 16; ++k) {
             const uint64_t ad = sw128_desc(a_base + k * 32, 16, 1024);
             const uint64_t bd = sw128_desc(b_base + k * 32, 16, 1024);
-            umma_f16_pair(d_tmem, ad, bd, p.idesc, (kb > w.k0 || k > 0) ? 1u : 0u);
+            if (FP8)
+              umma_f8_pair(d_tmem, ad, bd, p.idesc, (kb > w.k0 || k > 0) ? 1u : 0u);
+            else
+              umma_f16_pair(d_tmem, ad, bd, p.idesc, (kb > w.k0 || k > 0) ? 1u : 0u);
           }
           umma_commit_pair(&empty[stage], 0x3);
           if (++stage == STAGES) {
@@ -320,6 +333,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       // the bias is added once per tile, by the piece that starts at k = 0
       const uint4 bpre = w.k0 == 0 ? epi_bias_preload<PN>(tl.g ? p.bias[1] : p.bias[0], tl.n0, p.N)
                                    : make_uint4(0u, 0u, 0u, 0u);
+      EpiScale escale;
+      if (FP8) escale = epi_scale_preload<PN>(p.a_scale, tl.g ? p.b_scale[1] : p.b_scale[0],
+                                              tl.m0 + 128 * static_cast<int>(rank) + q * 32,
+                                              min(32, max(0, tl.rows - (tl.m0 - tl.row_base) -
+                                                                 (128 * static_cast<int>(rank) + q * 32))),
+                                              tl.n0, p.N);
       if (!mbar_wait_warp(&tfull[acc], acc_phase, abort_flag, err, DEV_TIMEOUT_GEMM + 256 * 5)) break;
       tc_fence_after();
       const int off = 128 * static_cast<int>(rank) + q * 32;  // slab offset in the pair tile
@@ -331,7 +350,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       sl.n0 = tl.n0;
       const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * PN);
       const int a = acc;
-      epilogue_warp<PN>(p, &tmOut, taddr, sl, bpre, stage, buf, [&] {
+      epilogue_warp<PN>(p, &tmOut, taddr, sl, bpre, escale, stage, buf, [&] {
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&tempty[a]), 0));
@@ -353,22 +372,29 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
 
 }  // namespace
 
-bool gemm_pair_supported(const GemmArgs& a) { return a.K % BK == 0 && a.N % PN == 0; }
+bool gemm_pair_supported(const GemmArgs& a) { return a.K % (a.fp8 ? 128 : BK) == 0 && a.N % PN == 0; }
 
 cudaError_t launch_gemm_pair(const GemmArgs& a, int num_sms, cudaStream_t st) {
   if (!gemm_pair_supported(a)) return cudaErrorInvalidValue;
   CUtensorMap tA, tB0, tB1;
-  if (!encode_tmap_bf16_2d(&tA, a.A, a.K, a.R, a.K, BK, 128)) return cudaErrorInvalidValue;
-  if (!encode_tmap_bf16_2d(&tB0, a.g[0].weight ? a.g[0].weight : a.g[1].weight, a.K, a.N, a.K, BK, 128))
+  // FP8: bytes are the elements, 128 per swizzled row (box 128 x 128)
+  const TmapType tt = a.fp8 ? TMAP_U8 : TMAP_BF16;
+  const uint32_t bk = a.fp8 ? 128 : BK;
+  if (!encode_tmap_2d(&tA, tt, a.A, a.K, a.R, a.K, bk, 128)) return cudaErrorInvalidValue;
+  if (!encode_tmap_2d(&tB0, tt, a.g[0].weight ? a.g[0].weight : a.g[1].weight, a.K, a.N, a.K, bk, 128))
     return cudaErrorInvalidValue;
-  if (!encode_tmap_bf16_2d(&tB1, a.g[1].weight ? a.g[1].weight : a.g[0].weight, a.K, a.N, a.K, BK, 128))
+  if (!encode_tmap_2d(&tB1, tt, a.g[1].weight ? a.g[1].weight : a.g[0].weight, a.K, a.N, a.K, bk, 128))
     return cudaErrorInvalidValue;
   CUtensorMap tOut;
   if (!encode_epilogue_map(&tOut, a)) return cudaErrorInvalidValue;
   Params p;
   p.N = a.N;
   p.K = a.K;
-  p.idesc = idesc_kind_f16(PM, PN, 0, 0, a.op_f16 ? 0 : 1);
+  // format code 0: fp16 for kind::f16, E4M3 for kind::f8f6f4
+  p.idesc = idesc_kind_f16(PM, PN, 0, 0, (a.op_f16 || a.fp8) ? 0 : 1);
+  p.a_scale = a.a_scale;
+  p.b_scale[0] = a.g[0].w_scale;
+  p.b_scale[1] = a.g[1].w_scale;
   long long upper = 0;
   for (int g = 0; g < 2; ++g) {
     p.row_base[g] = a.g[g].row_base;
@@ -384,7 +410,8 @@ cudaError_t launch_gemm_pair(const GemmArgs& a, int num_sms, cudaStream_t st) {
   p.resid_src[1] = a.resid_src[1];
   p.resid_f32 = a.resid_f32;
   if (upper <= 0) return cudaSuccess;
-  cudaError_t e = cudaFuncSetAttribute(gemm2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  auto* kern = a.fp8 ? gemm2_kernel<true> : gemm2_kernel<false>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
   if (e != cudaSuccess) return e;
   // persistent grid: as many co-resident CTA pairs as the device holds
   static int max_pairs = 0;
@@ -401,15 +428,15 @@ cudaError_t launch_gemm_pair(const GemmArgs& a, int num_sms, cudaStream_t st) {
     cfg.attrs = &attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, gemm2_kernel, &cfg) != cudaSuccess || n <= 0) {
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n <= 0) {
       cudaGetLastError();
       n = num_sms / 2;
     }
     max_pairs = n;
   }
   const long long pairs = upper < max_pairs ? upper : max_pairs;
-  return launch_pdl(gemm2_kernel, dim3(static_cast<int>(2 * pairs)), dim3(THREADS), SMEM_BYTES, st, tA,
-                    tB0, tB1, tOut, p);
+  return launch_pdl(kern, dim3(static_cast<int>(2 * pairs)), dim3(THREADS), SMEM_BYTES, st, tA, tB0, tB1, tOut,
+                    p);
 }
 
 int gemm2_take_device_error() {

@@ -76,6 +76,40 @@ __device__ __forceinline__ void epi_bias8(const uint4& b, int src, float* f) {
   bf16x8(v, f);
 }
 
+// FP8 dequantisation of one warp's slab: this lane's row scale and 8 column
+// scales per lane (columns n0 + 8 lane .. + 7), taken per chunk by shuffles
+// like the bias. `on` false: no scaling.
+struct EpiScale {
+  bool on = false;
+  float sa = 1.0f;
+  uint4 s0 = make_uint4(0u, 0u, 0u, 0u), s1 = make_uint4(0u, 0u, 0u, 0u);
+};
+
+template <int NC>
+__device__ __forceinline__ EpiScale epi_scale_preload(const float* a_scale, const float* w_scale, int row0,
+                                                      int nvalid, int n0, int N) {
+  EpiScale e;
+  e.on = true;
+  const int lane = lane_id();
+  e.sa = lane < nvalid ? __ldg(a_scale + row0 + lane) : 0.0f;
+  const int col = n0 + 8 * lane;
+  if (8 * lane < NC && col < N) {
+    e.s0 = __ldg(reinterpret_cast<const uint4*>(w_scale + col));
+    e.s1 = __ldg(reinterpret_cast<const uint4*>(w_scale + col + 4));
+  }
+  return e;
+}
+
+// The 8 column scales held by lane `src` (warp-uniform), times the row's.
+__device__ __forceinline__ void epi_scale8(const EpiScale& e, int src, float* f) {
+  const uint32_t w[8] = {__shfl_sync(0xffffffffu, e.s0.x, src), __shfl_sync(0xffffffffu, e.s0.y, src),
+                         __shfl_sync(0xffffffffu, e.s0.z, src), __shfl_sync(0xffffffffu, e.s0.w, src),
+                         __shfl_sync(0xffffffffu, e.s1.x, src), __shfl_sync(0xffffffffu, e.s1.y, src),
+                         __shfl_sync(0xffffffffu, e.s1.z, src), __shfl_sync(0xffffffffu, e.s1.w, src)};
+#pragma unroll
+  for (int i = 0; i < 8; ++i) f[i] = e.sa * __uint_as_float(w[i]);
+}
+
 struct EpiSlab {
   int g;         // row group (weights / bias / residual source)
   int row0;      // row of lane 0 in the row space
@@ -110,12 +144,13 @@ __device__ __forceinline__ unsigned char* epi_box(unsigned char* stage, int& buf
 
 // Epilogue of one warp over NC accumulator columns at TMEM address `taddr`
 // (lane quarter already applied); `bpre` is epi_bias_preload's value for the
-// tile. `release()` is called by the whole warp once the last tcgen05.ld of
-// the accumulator has completed.
+// tile, `sc` the FP8 dequantisation scales (acc * row scale * column scale
+// + bias) or off. `release()` is called by the whole warp once the last
+// tcgen05.ld of the accumulator has completed.
 template <int NC, class P, class Release>
 __device__ __forceinline__ void epilogue_warp(const P& p, const CUtensorMap* tm_out, uint32_t taddr,
-                                              const EpiSlab& s, const uint4& bpre, unsigned char* stage,
-                                              int& buf, Release release) {
+                                              const EpiSlab& s, const uint4& bpre, const EpiScale& sc,
+                                              unsigned char* stage, int& buf, Release release) {
   static_assert(NC <= 256, "one bias uint4 per lane covers 256 columns");
   // parameters held in registers for the whole tile (the asm statements
   // below clobber memory, which would otherwise force them to be re-read)
@@ -142,6 +177,12 @@ __device__ __forceinline__ void epilogue_warp(const P& p, const CUtensorMap* tm_
         float bv[8];
         epi_bias8(bpre, 8 * c + j, bv);
         float w[8];
+        if (sc.on) {
+          float sv[8];
+          epi_scale8(sc, 8 * c + j, sv);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) v[8 * j + i] *= sv[i];
+        }
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
           w[i] = v[8 * j + i] + bv[i];
@@ -204,6 +245,15 @@ __device__ __forceinline__ void epilogue_warp(const P& p, const CUtensorMap* tm_
     float bv[32];
 #pragma unroll
     for (int j = 0; j < 4; ++j) epi_bias8(bpre, 4 * c + j, bv + 8 * j);
+    if (sc.on) {
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        float sv[8];
+        epi_scale8(sc, 4 * c + j, sv);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) v[8 * j + i] *= sv[i];
+      }
+    }
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] += bv[i];
     if (!inplace) {

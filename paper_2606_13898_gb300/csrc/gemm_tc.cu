@@ -251,7 +251,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       sl.n0 = tl.n0;
       const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
       const int a = acc;
-      epilogue_warp<BN>(p, &tmOut, taddr, sl, bpre, stage, buf, [&] {
+      epilogue_warp<BN>(p, &tmOut, taddr, sl, bpre, EpiScale{}, stage, buf, [&] {
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty[a]);
@@ -317,6 +317,11 @@ cudaError_t launch_gemm(const GemmArgs& a, int num_sms, cudaStream_t st) {
   // CTA pairs with 256x256 tiles where N allows (half the W traffic per SM);
   // else one CTA per tile: 256-wide tiles, or 128-wide where N is so small
   // that 256 would leave SMs idle.
+  if (a.fp8) {
+    // e4m3 operands run on the pair kernel only
+    if (a.N >= 1024 && gemm_pair_supported(a)) return launch_gemm_pair(a, num_sms, st);
+    return cudaErrorInvalidValue;
+  }
   if (a.N >= 1024 && gemm_pair_supported(a)) return launch_gemm_pair(a, num_sms, st);
   if (a.N <= 1024) return launch_bn<128>(a, num_sms, st);
   return launch_bn<256>(a, num_sms, st);

@@ -37,8 +37,11 @@ cudaError_t launch_unpack_update(const float* out_img, const int32_t* tok_row, v
                                  long long ntok, int d, float alpha, int num_sms,
                                  cudaStream_t st);
 cudaError_t launch_layernorm(const void* in_txt, const void* in_img, int in_f32, float* resid,
-                             void* ln, int ln_f16, const int32_t* cu_img, int B, int n_txt, int cap,
-                             int d, int num_sms, cudaStream_t st);
+                             void* ln, int ln_mode, float* ln_scale, const int32_t* cu_img, int B, int n_txt,
+                             int cap, int d, int num_sms, cudaStream_t st);
+cudaError_t launch_quant_rows(const void* src, int type, int cols, int rows_static, const int32_t* cu_img,
+                              int B, int n_txt, int cap, uint8_t* dst, float* scale, int num_sms,
+                              cudaStream_t st);
 cudaError_t launch_bf16_to_f16(const void* src, void* dst, long long n, int num_sms,
                                cudaStream_t st);
 
@@ -64,15 +67,18 @@ struct GemmGroupArgs {
   int row_base;
   int rows_static;
   const int32_t* rows_dev;
-  const void* weight;  // bf16 [N, K]
+  const void* weight;  // bf16 [N, K] (e4m3 with GemmArgs::fp8)
   const void* bias;    // bf16 [N]
   int rows_cap;        // upper bound of rows (grid sizing)
+  const float* w_scale = nullptr;  // fp8: dequantisation scale per output column
 };
 
 struct GemmArgs {
   const void* A;  // [R, K] row space, bf16 (op_f16 = 0) or fp16 (op_f16 = 1); W_g the same type
   int R, N, K;
   int op_f16;
+  int fp8 = 0;                     // A and W_g e4m3 (kind::f8f6f4), pair kernel only
+  const float* a_scale = nullptr;  // fp8: dequantisation scale per row of A
   GemmGroupArgs g[2];
   int epilogue;
   void* out;  // bf16 or f32 [R, N]
@@ -105,7 +111,7 @@ int attn_take_device_error();
 int set_error(int status, const char* msg);
 
 // ---- tensor maps (api.cu): 2-D, row-major, 128-byte swizzled boxes
-enum TmapType : int { TMAP_BF16 = 0, TMAP_F16 = 1, TMAP_F32 = 2 };
+enum TmapType : int { TMAP_BF16 = 0, TMAP_F16 = 1, TMAP_F32 = 2, TMAP_U8 = 3 };
 bool encode_tmap_2d(CUtensorMap* map, TmapType type, const void* base, uint64_t inner, uint64_t outer,
                     uint64_t row_stride_elems, uint32_t box_inner, uint32_t box_outer);
 bool encode_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,

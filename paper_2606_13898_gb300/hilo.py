@@ -20,6 +20,7 @@ import torch
 from . import build as _build
 
 HILO_OK = 0
+HILO_F16 = 2
 HILO_ERR_SHAPE = -2
 HILO_KEEP, HILO_POOL2, HILO_POOL4 = 0, 1, 2
 HILO_BF16, HILO_F32 = 0, 1
@@ -47,13 +48,25 @@ class hilo_block_weights(ctypes.Structure):
     _fields_ = [("txt", hilo_stream_weights), ("img", hilo_stream_weights)]
 
 
+_FP8_FIELDS = ("w_qkv", "w_o", "w_1", "w_2", "s_qkv", "s_o", "s_1", "s_2", "b_qkv", "b_o", "b_1", "b_2")
+
+
+class hilo_stream_weights_fp8(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in _FP8_FIELDS]
+
+
+class hilo_block_weights_fp8(ctypes.Structure):
+    _fields_ = [("txt", hilo_stream_weights_fp8), ("img", hilo_stream_weights_fp8)]
+
+
 EXPORTS = ("hilo_status_string", "hilo_last_error", "hilo_sync_status", "hilo_device_info",
            "hilo_score", "hilo_split_workspace_bytes", "hilo_split", "hilo_pack",
            "hilo_block_workspace_bytes", "hilo_block_forward", "hilo_unpack", "hilo_unpack_update",
            "hilo_convert_bf16_to_f16", "hilo_set_stage_events", "hilo_launch_count",
            "hilo_block_forward_static_ws", "hilo_sobel_workspace_bytes", "hilo_sobel_select",
            "hilo_split_regions", "hilo_unpack_delta", "hilo_row_sizes", "hilo_block_forward_prop",
-           "hilo_row_capacity")
+           "hilo_row_capacity", "hilo_quantize_rows_e4m3", "hilo_block_fp8_workspace_bytes",
+           "hilo_block_forward_fp8")
 
 _lib = None
 
@@ -99,6 +112,10 @@ def lib() -> ctypes.CDLL:
         "hilo_unpack_delta": (I, [shp, P, P, P, spo, P, P]),
         "hilo_row_sizes": (I, [shp, spo, P, ctypes.c_int32, P]),
         "hilo_row_capacity": (S, [shp]),
+        "hilo_quantize_rows_e4m3": (I, [P, I, ctypes.c_int64, ctypes.c_int32, P, P, P]),
+        "hilo_block_fp8_workspace_bytes": (S, [shp, ctypes.c_int32]),
+        "hilo_block_forward_fp8": (I, [shp, ctypes.POINTER(hilo_block_weights_fp8), P, ctypes.c_int32, P, P, I,
+                                       P, P, S, P]),
         "hilo_block_forward_prop": (I, [shp, ctypes.POINTER(hilo_block_weights), P, ctypes.c_int32, P, P, I,
                                         P, P, P, S, P]),
     }
@@ -220,6 +237,39 @@ class DeviceWeights:
         return hilo_block_weights(sw("txt"), sw("img"))
 
 
+@dataclasses.dataclass
+class DeviceWeightsFP8:
+    """One block's weights for hilo_block_forward_fp8: every matrix as e4m3
+    codes with one fp32 scale per output channel, quantised on the device
+    from the bf16 values (hilo_quantize_rows_e4m3); biases bf16."""
+
+    tensors: dict
+
+    @staticmethod
+    def from_host(w, device="cuda") -> "DeviceWeightsFP8":
+        t = {}
+        for sname in ("txt", "img"):
+            sw = getattr(w, sname)
+            for m in ("qkv", "o", "1", "2"):
+                v, b = getattr(sw, "w_" + m), getattr(sw, "b_" + m)
+                if v is None:
+                    t[(sname, "w_" + m)] = t[(sname, "s_" + m)] = t[(sname, "b_" + m)] = None
+                    continue
+                src = bf16_from_bits(v, device)
+                q = torch.empty(src.shape, dtype=torch.uint8, device=device)
+                sc = torch.empty(src.shape[0], dtype=torch.float32, device=device)
+                hilo_quantize_rows_e4m3(src, HILO_BF16, src.shape[0], src.shape[1], q, sc)
+                t[(sname, "w_" + m)], t[(sname, "s_" + m)] = q, sc
+                t[(sname, "b_" + m)] = bf16_from_bits(b, device)
+        torch.cuda.synchronize()
+        return DeviceWeightsFP8(t)
+
+    def c(self) -> hilo_block_weights_fp8:
+        def sw(s):
+            return hilo_stream_weights_fp8(*(_ptr(self.tensors[(s, f)]) for f in _FP8_FIELDS))
+        return hilo_block_weights_fp8(sw("txt"), sw("img"))
+
+
 # ---------------------------------------------------------------------------
 # The C entry points
 # ---------------------------------------------------------------------------
@@ -313,6 +363,25 @@ def hilo_block_forward_prop(shape: Shape, weights: DeviceWeights, cu_img, cap: i
         _ptr(out), _ptr(ws), ws_bytes, _stream(stream)))
 
 
+def hilo_quantize_rows_e4m3(src, src_dtype: int, rows: int, cols: int, dst, scale, stream=None) -> None:
+    _check("hilo_quantize_rows_e4m3", lib().hilo_quantize_rows_e4m3(_ptr(src), src_dtype, rows, cols, _ptr(dst),
+                                                                    _ptr(scale), _stream(stream)))
+
+
+def hilo_block_fp8_workspace_bytes(shape: Shape, cap: int) -> int:
+    s = shape.c()
+    return int(lib().hilo_block_fp8_workspace_bytes(ctypes.byref(s), cap))
+
+
+def hilo_block_forward_fp8(shape: Shape, weights: DeviceWeightsFP8, cu_img, cap: int, in_txt, in_img,
+                           in_dtype: int, out, ws, ws_bytes: int, stream=None) -> None:
+    s = shape.c()
+    w = weights.c()
+    _check("hilo_block_forward_fp8", lib().hilo_block_forward_fp8(
+        ctypes.byref(s), ctypes.byref(w), _ptr(cu_img), cap, _ptr(in_txt), _ptr(in_img), in_dtype, _ptr(out),
+        _ptr(ws), ws_bytes, _stream(stream)))
+
+
 def hilo_row_sizes(shape: Shape, split: SplitBuffers, n_img, cap: int, stream=None) -> None:
     s = shape.c()
     o = split.c()
@@ -392,18 +461,29 @@ class HotPath:
         self.n_img = torch.empty(self.cap, dtype=torch.float32, device=device)
         self.ws_bytes = hilo_block_workspace_bytes(shape, self.cap)
         self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=device)
+        self.weights_fp8 = None
+
+    def enable_fp8(self, weights_fp8: list) -> None:
+        """Makes run(..., fp8=True) available: one DeviceWeightsFP8 per block
+        and the FP8 workspace (which the bf16 blocks' workspace is grown to)."""
+        self.weights_fp8 = weights_fp8
+        need = hilo_block_fp8_workspace_bytes(self.shape, self.cap)
+        if need > self.ws_bytes:
+            self.ws_bytes = need
+            self.ws = torch.empty(need, dtype=torch.uint8, device=self.ws.device)
 
     @property
     def out_img(self) -> torch.Tensor:
         return self.out[self.shape.B * self.shape.T:]
 
     def run(self, x, text, mask, k_keep, k_mid, stream=None, unpack: bool = True, regions: bool = False,
-            prop: bool = False) -> None:
+            prop: bool = False, fp8: bool = False) -> None:
         """One pass. regions=True takes the window-granular split and the
         delta unpool instead of the token-granular split and the nearest
         unpool; prop=True weights each packed row's attention by its row size
         (proportional attention). A shape with lf > 0 runs the separate
-        low-frequency token set (with the delta unpool)."""
+        low-frequency token set (with the delta unpool). fp8=True runs the
+        blocks with e4m3 GEMM operands (enable_fp8 first)."""
         sh = self.shape
         hilo_score(sh, x, self.score, stream)
         (hilo_split_regions if regions else hilo_split)(sh, self.score, mask, k_keep, k_mid, self.split, None, 0,
@@ -411,7 +491,12 @@ class HotPath:
         hilo_pack(sh, x, self.split, self.packed, self.cap, stream)
         if prop:
             hilo_row_sizes(sh, self.split, self.n_img, self.cap, stream)
-        self.blocks(text, self.packed, HILO_BF16, stream, self.n_img if prop else None)
+        if fp8:
+            if prop:
+                raise ValueError("proportional attention has no FP8 block")
+            self.blocks_fp8(text, self.packed, HILO_BF16, stream)
+        else:
+            self.blocks(text, self.packed, HILO_BF16, stream, self.n_img if prop else None)
         if unpack:
             # pooled or low-frequency tokens keep their own detail in the
             # window-granular and low-frequency modes (delta unpool)
@@ -419,6 +504,13 @@ class HotPath:
                 hilo_unpack_delta(sh, self.out_img, self.packed, x, self.split, self.y, stream)
             else:
                 hilo_unpack(sh, self.out_img, self.split, self.y, stream)
+
+    def blocks_fp8(self, in_txt, in_img, in_dtype, stream=None) -> None:
+        sh = self.shape
+        for i, w in enumerate(self.weights_fp8):
+            args = (in_txt, in_img, in_dtype) if i == 0 else (self.out, self.out_img, HILO_F32)
+            hilo_block_forward_fp8(sh, w, self.split.cu_img, self.cap, *args, self.out, self.ws, self.ws_bytes,
+                                   stream)
 
     def blocks(self, in_txt, in_img, in_dtype, stream=None, n_img=None) -> None:
         sh = self.shape
