@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--impl", choices=["hilo", "reference"], default="hilo")
     ap.add_argument("--ratio", default="1/4", help="keep ratio of the timed workload")
     ap.add_argument("--no-extras", action="store_true", help="skip sweep / dense / e2e / cpu_baseline")
+    ap.add_argument("--variant", choices=["bf16", "fp8"], default="bf16",
+                    help="fp8: the timed step's blocks take e4m3 GEMM operands (no extras)")
     return ap.parse_args()
 
 
@@ -130,13 +132,13 @@ def source_sha(files) -> str:
     return h.hexdigest()[:16]
 
 
-def gemm_traffic_per_launch():
+def gemm_traffic_per_launch(key: str = "gemm2_kernel"):
     """DRAM bytes per GEMM launch from the committed ncu summary, if still current."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as fh:
             t = json.load(fh)
-        g = t["gemm2_kernel"]
+        g = t[key]
         if g["source_sha"] != source_sha(g["sources"]):
             return None
         return float(g["bytes_per_launch_mean"])
@@ -625,6 +627,9 @@ def run_hilo(args):
     dw = H.DeviceWeights.from_host(w)
     sh = H.Shape(B=wl.B, H=wl.H, W=wl.W, d=wl.d, T=wl.T, heads=wl.heads, mlp=int(wl.mlp), levels=wl.levels)
     hp = H.HotPath(sh, [dw])
+    fp8 = args.variant == "fp8"
+    if fp8:
+        hp.enable_fp8([H.DeviceWeightsFP8.from_host(w)])
 
     def dev_inputs(b):
         return (H.bf16_from_bits(b.x), H.bf16_from_bits(b.text), torch.from_numpy(b.mask).cuda(),
@@ -632,7 +637,7 @@ def run_hilo(args):
 
     x, text, mask, kk, km = dev_inputs(batch)
     for _ in range(max(3, args.warmup)):
-        hp.run(x, text, mask, kk, km)
+        hp.run(x, text, mask, kk, km, fp8=fp8)
     H.hilo_sync_status()
     cu = hp.split.cu_img.cpu().numpy()
     L = int(cu[-1])
@@ -660,7 +665,7 @@ def run_hilo(args):
     for i in range(K):
         e = ev.get(i)
         if e is None:
-            hp.run(x, text, mask, kk, km)
+            hp.run(x, text, mask, kk, km, fp8=fp8)
             continue
         H.hilo_set_stage_events(e[3:11])
         e[0].record(stream)
@@ -669,7 +674,10 @@ def run_hilo(args):
         H.hilo_split(sh, hp.score, mask, kk, km, hp.split)
         e[2].record(stream)
         H.hilo_pack(sh, x, hp.split, hp.packed, hp.cap)
-        hp.blocks(text, hp.packed, H.HILO_BF16)
+        if fp8:
+            hp.blocks_fp8(text, hp.packed, H.HILO_BF16)
+        else:
+            hp.blocks(text, hp.packed, H.HILO_BF16)
         e[11].record(stream)
         H.hilo_unpack(sh, hp.out_img, hp.split, hp.y)
         e[12].record(stream)
@@ -716,7 +724,8 @@ def run_hilo(args):
         "split": {"ms": t_split},
         "pack": {"ms": t_pack, "GB/s": bw(bytes_pack, t_pack), "frac_hbm": bw(bytes_pack, t_pack) / hbm_peak},
         "layernorm": {"ms": t_ln1 + t_ln2},
-        "gemm": {"ms": gemm_ms, "TFLOP/s": gemm_tflops, "frac_bf16": gemm_tflops / bf16_peak,
+        "gemm": {"ms": gemm_ms, "TFLOP/s": gemm_tflops,
+                 ("frac_fp8" if fp8 else "frac_bf16"): gemm_tflops / (2 * bf16_peak if fp8 else bf16_peak),
                  "qkv_ms": t_qkv, "o_ms": t_o, "mlp1_ms": t_mlp1, "mlp2_ms": t_mlp2},
         "attention": {"ms": t_attn, "TFLOP/s": attn_tflops, "frac_bf16": attn_tflops / bf16_peak},
         "unpack": {"ms": t_unpack, "GB/s": bw(bytes_unpack, t_unpack),
@@ -724,26 +733,32 @@ def run_hilo(args):
     }
     block_tflops = (gemm_flops + attn_flops) / (t_block * 1e-3) / 1e12
     value = N * K * world / (ms_total * 1e-3)
-    traffic = gemm_traffic_per_launch()
+    traffic = gemm_traffic_per_launch("gemm2_kernel_fp8" if fp8 else "gemm2_kernel")
+    # the GEMMs' peak: measured bf16, or twice it for e4m3 operands (the
+    # nominal fp8 : bf16 ratio); in the fp8 step the MLP1 stage includes the
+    # hidden rows' quantisation pass
+    gemm_peak = 2 * bf16_peak if fp8 else bf16_peak
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
         "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": wl.name, "B": wl.B, "H": wl.H, "W": wl.W, "T": wl.T, "d": wl.d,
+        "dtype": "fp8-e4m3 GEMM operands, bf16 attention" if fp8 else "bf16", "data": "synthetic",
+        "config": {"workload": wl.name + ("_fp8" if fp8 else ""), "B": wl.B, "H": wl.H, "W": wl.W, "T": wl.T, "d": wl.d,
                    "heads": wl.heads, "mlp": "4x GELU", "keep_ratio": args.ratio, "mask": "rect 10-40%",
                    "packed_image_rows": L, "block_rows": M, "parallelism": f"replicas x{world}",
-                   "l2": "no flush: per-step working set 0.53 GB (bf16 weights 453 MB) > 129 MB L2"},
+                   "l2": "no flush: per-step working set > 129 MB L2 (weights: 453 MB bf16, 227 MB e4m3)"},
         "block_ms": t_block, "block_tflops": block_tflops,
-        "roofline": {"bound": "tensor", "kernel": "gemm2_kernel (tcgen05 cta_group::2)", "achieved": gemm_tflops,
-                     "peak": bf16_peak, "unit": "TFLOP/s", "frac": gemm_tflops / bf16_peak,
-                     "traffic": traffic, "peak_source": f"{peak_src} bf16 dense (burst)",
+        "roofline": {"bound": "tensor", "kernel": "gemm2_kernel (tcgen05 cta_group::2" +
+                     (", kind::f8f6f4)" if fp8 else ")"), "achieved": gemm_tflops,
+                     "peak": gemm_peak, "unit": "TFLOP/s", "frac": gemm_tflops / gemm_peak,
+                     "traffic": traffic, "peak_source": f"{peak_src} bf16 dense (burst)" +
+                     (" x 2 (nominal fp8 : bf16)" if fp8 else ""),
                      "algorithmic": f"24*M*d^2 FLOP per step over 4 launches, M={M} rows",
                      "timed_launches": f"events on every {INSTR}th step of the timed region ({len(inst)} steps)"},
         "kernels": kernels,
         "gpu_launches": int(launches),
         "clocks": clk,
     }
-    if not args.no_extras:
+    if not args.no_extras and not fp8:
         extras = {}
         # keep-ratio sweep and the dense uncompressed block on the same kernels
         Ks = max(5, min(K, 200))
