@@ -508,29 +508,29 @@ E4M3_MAX = 448.0
 def e4m3_encode(t: np.ndarray) -> np.ndarray:
     """fp32 values -> e4m3 codes (uint8): 1 sign bit, 4 exponent bits (bias
     7), 3 mantissa bits; round to nearest, ties to even; values beyond the
-    largest finite magnitude 448 saturate to +-448 (NaN is not expected)."""
-    t = np.asarray(t, dtype=np.float32).astype(np.float64)
-    sign = (np.signbit(t)).astype(np.uint8) << 7
+    largest finite magnitude 448 saturate to +-448 (NaN is not expected).
+
+    Worked on the fp32 bit pattern. A magnitude at or above 2^-6 (the
+    smallest normal e4m3) keeps 3 of its 23 mantissa bits: add 2^19 - 1 plus
+    the lowest kept bit (round half to even) and clear the 20 dropped bits; a
+    carry into the exponent is the next binade's value, as it should be.
+    Below 2^-6 the values are multiples of the subnormal quantum 2^-9,
+    rounded half to even by rint."""
+    t = np.asarray(t, dtype=np.float32)
+    sign = ((t.view(np.uint32) >> 24) & 0x80).astype(np.uint8)
     a = np.abs(t)
-    # quantum of the binade holding a: 2^(e-3) for e >= -6, 2^-9 below
-    # (subnormals); frexp gives a = m 2^x with m in [0.5, 1)
-    _, x = np.frexp(np.where(a > 0, a, 1.0))
-    e = np.maximum(x - 1, -6)
-    q = np.ldexp(1.0, e - 3)
-    m = a / q                       # exact: q is a power of two
-    r = np.floor(m)
-    frac = m - r
-    up = (frac > 0.5) | ((frac == 0.5) & (np.mod(r, 2) == 1))
-    v = (r + up) * q                # rounded magnitude (may step to the next binade)
-    v = np.minimum(v, E4M3_MAX)
-    # bits of the rounded magnitude
-    _, xv = np.frexp(np.where(v > 0, v, 1.0))
-    ev = xv - 1
-    sub = v < 2.0 ** -6
-    exp_field = np.where(sub, 0, ev + 7)
-    mant = np.where(sub, v / 2.0 ** -9, v / np.ldexp(1.0, ev) * 8 - 8)
-    code = (exp_field.astype(np.int64) << 3) | mant.astype(np.int64)
-    return (sign | code.astype(np.uint8)).astype(np.uint8)
+    bits = a.view(np.uint32)  # sign cleared: adding < 2^20 cannot overflow
+    rb = (bits + np.uint32(0x7FFFF) + ((bits >> 20) & np.uint32(1))) & np.uint32(0xFFF00000)
+    vn = rb.view(np.float32)
+    vs = (np.rint(a * np.float32(2.0 ** 9)) * np.float32(2.0 ** -9)).astype(np.float32)
+    normal = a >= np.float32(2.0 ** -6)
+    v = np.minimum(np.where(normal, vn, vs), np.float32(E4M3_MAX))
+    # fields of the rounded magnitude
+    vb = v.view(np.uint32)
+    vnorm = v >= np.float32(2.0 ** -6)
+    exp_field = np.where(vnorm, ((vb >> 23) & 0xFF).astype(np.int32) - 120, 0)
+    mant = np.where(vnorm, (vb >> 20) & 7, (v * np.float32(2.0 ** 9)).astype(np.int32)).astype(np.int32)
+    return sign | ((exp_field << 3) | mant).astype(np.uint8)
 
 
 def e4m3_decode(c: np.ndarray) -> np.ndarray:
@@ -623,6 +623,50 @@ def block_fp8(u_txt, u_img, cu_img, T: int, weights_q, heads: int, mlp: bool):
             u = u + q_gemm(hid, w.w_2, w.b_2)
         out.append(u)
     return out[0], out[1]
+
+
+def block_rows_fp8(u_txt, u_img, cu_img, T: int, weights_q, heads: int, mlp: bool, b: int, txt_rows,
+                   img_rows):
+    """block_fp8's outputs for selected rows of image ``b`` only: keys and
+    values of the whole joint sequence of image b (each row's quantisation
+    depends on that row alone), queries, attention, out-projection and MLP
+    for the given rows (absolute row ids in u_txt / u_img). fp64 (txt, img)."""
+    ut = _as_f64(u_txt)
+    ui = _as_f64(u_img)
+    d = ut.shape[1] if ut.size else ui.shape[1]
+    hd = d // heads
+    t0, t1 = b * T, (b + 1) * T
+    i0, i1 = int(cu_img[b]), int(cu_img[b + 1])
+    wt, wi = weights_q.txt, weights_q.img
+
+    def rows_of(wq, lo, hi):
+        return (wq[0][lo:hi], wq[1][lo:hi])
+
+    def qkv_part(u, w, lo, hi):
+        # columns [lo, hi) of the QKV output, rounded to bf16 as the kernels store it
+        r = gemm_e4m3(layer_norm(u), rows_of(w.w_qkv, lo, hi), np.asarray(w.b_qkv)[lo:hi])
+        return bf16_to_f32(f32_to_bf16(r)).astype(np.float64)
+
+    kv = np.concatenate([qkv_part(ut[t0:t1], wt, d, 3 * d) if t1 > t0 else np.zeros((0, 2 * d)),
+                         qkv_part(ui[i0:i1], wi, d, 3 * d) if i1 > i0 else np.zeros((0, 2 * d))], axis=0)
+    res = []
+    for rows, u_all, w in ((np.asarray(txt_rows, int), ut, wt), (np.asarray(img_rows, int), ui, wi)):
+        if rows.size == 0:
+            res.append(np.zeros((0, d)))
+            continue
+        u = u_all[rows]
+        q = qkv_part(u, w, 0, d)
+        o = np.empty((len(rows), d))
+        for h in range(heads):
+            c = slice(h * hd, (h + 1) * hd)
+            o[:, c] = softmax_attention(q[:, c], kv[:, :d][:, c], kv[:, d:][:, c])
+        a16 = bf16_to_f32(f32_to_bf16(o)).astype(np.float64)
+        u = u + gemm_e4m3(a16, w.w_o, w.b_o)
+        if mlp:
+            hid = f32_to_f16_sat(gelu_tanh(gemm_e4m3(layer_norm(u), w.w_1, w.b_1)))
+            u = u + gemm_e4m3(hid, w.w_2, w.b_2)
+        res.append(u)
+    return res[0], res[1]
 
 
 @dataclasses.dataclass

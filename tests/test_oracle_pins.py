@@ -790,6 +790,27 @@ def test_block_fp8_error_follows_the_e4m3_model():
     assert qt0.shape == qt.shape
 
 
+def test_block_rows_fp8_matches_block_fp8():
+    rng = np.random.default_rng(12)
+    d, heads, T = 128, 2, 6
+    std = 1 / np.sqrt(d)
+
+    def one():
+        s = I.StreamWeights(w_qkv=bits(rng.normal(0, std, (3 * d, d))), b_qkv=bits(rng.normal(0, std, 3 * d)),
+                            w_o=bits(rng.normal(0, std, (d, d))), b_o=bits(rng.normal(0, std, d)))
+        s.w_1, s.b_1 = bits(rng.normal(0, std, (4 * d, d))), bits(rng.normal(0, std, 4 * d))
+        s.w_2, s.b_2 = bits(rng.normal(0, std / 2, (d, 4 * d))), bits(rng.normal(0, std, d))
+        return s
+    wq = O.quantize_weights(I.BlockWeights(txt=one(), img=one()))
+    ut = bits(rng.standard_normal((2 * T, d)))
+    ui = bits(rng.standard_normal((23, d)))
+    cu = [0, 9, 23]
+    ft, fi = O.block_fp8(ut, ui, cu, T, wq, heads, True)
+    rt, ri = O.block_rows_fp8(ut, ui, cu, T, wq, heads, True, 1, [6, 11], [9, 15, 22])
+    assert np.allclose(rt, ft[[6, 11]], rtol=0, atol=1e-12)
+    assert np.allclose(ri, fi[[9, 15, 22]], rtol=0, atol=1e-12)
+
+
 def test_keep_ratio_one_is_dense_block():
     wl = I.tiny_layer(keep_ratio=1024, H=16, W=16, d=64, heads=2, T=8)
     b = I.make_batch(wl)
