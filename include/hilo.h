@@ -296,6 +296,7 @@ size_t hilo_block_workspace_bytes(const hilo_shape* shape, int32_t cap);
  *   out      fp32 [B*T + cap, d]: the residual stream after the block, text
  *            rows first (row space). With in_dtype == HILO_F32, in-place use
  *            (in_txt == out, in_img == out + B*T*d) is allowed.
+ * in_txt, in_img and out must be 16-byte aligned (HILO_ERR_ARG otherwise).
  * QKV / out-projection GEMM operands and attention inputs are bf16, the MLP
  * GEMM operands fp16 (saturating conversion), all with fp32 accumulation; the
  * residual stream stays fp32.

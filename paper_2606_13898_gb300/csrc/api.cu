@@ -360,6 +360,9 @@ static int block_forward_impl(const hilo_shape* shape, const hilo_block_weights*
   if (st) return st;
   if (!w || !cu_img || !in_img || !out) return fail(HILO_ERR_ARG, "hilo_block_forward: NULL pointer");
   if (shape->T > 0 && !in_txt) return fail(HILO_ERR_ARG, "hilo_block_forward: in_txt is NULL with T>0");
+  if ((reinterpret_cast<uintptr_t>(in_txt) | reinterpret_cast<uintptr_t>(in_img) |
+       reinterpret_cast<uintptr_t>(out)) & 15)
+    return fail(HILO_ERR_ARG, "hilo_block_forward: in_txt, in_img and out must be 16-byte aligned");
   if (in_dtype != HILO_BF16 && in_dtype != HILO_F32)
     return fail(HILO_ERR_ARG, "hilo_block_forward: in_dtype=%d", in_dtype);
   if (cap < 0) return fail(HILO_ERR_ARG, "hilo_block_forward: cap=%d", cap);
@@ -512,6 +515,9 @@ int hilo_block_forward_fp8(const hilo_shape* shape, const hilo_block_weights_fp8
                 shape->d);
   if (!w || !cu_img || !in_img || !out) return fail(HILO_ERR_ARG, "hilo_block_forward_fp8: NULL pointer");
   if (shape->T > 0 && !in_txt) return fail(HILO_ERR_ARG, "hilo_block_forward_fp8: in_txt is NULL with T>0");
+  if ((reinterpret_cast<uintptr_t>(in_txt) | reinterpret_cast<uintptr_t>(in_img) |
+       reinterpret_cast<uintptr_t>(out)) & 15)
+    return fail(HILO_ERR_ARG, "hilo_block_forward_fp8: in_txt, in_img and out must be 16-byte aligned");
   if (in_dtype != HILO_BF16 && in_dtype != HILO_F32)
     return fail(HILO_ERR_ARG, "hilo_block_forward_fp8: in_dtype=%d", in_dtype);
   if (cap < 0) return fail(HILO_ERR_ARG, "hilo_block_forward_fp8: cap=%d", cap);

@@ -339,13 +339,23 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
                                               min(32, max(0, tl.rows - (tl.m0 - tl.row_base) -
                                                                  (128 * static_cast<int>(rank) + q * 32))),
                                               tl.n0, p.N);
+      const int off = 128 * static_cast<int>(rank) + q * 32;  // slab offset in the pair tile
+      const int nvalid = min(32, max(0, tl.rows - (tl.m0 - tl.row_base) - off));
+      if (p.epilogue == EPI_BIAS_RESIDIN_F32 && lane < nvalid && tl.n0 < p.N) {
+        // this lane's residual row into L2 while the accumulator is still
+        // being computed, so that the epilogue's chunk loads do not each
+        // wait for DRAM
+        const int esz = p.resid_f32 ? 4 : 2;
+        const char* r = static_cast<const char*>(tl.g ? p.resid_src[1] : p.resid_src[0]) +
+                        (static_cast<long long>(tl.m0 + off + lane - tl.row_base) * p.N + tl.n0) * esz;
+        for (int j = 0; j < PN * esz / 128; ++j) prefetch_l2(r + 128 * j);
+      }
       if (!mbar_wait_warp(&tfull[acc], acc_phase, abort_flag, err, DEV_TIMEOUT_GEMM + 256 * 5)) break;
       tc_fence_after();
-      const int off = 128 * static_cast<int>(rank) + q * 32;  // slab offset in the pair tile
       EpiSlab sl;
       sl.g = tl.g;
       sl.row0 = tl.m0 + off;
-      sl.nvalid = min(32, max(0, tl.rows - (tl.m0 - tl.row_base) - off));
+      sl.nvalid = nvalid;
       sl.row_base = tl.row_base;
       sl.n0 = tl.n0;
       const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * PN);

@@ -148,8 +148,13 @@ def test_workspace_size_and_check(H):
         sw = getattr(w, f)
         for n in ("w_qkv", "b_qkv", "w_o", "b_o", "w_1", "b_1", "w_2", "b_2"):
             setattr(sw, n, 1)
-    rc = H.lib().hilo_block_forward(ctypes.byref(s), ctypes.byref(w), 1, cap, 1, 1, 0, 1, 1, nb - 1, None)
+    rc = H.lib().hilo_block_forward(ctypes.byref(s), ctypes.byref(w), 1, cap, 256, 256, 0, 256, 1, nb - 1, None)
     assert rc == -4
+    # the rows are read with 16-byte copies: unaligned row buffers are refused
+    for args in ((264, 256, 256), (256, 260, 256), (256, 256, 258)):
+        rc = H.lib().hilo_block_forward(ctypes.byref(s), ctypes.byref(w), 1, cap, *args[:2], 0, args[2], 1, nb, None)
+        assert rc == -1
+        assert b"16-byte aligned" in H.lib().hilo_last_error()
 
 
 @pytest.mark.parametrize("channels,patch,radius,thr,code", [
