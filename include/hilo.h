@@ -172,6 +172,18 @@ const char* hilo_last_error(void);
  */
 int hilo_sync_status(void* stream);
 
+/*
+ * hilo_debug_wait_timeout -- test hook for the device-side failure path.
+ * Launches one CTA whose thread 0 waits, with the same bounded mbarrier wait
+ * the tcgen05 kernels use (1 s limit on %globaltimer), on an mbarrier that
+ * nothing arrives at. The wait runs out, latches its code in the probe's
+ * device word and the kernel returns: nothing faults, traps or hangs. The
+ * next hilo_sync_status(stream) returns HILO_ERR_TIMEOUT ("probe=3" in
+ * hilo_last_error) and clears the word; the context stays usable.
+ * Returns HILO_OK once launched, HILO_ERR_CUDA if the launch failed.
+ */
+int hilo_debug_wait_timeout(void* stream);
+
 /* Number of SMs of the current device and whether it is sm_103 (1/0). */
 int hilo_device_info(int* num_sms, int* is_sm103);
 

@@ -233,12 +233,18 @@ int hilo_sync_status(void* stream) {
   const int g = hilo::gemm_take_device_error();
   const int g2 = hilo::gemm2_take_device_error();
   const int a = hilo::attn_take_device_error();
-  if (g < 0 || g2 < 0 || a < 0)
+  const int pr = hilo::probe_take_device_error();
+  if (g < 0 || g2 < 0 || a < 0 || pr < 0)
     return fail(HILO_ERR_CUDA, "hilo_sync_status: reading the device error word failed");
-  if (g || g2 || a)
-    return fail(HILO_ERR_TIMEOUT, "device-side wait ran out (gemm=%d, gemm pair=%d, attention=%d)", g, g2,
-                a);
+  if (g || g2 || a || pr)
+    return fail(HILO_ERR_TIMEOUT, "device-side wait ran out (gemm=%d, gemm pair=%d, attention=%d, probe=%d)", g,
+                g2, a, pr);
   return HILO_OK;
+}
+
+int hilo_debug_wait_timeout(void* stream) {
+  const cudaError_t e = hilo::launch_wait_probe(static_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_debug_wait_timeout");
 }
 
 int hilo_score(const hilo_shape* shape, const void* x, float* score, void* stream) {

@@ -1237,4 +1237,34 @@ cudaError_t launch_layernorm(const void* in_txt, const void* in_img, int in_f32,
   }
 }
 
+// ================================================== wait-timeout probe =====
+// One thread waits on an mbarrier that nothing arrives at, with the bounded
+// wait of the tcgen05 kernels; when the limit passes, the wait latches
+// DEV_TIMEOUT_PROBE in g_probe_err and the kernel returns.
+
+__device__ int g_probe_err;
+
+__global__ void wait_probe_kernel() {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);
+  abort_flag = 0;
+  fence_mbar_init();
+  mbar_wait(&bar, 0, &abort_flag, &g_probe_err, DEV_TIMEOUT_PROBE);
+}
+
+cudaError_t launch_wait_probe(cudaStream_t st) {
+  wait_probe_kernel<<<1, 32, 0, st>>>();
+  return cudaGetLastError();
+}
+
+int probe_take_device_error() {
+  int v = 0;
+  const int z = 0;
+  if (cudaMemcpyFromSymbol(&v, g_probe_err, sizeof(int)) != cudaSuccess) return -1;
+  if (v) cudaMemcpyToSymbol(g_probe_err, &z, sizeof(int));
+  return v;
+}
+
 }  // namespace hilo

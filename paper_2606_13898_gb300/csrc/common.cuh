@@ -19,6 +19,7 @@ enum : int {
   DEV_OK = 0,
   DEV_TIMEOUT_GEMM = 1,
   DEV_TIMEOUT_ATTN = 2,
+  DEV_TIMEOUT_PROBE = 3,
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {

@@ -106,6 +106,10 @@ struct AttnArgs {
 };
 cudaError_t launch_attention(const AttnArgs& a, int num_sms, cudaStream_t st);
 int attn_take_device_error();
+// The wait-timeout probe: one bounded mbarrier wait that runs out; its code
+// is read (and cleared) like the kernels' device error words.
+cudaError_t launch_wait_probe(cudaStream_t st);
+int probe_take_device_error();
 
 // ---- error text of the calling thread (api.cu)
 int set_error(int status, const char* msg);

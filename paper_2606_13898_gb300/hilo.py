@@ -66,7 +66,7 @@ EXPORTS = ("hilo_status_string", "hilo_last_error", "hilo_sync_status", "hilo_de
            "hilo_block_forward_static_ws", "hilo_sobel_workspace_bytes", "hilo_sobel_select",
            "hilo_split_regions", "hilo_unpack_delta", "hilo_row_sizes", "hilo_block_forward_prop",
            "hilo_row_capacity", "hilo_quantize_rows_e4m3", "hilo_block_fp8_workspace_bytes",
-           "hilo_block_forward_fp8")
+           "hilo_block_forward_fp8", "hilo_debug_wait_timeout")
 
 _lib = None
 
@@ -91,6 +91,7 @@ def lib() -> ctypes.CDLL:
         "hilo_status_string": (ctypes.c_char_p, [I]),
         "hilo_last_error": (ctypes.c_char_p, []),
         "hilo_sync_status": (I, [P]),
+        "hilo_debug_wait_timeout": (I, [P]),
         "hilo_device_info": (I, [ctypes.POINTER(I), ctypes.POINTER(I)]),
         "hilo_score": (I, [shp, P, P, P]),
         "hilo_split_workspace_bytes": (S, [shp]),
@@ -283,6 +284,11 @@ def hilo_device_info() -> tuple[int, int]:
 
 def hilo_sync_status(stream=None) -> None:
     _check("hilo_sync_status", lib().hilo_sync_status(_stream(stream)))
+
+
+def hilo_debug_wait_timeout(stream=None) -> None:
+    """Launch the wait-timeout probe; the next hilo_sync_status raises HILO_ERR_TIMEOUT."""
+    _check("hilo_debug_wait_timeout", lib().hilo_debug_wait_timeout(_stream(stream)))
 
 
 def hilo_score(shape: Shape, x, score, stream=None) -> None:
