@@ -54,7 +54,8 @@ enum {
   HILO_ERR_CUDA = -3,        /* a CUDA runtime/driver call failed */
   HILO_ERR_WORKSPACE = -4,   /* workspace missing or smaller than required */
   HILO_ERR_TIMEOUT = -5,     /* a device-side bounded wait ran out (see hilo_sync_status) */
-  HILO_ERR_UNSUPPORTED = -6  /* no sm_103a device, or a feature not built */
+  HILO_ERR_UNSUPPORTED = -6, /* no sm_103a device, or a feature not built */
+  HILO_ERR_CHECK = -7        /* a device-side index check failed (checks build only) */
 };
 
 /* Per-token labels written by hilo_split (HILO_LF: a non-kept token of the
@@ -166,9 +167,12 @@ const char* hilo_status_string(int status);
 const char* hilo_last_error(void);
 
 /*
- * Synchronises `stream`, then reads and clears the device error word.
+ * Synchronises `stream`, then reads and clears the device error words.
  * Returns HILO_OK, HILO_ERR_TIMEOUT if a device-side bounded wait ran out
- * since the last call, or HILO_ERR_CUDA if the stream reported an error.
+ * since the last call, HILO_ERR_CHECK if (in the checks build of the
+ * library, compiled with -DHILO_DEVICE_CHECKS) a kernel found an index read
+ * from device data out of range and skipped that access, or HILO_ERR_CUDA
+ * if the stream reported an error.
  */
 int hilo_sync_status(void* stream);
 

@@ -4,6 +4,12 @@ Each CUDA translation unit is compiled in parallel, then linked into
 ``paper_2606_13898_gb300/_build/libhilo.so`` (CUDA runtime linked statically;
 the driver's tensor-map encoder is resolved at run time). A unit is rebuilt when it or a header is newer than its
 object file.
+
+``build(variant="checks")`` links ``_build_checks/libhilo.so``: the translation
+units that hold device-side index checks are compiled with
+``-DHILO_DEVICE_CHECKS`` (a failed check is reported by hilo_sync_status as
+HILO_ERR_CHECK and its access skipped); the others are the release objects.
+Select it at run time with the HILO_LIBRARY environment variable.
 """
 from __future__ import annotations
 
@@ -19,6 +25,9 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libhilo.so")
+BUILD_CHECKS = os.path.join(PKG, "_build_checks")
+LIB_CHECKS = os.path.join(BUILD_CHECKS, "libhilo.so")
+CHECKED = ("bw_kernels.cu",)  # translation units with HILO_DCHECK sites
 SOURCES = ["api.cu", "bw_kernels.cu", "gemm_tc.cu", "gemm2_tc.cu", "attn_tc.cu", "noalloc.cu", "select.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fno-strict-aliasing",
@@ -45,9 +54,15 @@ def _stale(target: str, deps: list[str]) -> bool:
     return any(os.path.getmtime(dep) > t for dep in deps)
 
 
-def build(verbose: bool = False, extra_flags: list[str] | None = None) -> str:
-    """Compile and link libhilo.so; returns its path."""
+def build(verbose: bool = False, extra_flags: list[str] | None = None, variant: str = "release") -> str:
+    """Compile and link libhilo.so (variant "release" or "checks"); returns its path."""
+    if variant not in ("release", "checks"):
+        raise ValueError(f"unknown build variant {variant!r}")
+    checks = variant == "checks"
     os.makedirs(BUILD, exist_ok=True)
+    if checks:
+        os.makedirs(BUILD_CHECKS, exist_ok=True)
+    lib = LIB_CHECKS if checks else LIB
     nvcc = _nvcc()
     headers = _headers()
     flags = FLAGS + list(extra_flags or [])
@@ -55,10 +70,12 @@ def build(verbose: bool = False, extra_flags: list[str] | None = None) -> str:
     objs = []
     for src in SOURCES:
         path = os.path.join(CSRC, src)
-        obj = os.path.join(BUILD, src.replace(".cu", ".o"))
+        checked = checks and src in CHECKED
+        obj = os.path.join(BUILD_CHECKS if checked else BUILD, src.replace(".cu", ".o"))
         objs.append(obj)
         if _stale(obj, [path] + headers):
-            jobs.append([nvcc, *ARCH, *flags, "-c", path, "-o", obj])
+            extra = ["-DHILO_DEVICE_CHECKS"] if checked else []
+            jobs.append([nvcc, *ARCH, *flags, *extra, "-c", path, "-o", obj])
 
     def run(cmd):
         if verbose:
@@ -71,10 +88,10 @@ def build(verbose: bool = False, extra_flags: list[str] | None = None) -> str:
 
     with cf.ThreadPoolExecutor(max_workers=max(1, len(jobs))) as ex:
         list(ex.map(run, jobs))
-    if jobs or _stale(LIB, objs):
-        link = [nvcc, *ARCH, "-shared", "-o", LIB, *objs]
+    if jobs or _stale(lib, objs):
+        link = [nvcc, *ARCH, "-shared", "-o", lib, *objs]
         run(link)
-    return LIB
+    return lib
 
 
 if __name__ == "__main__":

@@ -209,6 +209,7 @@ const char* hilo_status_string(int status) {
     case HILO_ERR_WORKSPACE: return "HILO_ERR_WORKSPACE";
     case HILO_ERR_TIMEOUT: return "HILO_ERR_TIMEOUT";
     case HILO_ERR_UNSUPPORTED: return "HILO_ERR_UNSUPPORTED";
+    case HILO_ERR_CHECK: return "HILO_ERR_CHECK";
     default: return "HILO_ERR_UNKNOWN";
   }
 }
@@ -234,11 +235,13 @@ int hilo_sync_status(void* stream) {
   const int g2 = hilo::gemm2_take_device_error();
   const int a = hilo::attn_take_device_error();
   const int pr = hilo::probe_take_device_error();
-  if (g < 0 || g2 < 0 || a < 0 || pr < 0)
+  const int dc = hilo::dcheck_take_bw();
+  if (g < 0 || g2 < 0 || a < 0 || pr < 0 || dc < 0)
     return fail(HILO_ERR_CUDA, "hilo_sync_status: reading the device error word failed");
   if (g || g2 || a || pr)
     return fail(HILO_ERR_TIMEOUT, "device-side wait ran out (gemm=%d, gemm pair=%d, attention=%d, probe=%d)", g,
                 g2, a, pr);
+  if (dc) return fail(HILO_ERR_CHECK, "device-side index check %d failed (checks build)", dc);
   return HILO_OK;
 }
 
@@ -657,7 +660,8 @@ int hilo_unpack(const hilo_shape* shape, const float* out_img, const hilo_split_
   DevInfo* dev;
   if ((st = current_device(&dev))) return st;
   const long long ntok = static_cast<long long>(shape->B) * shape->H * shape->W;
-  cudaError_t e = hilo::launch_unpack(out_img, split->tok_row, y, ntok, shape->d, dev->num_sms,
+  const long long rows_max = static_cast<long long>(hilo_row_capacity(shape));
+  cudaError_t e = hilo::launch_unpack(out_img, split->tok_row, y, ntok, shape->d, rows_max, dev->num_sms,
                                       static_cast<cudaStream_t>(stream));
   if (e == cudaSuccess) count(1);
   return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_unpack");
@@ -676,7 +680,8 @@ int hilo_unpack_delta(const hilo_shape* shape, const float* out_img, const void*
   if ((st = current_device(&dev))) return st;
   const long long ntok = static_cast<long long>(shape->B) * shape->H * shape->W;
   cudaError_t e = hilo::launch_unpack_delta(out_img, packed, x, split->labels, split->tok_row, y, ntok,
-                                            shape->d, dev->num_sms, static_cast<cudaStream_t>(stream));
+                                            shape->d, static_cast<long long>(hilo_row_capacity(shape)),
+                                            dev->num_sms, static_cast<cudaStream_t>(stream));
   if (e == cudaSuccess) count(1);
   return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_unpack_delta");
 }
@@ -691,7 +696,8 @@ int hilo_unpack_update(const hilo_shape* shape, const float* out_img, const hilo
   if ((st = current_device(&dev))) return st;
   const long long ntok = static_cast<long long>(shape->B) * shape->H * shape->W;
   cudaError_t e = hilo::launch_unpack_update(out_img, split->tok_row, x, ntok, shape->d, alpha,
-                                             dev->num_sms, static_cast<cudaStream_t>(stream));
+                                             static_cast<long long>(hilo_row_capacity(shape)), dev->num_sms,
+                                             static_cast<cudaStream_t>(stream));
   if (e == cudaSuccess) count(1);
   return e == cudaSuccess ? HILO_OK : cuda_fail(e, "hilo_unpack_update");
 }

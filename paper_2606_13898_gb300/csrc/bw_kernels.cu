@@ -658,13 +658,15 @@ __global__ void __launch_bounds__(256) pack_kernel(const __nv_bfloat16* __restri
     const int src = row_src[r];
     const __nv_bfloat16* xb = x + static_cast<long long>(b) * N * d;
     uint4* dst = reinterpret_cast<uint4*>(packed + static_cast<long long>(r) * d);
+    const int size = local < nk ? 1 : local < nk + n2 ? 2 : 4;
+    // the row source: a token of the image, or a window of its size
+    if (!HILO_DCHECK(local >= 0 && src >= 0 && src < (H / size) * (W / size), DCHECK_PACK_SRC)) continue;
     if (local < nk) {
       const uint4* sp = reinterpret_cast<const uint4*>(xb + static_cast<long long>(src) * d);
 #pragma unroll 4
       for (int c = c0; c < G; c += CSTEP) dst[c] = __ldg(sp + c);
       continue;
     }
-    const int size = local < nk + n2 ? 2 : 4;
     const uint8_t cls = size == 2 ? HILO_LABEL_POOL2 : HILO_LABEL_POOL4;
     const int Wn = W / size;
     const int t0 = (size * (src / Wn)) * W + size * (src % Wn);
@@ -745,6 +747,8 @@ __global__ void __launch_bounds__(256) pack_lf_kernel(const __nv_bfloat16* __res
     const int src = row_src[r];
     const __nv_bfloat16* xb = x + static_cast<long long>(b) * N * d;
     uint4* dst = reinterpret_cast<uint4*>(packed + static_cast<long long>(r) * d);
+    const int size = local < counts[3 * b] ? 1 : LF;
+    if (!HILO_DCHECK(local >= 0 && src >= 0 && src < (H / size) * (W / size), DCHECK_PACK_LF_SRC)) continue;
     if (local < counts[3 * b]) {
       const uint4* sp = reinterpret_cast<const uint4*>(xb + static_cast<long long>(src) * d);
 #pragma unroll 4
@@ -782,6 +786,7 @@ __global__ void __launch_bounds__(256) row_sizes_kernel(const uint8_t* __restric
     const uint8_t cls = lf ? HILO_LABEL_LF : (size == 2 ? HILO_LABEL_POOL2 : HILO_LABEL_POOL4);
     const int src = row_src[r];
     const int Wn = W / size;
+    if (!HILO_DCHECK(local >= 0 && src >= 0 && src < (H / size) * Wn, DCHECK_ROW_SIZES_SRC)) continue;
     const uint8_t* lab = labels + static_cast<long long>(b) * N + (size * (src / Wn)) * W + size * (src % Wn);
     int c = 0;
     for (int i = 0; i < size; ++i)
@@ -795,7 +800,7 @@ __global__ void __launch_bounds__(256) row_sizes_kernel(const uint8_t* __restric
 __global__ void __launch_bounds__(256) unpack_kernel(const float* __restrict__ out_img,
                                                      const int32_t* __restrict__ tok_row,
                                                      float* __restrict__ y, long long ntok,
-                                                     int d) {
+                                                     int d, long long rows_max) {
   pdl_trigger();
   pdl_wait();
   const int lane = threadIdx.x & 31;
@@ -803,6 +808,7 @@ __global__ void __launch_bounds__(256) unpack_kernel(const float* __restrict__ o
   for (long long t = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
        t < ntok; t += wstep) {
     const int r = __ldg(tok_row + t);
+    if (!HILO_DCHECK(r >= 0 && r < rows_max, DCHECK_UNPACK_ROW)) continue;
     const float4* s = reinterpret_cast<const float4*>(out_img + static_cast<long long>(r) * d);
     float4* o = reinterpret_cast<float4*>(y + t * d);
     for (int c = lane; c < (d >> 2); c += 32) __stcs(o + c, __ldg(s + c));
@@ -817,7 +823,8 @@ __global__ void __launch_bounds__(256) unpack_delta_kernel(const float* __restri
                                                            const __nv_bfloat16* __restrict__ x,
                                                            const uint8_t* __restrict__ labels,
                                                            const int32_t* __restrict__ tok_row,
-                                                           float* __restrict__ y, long long ntok, int d) {
+                                                           float* __restrict__ y, long long ntok, int d,
+                                                           long long rows_max) {
   pdl_trigger();
   pdl_wait();
   const int lane = threadIdx.x & 31;
@@ -825,6 +832,7 @@ __global__ void __launch_bounds__(256) unpack_delta_kernel(const float* __restri
   for (long long t = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
        t < ntok; t += wstep) {
     const int r = __ldg(tok_row + t);
+    if (!HILO_DCHECK(r >= 0 && r < rows_max, DCHECK_UNPACK_DELTA_ROW)) continue;
     const float4* s = reinterpret_cast<const float4*>(out_img + static_cast<long long>(r) * d);
     float4* o = reinterpret_cast<float4*>(y + t * d);
     if (__ldg(labels + t) == HILO_LABEL_KEEP) {
@@ -851,7 +859,8 @@ __global__ void __launch_bounds__(256) unpack_delta_kernel(const float* __restri
 __global__ void __launch_bounds__(256) unpack_update_kernel(const float* __restrict__ out_img,
                                                             const int32_t* __restrict__ tok_row,
                                                             __nv_bfloat16* __restrict__ x,
-                                                            long long ntok, int d, float alpha) {
+                                                            long long ntok, int d, float alpha,
+                                                            long long rows_max) {
   pdl_trigger();
   pdl_wait();
   const int lane = threadIdx.x & 31;
@@ -859,6 +868,7 @@ __global__ void __launch_bounds__(256) unpack_update_kernel(const float* __restr
   for (long long t = static_cast<long long>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
        t < ntok; t += wstep) {
     const int r = __ldg(tok_row + t);
+    if (!HILO_DCHECK(r >= 0 && r < rows_max, DCHECK_UNPACK_UPDATE_ROW)) continue;
     const float4* s = reinterpret_cast<const float4*>(out_img + static_cast<long long>(r) * d);
     uint4* xr = reinterpret_cast<uint4*>(x + t * d);
     for (int c = lane; c < (d >> 3); c += 32) {
@@ -1168,9 +1178,9 @@ cudaError_t launch_pack(const void* x, const uint8_t* labels, const int32_t* row
 }
 
 cudaError_t launch_unpack(const float* out_img, const int32_t* tok_row, float* y, long long ntok,
-                          int d, int num_sms, cudaStream_t st) {
+                          int d, long long rows_max, int num_sms, cudaStream_t st) {
   return launch_pdl(unpack_kernel, dim3(grid_for(ntok, 8, num_sms, 8)), dim3(256), 0, st, out_img,
-                    tok_row, y, ntok, d);
+                    tok_row, y, ntok, d, rows_max);
 }
 
 cudaError_t launch_row_sizes(const uint8_t* labels, const int32_t* row_src, const int32_t* counts,
@@ -1183,17 +1193,17 @@ cudaError_t launch_row_sizes(const uint8_t* labels, const int32_t* row_src, cons
 
 cudaError_t launch_unpack_delta(const float* out_img, const void* packed, const void* x,
                                 const uint8_t* labels, const int32_t* tok_row, float* y, long long ntok,
-                                int d, int num_sms, cudaStream_t st) {
+                                int d, long long rows_max, int num_sms, cudaStream_t st) {
   return launch_pdl(unpack_delta_kernel, dim3(grid_for(ntok, 8, num_sms, 8)), dim3(256), 0, st, out_img,
                     static_cast<const __nv_bfloat16*>(packed), static_cast<const __nv_bfloat16*>(x), labels,
-                    tok_row, y, ntok, d);
+                    tok_row, y, ntok, d, rows_max);
 }
 
 cudaError_t launch_unpack_update(const float* out_img, const int32_t* tok_row, void* x,
-                                 long long ntok, int d, float alpha, int num_sms,
+                                 long long ntok, int d, float alpha, long long rows_max, int num_sms,
                                  cudaStream_t st) {
   return launch_pdl(unpack_update_kernel, dim3(grid_for(ntok, 8, num_sms, 8)), dim3(256), 0, st,
-                    out_img, tok_row, static_cast<__nv_bfloat16*>(x), ntok, d, alpha);
+                    out_img, tok_row, static_cast<__nv_bfloat16*>(x), ntok, d, alpha, rows_max);
 }
 
 cudaError_t launch_quant_rows(const void* src, int type, int cols, int rows_static, const int32_t* cu_img,
@@ -1265,6 +1275,18 @@ int probe_take_device_error() {
   if (cudaMemcpyFromSymbol(&v, g_probe_err, sizeof(int)) != cudaSuccess) return -1;
   if (v) cudaMemcpyToSymbol(g_probe_err, &z, sizeof(int));
   return v;
+}
+
+int dcheck_take_bw() {
+#ifdef HILO_DEVICE_CHECKS
+  int v = 0;
+  const int z = 0;
+  if (cudaMemcpyFromSymbol(&v, g_dcheck, sizeof(int)) != cudaSuccess) return -1;
+  if (v) cudaMemcpyToSymbol(g_dcheck, &z, sizeof(int));
+  return v;
+#else
+  return 0;
+#endif
 }
 
 }  // namespace hilo

@@ -22,6 +22,28 @@ enum : int {
   DEV_TIMEOUT_PROBE = 3,
 };
 
+// ----------------------------------------------------------- device checks --
+// The checks variant of the library (built with -DHILO_DEVICE_CHECKS) tests
+// every index that a kernel reads from device data (row sources, token rows)
+// before it addresses memory with it. A failed HILO_DCHECK records its code in
+// the translation unit's check word (the first failure wins) and the guarded
+// access is skipped, so nothing traps; hilo_sync_status reads and clears the
+// word. In the normal build every check is the constant true.
+enum : int {
+  DCHECK_PACK_SRC = 1,
+  DCHECK_PACK_LF_SRC = 2,
+  DCHECK_ROW_SIZES_SRC = 3,
+  DCHECK_UNPACK_ROW = 4,
+  DCHECK_UNPACK_DELTA_ROW = 5,
+  DCHECK_UNPACK_UPDATE_ROW = 6,
+};
+#ifdef HILO_DEVICE_CHECKS
+static __device__ int g_dcheck;
+#define HILO_DCHECK(cond, code) ((cond) || (atomicCAS(&::hilo::g_dcheck, 0, (code)), false))
+#else
+#define HILO_DCHECK(cond, code) (true)
+#endif
+
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }

@@ -25,16 +25,18 @@ cudaError_t launch_split(const float* score, const uint8_t* mask, const int32_t*
 cudaError_t launch_pack(const void* x, const uint8_t* labels, const int32_t* row_src,
                         const int32_t* counts, const int32_t* cu_img, void* packed, int B, int H,
                         int W, int d, int cap, int lf, int num_sms, cudaStream_t st);
+// rows_max: rows of out_img (the row capacity); a token row at or past it
+// is an error of the checks build
 cudaError_t launch_unpack(const float* out_img, const int32_t* tok_row, float* y, long long ntok,
-                          int d, int num_sms, cudaStream_t st);
+                          int d, long long rows_max, int num_sms, cudaStream_t st);
 cudaError_t launch_row_sizes(const uint8_t* labels, const int32_t* row_src, const int32_t* counts,
                              const int32_t* cu_img, float* n_img, int B, int H, int W, int cap, int lf,
                              int num_sms, cudaStream_t st);
 cudaError_t launch_unpack_delta(const float* out_img, const void* packed, const void* x,
                                 const uint8_t* labels, const int32_t* tok_row, float* y, long long ntok,
-                                int d, int num_sms, cudaStream_t st);
+                                int d, long long rows_max, int num_sms, cudaStream_t st);
 cudaError_t launch_unpack_update(const float* out_img, const int32_t* tok_row, void* x,
-                                 long long ntok, int d, float alpha, int num_sms,
+                                 long long ntok, int d, float alpha, long long rows_max, int num_sms,
                                  cudaStream_t st);
 cudaError_t launch_layernorm(const void* in_txt, const void* in_img, int in_f32, float* resid,
                              void* ln, int ln_mode, float* ln_scale, const int32_t* cu_img, int B, int n_txt,
@@ -110,6 +112,8 @@ int attn_take_device_error();
 // is read (and cleared) like the kernels' device error words.
 cudaError_t launch_wait_probe(cudaStream_t st);
 int probe_take_device_error();
+// The check word of the bandwidth kernels (checks build; 0 otherwise).
+int dcheck_take_bw();
 
 // ---- error text of the calling thread (api.cu)
 int set_error(int status, const char* msg);

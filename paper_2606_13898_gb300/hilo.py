@@ -22,6 +22,7 @@ from . import build as _build
 HILO_OK = 0
 HILO_F16 = 2
 HILO_ERR_SHAPE = -2
+HILO_ERR_TIMEOUT, HILO_ERR_CHECK = -5, -7
 HILO_KEEP, HILO_POOL2, HILO_POOL4 = 0, 1, 2
 HILO_BF16, HILO_F32 = 0, 1
 
@@ -72,7 +73,8 @@ _lib = None
 
 
 def library_path() -> str:
-    return _build.LIB
+    """The library to load: HILO_LIBRARY if set (e.g. the checks build), else the in-tree build."""
+    return os.environ.get("HILO_LIBRARY") or _build.LIB
 
 
 def lib() -> ctypes.CDLL:
