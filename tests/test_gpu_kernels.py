@@ -193,6 +193,7 @@ def scaled_weights(rng, d, mlp, std):
     (128, 1, 64, [200], 0, 1.0),          # head_dim 128, ragged text and image tiles
     (128, 2, 64, [256, 77], 1, 1.0),      # head_dim 64, two images of different length
     (256, 2, 0, [130, 300, 5], 1, 1.0),   # no text, three images
+    (128, 1, 64, [0, 50], 1, 1.0),        # an image with no image rows: text-only joint sequence
     (512, 8, 200, [384], 1, 1.0),         # several 256-wide GEMM column tiles
     (1024, 8, 256, [4800], 1, 1.0),       # > 76 pair tiles: out-proj / MLP2 tiles split across SM pairs
 ])
