@@ -201,7 +201,8 @@ def cpu_baseline(ratio: str, min_seconds: float = 10.0):
 
 
 def run_reference(args):
-    rank = int(os.environ.get("RANK", "0"))
+    from paper_2606_13898_gb300 import replicas
+    rank, _, _ = replicas.env_rank_world()
     if rank != 0:
         return
     budget = 150.0
@@ -594,9 +595,8 @@ def run_hilo(args):
     from paper_2606_13898_gb300 import hilo as H
     from paper_2606_13898_gb300 import inputs as I
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    from paper_2606_13898_gb300 import replicas
+    rank, world, local = replicas.env_rank_world()
     torch.cuda.set_device(local)
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
@@ -608,18 +608,16 @@ def run_hilo(args):
             dist.barrier()
 
     def max_over_ranks(v: float) -> float:
-        if world == 1:
-            return v
-        t = torch.tensor([v], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+        return replicas.max_over_ranks(v, device="cuda")
 
     hbm_peak, bf16_peak, peak_src = peaks()
     stream = torch.cuda.current_stream()
 
     def setup(ratio: str):
         wl = workload(ratio)
-        b = I.make_batch(wl, seed_offset=17 * rank)
+        # weak scaling: a global batch of world x B images, this rank's slice
+        b0, _ = replicas.image_slice(world * wl.B, rank, world)
+        b = I.make_batch(wl, seed_offset=b0)
         return wl, b
 
     wl, batch = setup(args.ratio)
@@ -732,7 +730,7 @@ def run_hilo(args):
                    "frac_hbm": bw(bytes_unpack, t_unpack) / hbm_peak},
     }
     block_tflops = (gemm_flops + attn_flops) / (t_block * 1e-3) / 1e12
-    value = N * K * world / (ms_total * 1e-3)
+    value = replicas.whole_job_throughput(N * K, world, ms_total)
     traffic = gemm_traffic_per_launch("gemm2_kernel_fp8" if fp8 else "gemm2_kernel")
     # the GEMMs' peak: measured bf16, or twice it for e4m3 operands (the
     # nominal fp8 : bf16 ratio); in the fp8 step the MLP1 stage includes the
