@@ -411,6 +411,69 @@ def time_lf(H, torch, stream, wl, dw, inputs, steps: int, lf: int = 4) -> dict:
             "low_frequency_tokens": int(counts[1]), "packed_image_rows": int(hp.split.cu_img[-1].item())}
 
 
+def time_torch_context(H, torch, stream, wl, hp, dw, inputs, steps: int) -> dict:
+    """Context baseline (not the reference arm): the same compressed block in
+    plain PyTorch on the GPU, cuBLAS GEMMs through F.linear and the joint
+    attention through F.scaled_dot_product_attention, with the dtypes of the
+    tcgen05 path (bf16 QKV / out-projection operands, fp16 MLP operands, fp32
+    residual stream). Timed on the timed workload's packed rows, beside this
+    library's block on the same rows."""
+    import torch.nn.functional as F
+    x, text, mask, kk, km = inputs
+    hp.run(x, text, mask, kk, km)
+    cu = hp.split.cu_img.cpu().numpy()
+    sh, d, heads, T, B = hp.shape, wl.d, wl.heads, wl.T, wl.B
+    hd = d // heads
+    L = int(cu[-1])
+    t = {k: v for k, v in dw.tensors.items()}
+    for s_ in ("txt", "img"):  # MLP biases in the MLP operands' dtype
+        for f in ("b_1", "b_2"):
+            t[(s_, f)] = t[(s_, f)].to(torch.float16)
+    u_txt, u_img = text.view(B * T, d), hp.packed[:L]
+    Rt = B * T
+
+    def two(fn, a):
+        return torch.cat([fn(a[:Rt], "txt"), fn(a[Rt:], "img")])
+
+    def block():
+        u = torch.cat([u_txt.float(), u_img.float()])
+        h = F.layer_norm(u, (d,), eps=1e-6).to(torch.bfloat16)
+        qkv = two(lambda a, s_: F.linear(a, t[(s_, "w_qkv")], t[(s_, "b_qkv")]), h)
+        o = torch.empty(u.shape[0], d, dtype=torch.bfloat16, device=u.device)
+        for b in range(B):  # image b's joint sequence: its text rows, then its packed rows
+            rows = torch.cat([torch.arange(b * T, (b + 1) * T, device=u.device),
+                              torch.arange(Rt + int(cu[b]), Rt + int(cu[b + 1]), device=u.device)])
+            q, k, v = qkv[rows].view(-1, 3, heads, hd).permute(1, 2, 0, 3)
+            o[rows] = F.scaled_dot_product_attention(q[None], k[None], v[None])[0].permute(1, 0, 2).reshape(-1, d)
+        u = u + two(lambda a, s_: F.linear(a, t[(s_, "w_o")], t[(s_, "b_o")]), o).float()
+        h2 = F.layer_norm(u, (d,), eps=1e-6).to(torch.float16)
+        m = F.gelu(two(lambda a, s_: F.linear(a, t[(s_, "w_1")], t[(s_, "b_1")]), h2), approximate="tanh")
+        return u + two(lambda a, s_: F.linear(a, t[(s_, "w_2")], t[(s_, "b_2")]), m).float()
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(steps):
+            fn()
+        b_.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b_) / steps
+
+    cu_d = hp.split.cu_img
+    ours = timed(lambda: H.hilo_block_forward(sh, dw, cu_d, hp.cap, text, hp.packed, H.HILO_BF16, hp.out, hp.ws,
+                                              hp.ws_bytes, stream))
+    ref = timed(block)
+    # agreement of the two on these rows (both against the same bf16 inputs)
+    diff = (block() - hp.out[:Rt + L]).abs().max().item()
+    return {"torch_block_ms": ref, "hilo_block_ms_same_rows": ours, "hilo_speedup": ref / ours,
+            "max_abs_diff_vs_hilo": diff, "rows": Rt + L,
+            "what": "F.linear (cuBLAS) + F.scaled_dot_product_attention + F.layer_norm + F.gelu, "
+                    "same dtypes as the tcgen05 path; context only"}
+
+
 def time_fp8(H, I, torch, stream, wl, hp, inputs, bf16_peak: float, steps: int) -> dict:
     """FP8 (e4m3) GEMM operands on the timed workload: the block with and
     without them on the same packed rows, the hot path with them, and the FP8
@@ -803,6 +866,11 @@ def run_hilo(args):
                                  "tflops": dense_flops / (dense_ms * 1e-3) / 1e12,
                                  "speedup_of_compressed_block": dense_ms / t_block,
                                  "speedup_of_compressed_hot_path": dense_ms / ms_step}
+        try:  # context only: a failure here must not cost the bench line
+            extras["torch_context"] = time_torch_context(H, torch, stream, wl, hp, dw, (x, text, mask, kk, km),
+                                                         Ks)
+        except Exception as exc:  # noqa: BLE001
+            extras["torch_context"] = {"unavailable": f"{type(exc).__name__}: {exc}"[:300]}
         # end to end with host buffers, through the pipelined runner: every
         # step copies its inputs from pinned host memory and its result y back
         # to pinned host memory inside the timed region; the copies of
