@@ -550,23 +550,41 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
       tc_fence_after();
       const float inv = 1.0f / l;
       const int qr0 = i ? q_row0_1 : q_row0_0, qv = i ? q_valid_1 : q_valid_0;
-      uint4* dst = reinterpret_cast<uint4*>(p.out + static_cast<long long>(qr0 + row) * p.d + h * HD);
+      // O_i normalised to bf16 rows, staged through shared memory so that the
+      // global stores leave as whole 128-byte lines (one row per lane would
+      // write 16 bytes into 32 different rows per instruction). Each warp
+      // owns a slice of the K stages: every S product, the last reader of K,
+      // completed before O_i did, and no K copy is left to come. The 16-byte
+      // units of a row are XOR-swizzled by the row, so neither the writes
+      // (one row per lane) nor the reads (consecutive units of a row) collide
+      // in the shared-memory banks.
+      constexpr int UNITS = HD / 8;   // 16-byte units per row
+      constexpr int RPI = 32 / UNITS;  // rows per store instruction
+      uint4* stage = reinterpret_cast<uint4*>(smem + C::OFF_K) + warp * 32 * UNITS;
 #pragma unroll 1
       for (int c = 0; c < HD / 32; ++c) {
         float o[32];
         tmem_ld32(tO + c * 32, o);
         tmem_ld_wait();
-        if (row < qv) {
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            uint4 v;
-            v.x = pack_bf16x2(o[8 * j] * inv, o[8 * j + 1] * inv);
-            v.y = pack_bf16x2(o[8 * j + 2] * inv, o[8 * j + 3] * inv);
-            v.z = pack_bf16x2(o[8 * j + 4] * inv, o[8 * j + 5] * inv);
-            v.w = pack_bf16x2(o[8 * j + 6] * inv, o[8 * j + 7] * inv);
-            dst[4 * c + j] = v;
-          }
+        for (int j = 0; j < 4; ++j) {
+          uint4 v;
+          v.x = pack_bf16x2(o[8 * j] * inv, o[8 * j + 1] * inv);
+          v.y = pack_bf16x2(o[8 * j + 2] * inv, o[8 * j + 3] * inv);
+          v.z = pack_bf16x2(o[8 * j + 4] * inv, o[8 * j + 5] * inv);
+          v.w = pack_bf16x2(o[8 * j + 6] * inv, o[8 * j + 7] * inv);
+          stage[lane * UNITS + ((4 * c + j) ^ (lane & (UNITS - 1)))] = v;
         }
+      }
+      __syncwarp();
+      const int u = lane % UNITS;
+#pragma unroll 4
+      for (int k = 0; k < 32 / RPI; ++k) {
+        const int rr = k * RPI + lane / UNITS;  // row within the warp's 32
+        const int qrow = (warp & 3) * 32 + rr;  // row within the query tile
+        if (qrow < qv)
+          reinterpret_cast<uint4*>(p.out + static_cast<long long>(qr0 + qrow) * p.d + h * HD)[u] =
+              stage[rr * UNITS + (u ^ (rr & (UNITS - 1)))];
       }
     }
   }
