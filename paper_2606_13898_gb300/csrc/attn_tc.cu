@@ -131,6 +131,15 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// The largest of three floats in one instruction (three-input max.f32). A
+// maximum is exact, so grouping the row's values by threes gives the same
+// result as any other order.
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float y;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(y) : "f"(a), "f"(b), "f"(c));
+  return y;
+}
+
 // Row range of tile j of image b (text tiles first, then image tiles); used
 // for both query and key/value tiles.
 __device__ __forceinline__ void seq_tile(const AttnParams& p, int b, int L, int j, int& row0,
@@ -445,7 +454,8 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
       }
       tc_fence_after();
       // row max and row sum with 8 independent partials combined by a tree,
-      // so the reductions do not form one 128-long dependent chain; only the
+      // so the reductions do not form one 128-long dependent chain (the max
+      // of a full tile takes two keys per three-input max); only the
       // last key tile of a segment is ragged and needs masking
       const bool full_tile = valid == BKV;
       float s[BKV];
@@ -457,14 +467,16 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
       for (int u = 0; u < 8; ++u) mx8[u] = -INFINITY;
       if (full_tile) {
 #pragma unroll
-        for (int j = 0; j < BKV; ++j) mx8[j & 7] = fmaxf(mx8[j & 7], s[j]);
+        for (int j = 0; j < BKV; j += 16)
+#pragma unroll
+          for (int u = 0; u < 8; ++u) mx8[u] = fmax3(mx8[u], s[j + u], s[j + 8 + u]);
       } else {
 #pragma unroll
         for (int j = 0; j < BKV; ++j)
           if (j < valid) mx8[j & 7] = fmaxf(mx8[j & 7], s[j]);
       }
-      const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                             fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+      const float mx = fmax3(fmax3(mx8[0], mx8[1], mx8[2]), fmax3(mx8[3], mx8[4], mx8[5]),
+                             fmaxf(mx8[6], mx8[7]));
       const float m_tile = mx * p.scale_log2;
       bool rescale = false;
       float m_use = m;
