@@ -73,6 +73,21 @@ def test_score_linear_ramp_closed_form():
             assert np.all(s[i::2, j::2] == np.float32(d * e * e)), (i, j)
 
 
+def test_score_single_token_delta_position():
+    # zero field with one token (p0, q0) = (1, 2) set to c in every channel, on
+    # a 4 x 6 grid: its window (rows 0-1, cols 2-3) has mean c/4, so the token
+    # keeps 3c/4 and its three window mates -c/4; every other token is 0. The
+    # positions pin the grid's orientation (a transposed read moves them).
+    H, W, d, c = 4, 6, 16, 2.0
+    x = np.zeros((1, H, W, d))
+    x[0, 1, 2, :] = c
+    s = O.score(bits(x))[0].reshape(H, W)
+    want = np.zeros((H, W), dtype=np.float32)
+    want[0:2, 2:4] = np.float32(d * (c / 4) ** 2)
+    want[1, 2] = np.float32(d * (3 * c / 4) ** 2)
+    assert np.array_equal(s, want)
+
+
 def test_score_agrees_with_fp64_sum():
     wl = I.tiny_layer()
     b = I.make_batch(wl)
@@ -366,6 +381,18 @@ def test_pack_lf_is_the_downsampled_grid(lf):
 
 
 
+def test_pack_sums_members_in_raster_order():
+    # one 2x2 window, all four members pooled, channel values 2^26, 1, -2^26, 1
+    # in raster order: in fp32, (2^26 + 1) rounds to 2^26, so the raster-order
+    # sum is 1 and the mean 1/4 (column-major order would give 2 and 1/2)
+    v = np.array([2.0 ** 26, 1.0, -(2.0 ** 26), 1.0])
+    x = np.repeat(v.reshape(1, 2, 2, 1), 8, axis=3)
+    sp = O.split(np.zeros((1, 4), np.float32), np.zeros((1, 4), np.uint8), [0], [0], 2, 2, 1)
+    assert sp.counts[0].tolist() == [0, 1, 0]
+    packed = O.bf16_to_f32(O.pack(bits(x), sp))
+    assert np.all(packed == 0.25)
+
+
 def test_pack_constant_windows_lossless():
     rng = np.random.default_rng(4)
     H, W, d = 8, 8, 32
@@ -479,6 +506,15 @@ def test_attention_two_token_closed_form():
     k = np.array([[0.0], [math.log(2.0)]])
     v = np.array([[3.0], [6.0]])
     assert abs(O.softmax_attention(q, k, v)[0, 0] - 5.0) < 1e-12
+
+
+def test_attention_scale_closed_form():
+    # head_dim 4: the logit of key j is q.k_j / sqrt(4); with q.k = 2 ln 3
+    # the weights are 1/4 and 3/4 (a scale of 1/d or 1 would give others)
+    q = np.array([[1.0, 0.0, 0.0, 0.0]])
+    k = np.array([[0.0, 0.0, 0.0, 0.0], [2.0 * math.log(3.0), 0.0, 0.0, 0.0]])
+    v = np.array([[4.0, 0.0, 0.0, 0.0], [8.0, 0.0, 0.0, 0.0]])
+    assert abs(O.softmax_attention(q, k, v)[0, 0] - 7.0) < 1e-12
 
 
 def _rand_weights(rng, d, mlp):
