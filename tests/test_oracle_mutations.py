@@ -9,7 +9,9 @@ pins constrain that part of the oracle and do not just restate it:
 - a dropped value operand, and the row-size bias put on queries instead of keys;
 - square weights read transposed, the wrong pooling window, a different
   summation order of a window's members, a wrong e4m3 exponent bias and row
-  sizes off by one.
+  sizes off by one;
+- a delta unpool without the member's own value, e4m3 overflow to NaN, the
+  Sobel energy for its magnitude and a mask dilated one token short.
 """
 import math
 
@@ -21,6 +23,7 @@ from tests import test_oracle_pins as P
 
 _ranking, _layer_norm, _softmax, _bf16 = O.ranking, O.layer_norm, O.softmax_attention, O.bf16_to_f32
 _w, _members, _decode, _row_sizes = O._w, O.window_members, O.e4m3_decode, O.row_sizes
+_delta, _encode, _sobel, _dilate = O.unpack_delta, O.e4m3_encode, O.sobel_magnitude, O.dilate_mask
 
 
 def ranking_ties_high_index(s):
@@ -92,6 +95,28 @@ def row_sizes_plus_one(sp):
     return _row_sizes(sp) + np.float32(1.0)
 
 
+def delta_without_own_value(out_img, packed_bits, x_bits, sp):
+    # a pooled member gets the window's update but not its own value back
+    return _delta(out_img, packed_bits, np.zeros_like(x_bits), sp)
+
+
+def encode_no_saturation(t):
+    # magnitudes beyond 448 become NaN codes instead of saturating
+    c = _encode(t).copy()
+    big = np.abs(np.asarray(t, dtype=np.float64)) > 448.0
+    c[big] = (c[big] & 0x80) | 0x7F
+    return c
+
+
+def sobel_squared_magnitude(img):
+    # the gradient energy instead of its magnitude (square root dropped)
+    return _sobel(img) ** 2
+
+
+def dilate_one_short(mask, H, W, radius):
+    return _dilate(mask, H, W, max(0, radius - 1))
+
+
 def _brute_force_split():
     for seed in range(6):
         for levels in (1, 2):
@@ -106,6 +131,11 @@ def _block_brute_force():
 def _row_sizes_pins():
     for granular in (False, True):
         P.test_row_sizes_count_the_grid(granular)
+
+
+def _delta_pins():
+    for granular in (False, True):
+        P.test_unpack_delta_identity_block_returns_x(granular)
 
 
 def _hand_worked_splits():
@@ -139,6 +169,13 @@ MUTATIONS = {
     "e4m3 exponent bias off by one": ("e4m3_decode", decode_exponent_bias_off,
                                       [P.test_e4m3_codes_roundtrip_and_match_torch]),
     "row sizes off by one": ("row_sizes", row_sizes_plus_one, [_row_sizes_pins]),
+    "delta unpool drops the member's own value": ("unpack_delta", delta_without_own_value, [_delta_pins]),
+    "e4m3 overflow to NaN instead of saturation": ("e4m3_encode", encode_no_saturation,
+                                                   [P.test_e4m3_ties_saturation_subnormals]),
+    "Sobel energy instead of magnitude": ("sobel_magnitude", sobel_squared_magnitude,
+                                          [P.test_sobel_magnitude_matches_scipy_per_channel]),
+    "mask dilated one token short": ("dilate_mask", dilate_one_short,
+                                     [P.test_dilate_mask_brute_and_monotone_threshold]),
 }
 
 
