@@ -83,6 +83,13 @@ int check_shape(const hilo_shape* s, bool need_block) {
                 static_cast<long long>(s->H) * s->W);
   if (s->d < 128 || s->d % 128 || s->d > 4096)
     return fail(HILO_ERR_SHAPE, "d=%d must be a multiple of 128 in [128, 4096]", s->d);
+  {
+    // row indices (packed rows, cu_img, the block's row space) are int32
+    const long long N = static_cast<long long>(s->H) * s->W;
+    const long long per_image = N + (s->lf ? N / (s->lf * s->lf) : 0) + (s->T > 0 ? s->T : 0);
+    if (static_cast<long long>(s->B) * per_image > 0x7FFFFFFFLL)
+      return fail(HILO_ERR_SHAPE, "B=%d images of %lld rows exceed the int32 row space", s->B, per_image);
+  }
   if (need_block) {
     if (s->T < 0) return fail(HILO_ERR_SHAPE, "T=%d must be >= 0", s->T);
     if (s->heads < 1 || s->d % s->heads) return fail(HILO_ERR_SHAPE, "heads=%d must divide d=%d", s->heads, s->d);

@@ -51,6 +51,7 @@ def test_status_strings(H):
 @pytest.mark.parametrize("bad,code", [
     (dict(H=7), -2), (dict(W=0), -2), (dict(d=100), -2), (dict(d=8192), -2), (dict(B=0), -2),
     (dict(levels=3), -2), (dict(levels=2, H=6), -2), (dict(H=256, W=256), -2),
+    (dict(B=140000, H=128, W=128), -2),  # 2.3e9 rows: past the int32 row space
 ])
 def test_shape_rejected_before_launch(H, bad, code):
     kw = dict(B=1, H=8, W=8, d=128, T=4, heads=1, mlp=0, levels=1)
