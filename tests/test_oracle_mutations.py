@@ -11,7 +11,10 @@ pins constrain that part of the oracle and do not just restate it:
   summation order of a window's members, a wrong e4m3 exponent bias and row
   sizes off by one;
 - a delta unpool without the member's own value, e4m3 overflow to NaN, the
-  Sobel energy for its magnitude and a mask dilated one token short.
+  Sobel energy for its magnitude and a mask dilated one token short;
+- bf16 by truncation, the update's sign, e4m3 scales on the wrong axis, an
+  FP8 GEMM without its weight scale, an inclusive selector threshold and an
+  unpack that reads the next row.
 """
 import math
 
@@ -24,6 +27,7 @@ from tests import test_oracle_pins as P
 _ranking, _layer_norm, _softmax, _bf16 = O.ranking, O.layer_norm, O.softmax_attention, O.bf16_to_f32
 _w, _members, _decode, _row_sizes = O._w, O.window_members, O.e4m3_decode, O.row_sizes
 _delta, _encode, _sobel, _dilate = O.unpack_delta, O.e4m3_encode, O.sobel_magnitude, O.dilate_mask
+_update, _select = O.update, O.sobel_select
 
 
 def ranking_ties_high_index(s):
@@ -117,6 +121,35 @@ def dilate_one_short(mask, H, W, radius):
     return _dilate(mask, H, W, max(0, radius - 1))
 
 
+def bf16_truncating(a):
+    # fp32 -> bf16 by dropping the low half instead of rounding to nearest even
+    return (np.ascontiguousarray(a, dtype=np.float32).view(np.uint32) >> np.uint32(16)).astype(np.uint16)
+
+
+def update_sign_flipped(x_bits, y, alpha):
+    return _update(x_bits, y, -alpha)
+
+
+def dequant_scale_on_columns(codes, scale):
+    return O.e4m3_decode(codes) * np.asarray(scale, np.float64)[None, :]
+
+
+def gemm_e4m3_without_weight_scale(a64, wq, bias=None):
+    ca, sa = O.quantize_rows(np.asarray(a64, dtype=np.float32))
+    cw, _ = wq
+    out = (O.e4m3_decode(ca) @ O.e4m3_decode(cw).T) * sa.astype(np.float64)[:, None]
+    return out if bias is None else out + O._w(bias)
+
+
+def select_inclusive_threshold(img, mask, H, W, patch, radius, threshold):
+    # ">=" instead of the strict ">"
+    return _select(img, mask, H, W, patch, radius, float(np.nextafter(np.float32(threshold), np.float32(-1))))
+
+
+def unpack_next_row(out_img, sp):
+    return out_img[np.minimum(sp.tok_row + 1, out_img.shape[0] - 1)]
+
+
 def _brute_force_split():
     for seed in range(6):
         for levels in (1, 2):
@@ -176,6 +209,19 @@ MUTATIONS = {
                                           [P.test_sobel_magnitude_matches_scipy_per_channel]),
     "mask dilated one token short": ("dilate_mask", dilate_one_short,
                                      [P.test_dilate_mask_brute_and_monotone_threshold]),
+    "bf16 by truncation": ("f32_to_bf16", bf16_truncating,
+                           [P.test_bf16_rounding_matches_torch, P.test_update_closed_form]),
+    "update adds instead of subtracting": ("update", update_sign_flipped, [P.test_update_closed_form]),
+    "e4m3 scales broadcast over columns": ("dequant", dequant_scale_on_columns,
+                                          [P.test_quantize_rows_error_bound,
+                                           P.test_gemm_e4m3_exact_on_representable_operands_and_scale_invariance]),
+    "FP8 GEMM without the weight scale": ("gemm_e4m3", gemm_e4m3_without_weight_scale,
+                                          [P.test_gemm_e4m3_exact_on_representable_operands_and_scale_invariance]),
+    "selector threshold inclusive": ("sobel_select", select_inclusive_threshold,
+                                     [P.test_sobel_select_ramp_and_strict_threshold]),
+    "unpack reads the next row": ("unpack", unpack_next_row,
+                                  [P.test_pack_constant_windows_lossless,
+                                   P.test_unpack_pack_identity_on_kept_rows_and_brute_mean]),
 }
 
 
