@@ -33,8 +33,9 @@
  *   channels. Rows [0, B*T) are the text tokens (image b owns rows
  *   b*T .. b*T+T-1); rows [B*T, B*T + cu_img[B]) are the packed image rows
  *   (image b owns B*T + cu_img[b] .. B*T + cu_img[b+1] - 1). cap >= cu_img[B]
- *   is the capacity the caller allocated (B*H*W always suffices), so no host
- *   read-back of the data-dependent row counts is ever needed.
+ *   is the capacity the caller allocated (hilo_row_capacity always suffices:
+ *   B*H*W without the low-frequency set), so no host read-back of the
+ *   data-dependent row counts is ever needed.
  */
 #ifndef HILO_H
 #define HILO_H
@@ -79,7 +80,8 @@ enum { HILO_BF16 = 0, HILO_F32 = 1, HILO_F16 = 2 };
  *           concatenated with every token of a downsampled image; here the
  *           grid average-pooled lf-fold per side, all members included).
  *           Needs levels == 1 and H, W multiples of lf.
- * Any other combination returns HILO_ERR_SHAPE.
+ * Also H*W <= 32768, and B * (H*W (+ H*W/lf^2) + T) < 2^31 (row indices are
+ * int32). Any other combination returns HILO_ERR_SHAPE.
  */
 typedef struct {
   int32_t B, H, W, d, T, heads, mlp, levels, lf;
