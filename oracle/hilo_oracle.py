@@ -97,12 +97,13 @@ LF = 3
 
 
 def bf16_to_f32(bits: np.ndarray) -> np.ndarray:
-    """Exact widening of bf16 bit patterns to fp32."""
+    """Exact widening of bf16 bit patterns to fp32. Numeric helper (bf16 storage of activations and weights); no
+    paper passage."""
     return (np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)).view(np.float32)
 
 
 def f32_to_bf16(a: np.ndarray) -> np.ndarray:
-    """fp32 -> bf16 bit pattern, round to nearest, ties to even (finite inputs)."""
+    """fp32 -> bf16 bit pattern, round to nearest, ties to even (finite inputs). Numeric helper; no paper passage."""
     u = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32).astype(np.uint64)
     keep_lsb = (u >> np.uint64(16)) & np.uint64(1)
     rounded = (u + np.uint64(0x7FFF) + keep_lsb) >> np.uint64(16)
@@ -119,6 +120,8 @@ def score(x_bits: np.ndarray) -> np.ndarray:
 
     x_bits: uint16 [B,H,W,d] (bf16); H, W even; d a multiple of 8.
     Returns fp32 [B, H*W].
+
+    Paper: Sec. 2.3, HiLo-Token Selection (the frequency map, token-space form).
     """
     B, H, W, d = x_bits.shape
     assert H % 2 == 0 and W % 2 == 0 and d % 8 == 0
@@ -143,7 +146,7 @@ def score(x_bits: np.ndarray) -> np.ndarray:
 
 
 def score_f64(x_bits: np.ndarray) -> np.ndarray:
-    """The same energy in fp64, summed plainly (a sanity reference)."""
+    """The same energy in fp64, summed plainly (a sanity reference). Paper: Sec. 2.3, as score."""
     B, H, W, d = x_bits.shape
     x = bf16_to_f32(x_bits).astype(np.float64)
     m = x.reshape(B, H // 2, 2, W // 2, 2, d).mean(axis=(2, 4))
@@ -166,7 +169,8 @@ class Split:
 
 
 def ranking(s: np.ndarray) -> np.ndarray:
-    """Token ids ordered by (score descending, token index ascending)."""
+    """Token ids ordered by (score descending, token index ascending). Paper: Sec. 2.3, HiLo-Token Selection
+    (high-frequency tokens are selected)."""
     idx = np.arange(s.shape[0])
     return np.lexsort((idx, -s.astype(np.float64)))
 
@@ -270,7 +274,8 @@ def _split_lf(s, mask, k_keep, H: int, W: int, lf: int) -> Split:
 
 
 def window_members(w: int, size: int, W: int) -> list[int]:
-    """Token ids of aligned size x size window ``w`` in raster order."""
+    """Token ids of aligned size x size window ``w`` in raster order. Paper: Sec. 2.3 (the pooled low-frequency
+    regions)."""
     wp, wq = divmod(w, W // size)
     return [(size * wp + i) * W + size * wq + j for i in range(size) for j in range(size)]
 
@@ -278,7 +283,9 @@ def window_members(w: int, size: int, W: int) -> list[int]:
 def pack(x_bits: np.ndarray, sp: Split, lf: int = 0) -> np.ndarray:
     """Packed image rows, uint16 [rows, d] (bf16). With lf > 0 (a split made
     with the same lf) the rows after the kept tokens are the lf x lf window
-    means over all members."""
+    means over all members.
+
+    Paper: Sec. 2.3 (selected and low-frequency tokens concatenated along the token axis)."""
     B, H, W, d = x_bits.shape
     x = bf16_to_f32(x_bits).reshape(B, H * W, d)
     out = np.empty((int(sp.cu_img[-1]), d), dtype=np.uint16)
@@ -309,14 +316,15 @@ def pack(x_bits: np.ndarray, sp: Split, lf: int = 0) -> np.ndarray:
 
 
 def layer_norm(u: np.ndarray, eps: float = 1e-6) -> np.ndarray:
-    """LayerNorm over the last axis, no affine, biased variance."""
+    """LayerNorm over the last axis, no affine, biased variance. Paper: Sec. 2.1 (the DiT block of the editing
+    generalist)."""
     mu = u.mean(axis=-1, keepdims=True)
     var = ((u - mu) ** 2).mean(axis=-1, keepdims=True)
     return (u - mu) / np.sqrt(var + eps)
 
 
 def gelu_tanh(z: np.ndarray) -> np.ndarray:
-    """GELU, tanh approximation."""
+    """GELU, tanh approximation. Paper: Sec. 2.1 (the DiT block's MLP)."""
     return 0.5 * z * (1.0 + np.tanh(math.sqrt(2.0 / math.pi) * (z + 0.044715 * z ** 3)))
 
 
@@ -325,7 +333,9 @@ def softmax_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, key_n=None) -
 
     key_n (optional, one positive weight per key) is proportional attention:
     ln(key_n[j]) is added to every logit of key j, so a key standing for n
-    tokens receives the attention mass of n identical copies of itself."""
+    tokens receives the attention mass of n identical copies of itself.
+
+    Paper: Sec. 2.1 (the DiT's joint attention); Sec. 2.3 for the compressed keys."""
     sc = (q @ k.T) / math.sqrt(q.shape[-1])
     if key_n is not None:
         # a weight of 0 (a low-frequency row all of whose members are kept)
@@ -347,7 +357,9 @@ def _w(bits) -> np.ndarray:
 
 def weights_f64(w):
     """A copy of block weights widened to fp64 once (same values as _w gives
-    per call), for callers that run the block many times."""
+    per call), for callers that run the block many times.
+
+    Helper; no paper passage."""
     import copy
     out = copy.copy(w)
     for sname in ("txt", "img"):
@@ -373,6 +385,8 @@ def block(u_txt, u_img, cu_img, T: int, weights, heads: int, mlp: bool, n_img=No
     ``weights`` has ``.txt`` and ``.img`` with PyTorch-layout [out, in] arrays.
     n_img (optional): proportional attention, the number of grid tokens each
     packed image row stands for (text keys count 1), see softmax_attention.
+
+    Paper: Sec. 2.1 (the DiT block) on the sequence Sec. 2.3 compresses.
     """
     ut = _as_f64(u_txt)
     ui = _as_f64(u_img)
@@ -409,6 +423,8 @@ def block_rows(u_txt, u_img, cu_img, T: int, weights, heads: int, mlp: bool, b: 
     Same arithmetic as ``block``; keys and values of the whole joint sequence
     of image b are projected, queries, attention and MLP only for the given
     rows (absolute row ids in u_txt / u_img). Returns fp64 (txt_out, img_out).
+
+    Paper: Sec. 2.1, as block.
     """
     ut = _as_f64(u_txt)
     ui = _as_f64(u_img)
@@ -441,7 +457,8 @@ def block_rows(u_txt, u_img, cu_img, T: int, weights, heads: int, mlp: bool, b: 
 
 
 def block_dense(x_bits, text_bits, weights, heads: int, mlp: bool):
-    """The uncompressed block: every grid token in raster order, no pooling."""
+    """The uncompressed block: every grid token in raster order, no pooling. Paper: Sec. 2.1 (the uncompressed
+    DiT the speed-ups of Sec. 3.3 are measured against)."""
     B, H, W, d = x_bits.shape
     cu = np.arange(B + 1, dtype=np.int64) * (H * W)
     return block(text_bits.reshape(B * text_bits.shape[1], d), x_bits.reshape(B * H * W, d),
@@ -455,7 +472,9 @@ def block_dense(x_bits, text_bits, weights, heads: int, mlp: bool):
 
 def row_sizes(sp: Split) -> np.ndarray:
     """Number of grid tokens each packed image row stands for: 1 for a kept
-    token, the number of its class members for a pooled window (fp32)."""
+    token, the number of its class members for a pooled window (fp32).
+
+    Paper: Sec. 2.3 is silent on how pooled tokens attend; this supports the proportional reading."""
     n = np.zeros(int(sp.cu_img[-1]), dtype=np.float32)
     for b in range(sp.labels.shape[0]):
         np.add.at(n, sp.tok_row[b], np.float32(1.0))
@@ -463,7 +482,8 @@ def row_sizes(sp: Split) -> np.ndarray:
 
 
 def unpack(out_img: np.ndarray, sp: Split) -> np.ndarray:
-    """y[b, i] = out_img[tok_row[b, i]]  ->  [B, N, d]."""
+    """y[b, i] = out_img[tok_row[b, i]]  ->  [B, N, d]. Paper: Sec. 2.3 (the compressed tokens restored to the
+    full grid)."""
     return out_img[sp.tok_row]
 
 
@@ -490,7 +510,8 @@ def unpack_delta(out_img: np.ndarray, packed_bits: np.ndarray, x_bits: np.ndarra
 
 
 def update(x_bits: np.ndarray, y: np.ndarray, alpha: float) -> np.ndarray:
-    """x <- bf16(x - alpha * y), fp32 multiply then subtract (no FMA)."""
+    """x <- bf16(x - alpha * y), fp32 multiply then subtract (no FMA). No paper formula: a plain update step of
+    the denoising loop (Sec. 2.4 distils an 8-step sampler)."""
     x = bf16_to_f32(x_bits)
     t = np.float32(alpha) * np.asarray(y, dtype=np.float32)
     return f32_to_bf16(x - t)
@@ -515,7 +536,9 @@ def e4m3_encode(t: np.ndarray) -> np.ndarray:
     the lowest kept bit (round half to even) and clear the 20 dropped bits; a
     carry into the exponent is the next binade's value, as it should be.
     Below 2^-6 the values are multiples of the subnormal quantum 2^-9,
-    rounded half to even by rint."""
+    rounded half to even by rint.
+
+    Paper: Sec. 3.3 reports FP8 on top of HiLo-Token; the format is IEEE-style e4m3."""
     t = np.asarray(t, dtype=np.float32)
     sign = ((t.view(np.uint32) >> 24) & 0x80).astype(np.uint8)
     a = np.abs(t)
@@ -534,7 +557,7 @@ def e4m3_encode(t: np.ndarray) -> np.ndarray:
 
 
 def e4m3_decode(c: np.ndarray) -> np.ndarray:
-    """e4m3 codes -> values (fp64; 0x7f / 0xff are NaN)."""
+    """e4m3 codes -> values (fp64; 0x7f / 0xff are NaN). Paper: Sec. 3.3, as e4m3_encode."""
     c = np.asarray(c, dtype=np.uint8).astype(np.int64)
     s = np.where(c & 0x80, -1.0, 1.0)
     ef = (c >> 3) & 0xF
@@ -549,7 +572,9 @@ def quantize_rows(x) -> tuple[np.ndarray, np.ndarray]:
     the row, inv = 448 / amax and scale = amax / 448 (each one correctly
     rounded fp32 division; 1 for an all-zero row), code = e4m3(x * inv) with
     the product rounded to fp32 first. Returns (codes uint8 [R, C], scale
-    fp32 [R]); code value times scale approximates x."""
+    fp32 [R]); code value times scale approximates x.
+
+    Paper: Sec. 3.3 (FP8); the scaling scheme is this implementation's."""
     x = np.asarray(x, dtype=np.float32)
     amax = np.abs(x).max(axis=1) if x.shape[1] else np.zeros(x.shape[0], np.float32)
     pos = amax > 0
@@ -560,6 +585,7 @@ def quantize_rows(x) -> tuple[np.ndarray, np.ndarray]:
 
 
 def dequant(codes, scale) -> np.ndarray:
+    """Paper: Sec. 3.3 (FP8): codes times their row scales."""
     return e4m3_decode(codes) * np.asarray(scale, np.float64)[:, None]
 
 
@@ -567,7 +593,9 @@ def gemm_e4m3(a64, wq, bias=None) -> np.ndarray:
     """One FP8 GEMM as the kernels take it: the activations a [R, K] rounded
     to fp32 and quantised per row, the weights wq = (codes [N, K], scale [N])
     quantised per output channel; out = (codes_A codes_W^T) * scale_A[r] *
-    scale_W[o] (+ bias), in fp64."""
+    scale_W[o] (+ bias), in fp64.
+
+    Paper: Sec. 3.3 (FP8)."""
     ca, sa = quantize_rows(np.asarray(a64, dtype=np.float32))
     cw, sw = wq
     acc = e4m3_decode(ca) @ e4m3_decode(cw).T
@@ -576,7 +604,8 @@ def gemm_e4m3(a64, wq, bias=None) -> np.ndarray:
 
 
 def f32_to_f16_sat(a) -> np.ndarray:
-    """fp32 -> fp16 (round to nearest even, saturating at +-65504), as fp64."""
+    """fp32 -> fp16 (round to nearest even, saturating at +-65504), as fp64. Numeric helper (the MLP's fp16
+    operands); no paper passage."""
     a = np.clip(np.asarray(a, dtype=np.float64), -65504.0, 65504.0)
     return a.astype(np.float32).astype(np.float16).astype(np.float64)
 
@@ -589,7 +618,9 @@ def block_fp8(u_txt, u_img, cu_img, T: int, weights_q, heads: int, mlp: bool):
     MLP1 -> GELU rounded to fp16 -> per-row e4m3 -> MLP2. The residual stream
     stays fp64 here (fp32 in the kernels). ``weights_q`` per stream holds
     (codes, scale) for w_qkv, w_o, w_1, w_2 (see quantize_weights) and the
-    bf16 biases. Returns fp64 (txt, img)."""
+    bf16 biases. Returns fp64 (txt, img).
+
+    Paper: Sec. 3.3 (FP8 on top of HiLo-Token) applied to the Sec. 2.1 block."""
     ut = _as_f64(u_txt)
     ui = _as_f64(u_img)
     d = ut.shape[1] if ut.size else ui.shape[1]
@@ -630,7 +661,9 @@ def block_rows_fp8(u_txt, u_img, cu_img, T: int, weights_q, heads: int, mlp: boo
     """block_fp8's outputs for selected rows of image ``b`` only: keys and
     values of the whole joint sequence of image b (each row's quantisation
     depends on that row alone), queries, attention, out-projection and MLP
-    for the given rows (absolute row ids in u_txt / u_img). fp64 (txt, img)."""
+    for the given rows (absolute row ids in u_txt / u_img). fp64 (txt, img).
+
+    Paper: Sec. 3.3, as block_fp8."""
     ut = _as_f64(u_txt)
     ui = _as_f64(u_img)
     d = ut.shape[1] if ut.size else ui.shape[1]
@@ -689,7 +722,9 @@ class BlockWeightsQ:
 
 def quantize_weights(w) -> BlockWeightsQ:
     """Per-output-channel e4m3 weights (each row of W[out, in] quantised as
-    in quantize_rows, from the bf16 values); biases stay bf16."""
+    in quantize_rows, from the bf16 values); biases stay bf16.
+
+    Paper: Sec. 3.3 (FP8)."""
     def one(s):
         q = lambda m: quantize_rows(bf16_to_f32(m)) if m is not None else None
         return StreamWeightsQ(q(s.w_qkv), s.b_qkv, q(s.w_o), s.b_o, q(s.w_1), s.b_1, q(s.w_2), s.b_2)
@@ -763,6 +798,8 @@ def hot_path(x_bits, text_bits, mask, k_keep, k_mid, levels, weights_list, heads
     proportional attention (each packed row weighted by its row size).
 
     Returns (split, packed, (txt_out, img_out), y) with the block outputs in fp64.
+
+    Paper: Sec. 2.3 (selection, the DiT on the compressed sequence, restoration).
     """
     B, H, W, d = x_bits.shape
     T = text_bits.shape[1]
