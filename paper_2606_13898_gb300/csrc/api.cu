@@ -1,6 +1,8 @@
 // extern "C" entry points of libhilo (declared in include/hilo.h): argument
 // and shape validation on the host, workspace layout, launch orchestration
-// of the kernels, device error reporting.
+// of the kernels, device error reporting. The path they run is paper
+// Sec. 2.3 (selection, pooling, the DiT on the compressed sequence,
+// restoration); each entry point's passage is cited in include/hilo.h.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <atomic>

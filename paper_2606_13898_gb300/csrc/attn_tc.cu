@@ -1,4 +1,6 @@
-// Joint variable-length softmax attention of the MMDiT block on tcgen05.
+// Joint variable-length softmax attention of the MMDiT block on tcgen05
+// (paper Sec. 2.1: the DiT of the editing generalist; Sec. 2.3: the
+// compressed image tokens attend jointly with the text tokens).
 //
 // Image b attends over its joint sequence [T text rows ; L_b packed image
 // rows] (non-causal, scale 1/sqrt(head_dim)); L_b comes from the device

@@ -1,7 +1,9 @@
 // Bandwidth- and latency-bound kernels of the HiLo-Token hot path:
 //   score  (per-token high-frequency energy, Sec. 2.3 frequency map)
-//   split  (top-k select with index tie-break, mask union, compaction)
-//   pack / unpack / unpack_update (gather + pooling, scatter + broadcast)
+//   split  (top-k select with index tie-break, mask union, compaction;
+//          Sec. 2.3: high-frequency and mask tokens kept, the rest pooled)
+//   pack / unpack / unpack_update (gather + pooling, scatter + broadcast;
+//          Sec. 2.3: the packed sequence and its restoration to the grid)
 //   layernorm (the block's pre-norm: bf16 or fp16 operand for the next GEMM)
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>

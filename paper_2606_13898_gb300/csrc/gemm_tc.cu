@@ -1,5 +1,6 @@
 // Grouped bf16 GEMM on the 5th-generation tensor cores (tcgen05) for the
-// MMDiT block's linear layers: C[r, n] = sum_k A[r, k] * W_g[n, k] + b_g[n]
+// MMDiT block's linear layers (paper Sec. 2.1, the DiT's QKV, output and MLP
+// projections): C[r, n] = sum_k A[r, k] * W_g[n, k] + b_g[n]
 // with the text rows (group 0) and the packed image rows (group 1) of the
 // row space using their own weights. The image row count is read on the
 // device, so no host synchronisation is needed between split and block.

@@ -1,4 +1,5 @@
-"""Thin Python binding of libhilo's C ABI (include/hilo.h).
+"""Thin Python binding of libhilo's C ABI (include/hilo.h): the HiLo-Token
+hot path of paper Sec. 2.3 around the DiT block of Sec. 2.1.
 
 Functions carry the C names and only marshal arguments: torch tensors are
 passed as device pointers, the shape as a ``hilo_shape`` struct, the stream
