@@ -40,7 +40,7 @@ FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
 
 
-def parse():
+def parse(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=2000)
@@ -50,7 +50,7 @@ def parse():
     ap.add_argument("--no-extras", action="store_true", help="skip sweep / dense / e2e / cpu_baseline")
     ap.add_argument("--variant", choices=["bf16", "fp8"], default="bf16",
                     help="fp8: the timed step's blocks take e4m3 GEMM operands (no extras)")
-    return ap.parse_args()
+    return ap.parse_args(argv)
 
 
 def peaks():
@@ -206,10 +206,16 @@ def cpu_baseline(ratio: str, min_seconds: float = 10.0):
 
 
 def run_reference(args):
+    from oracle import hilo_oracle as O
+    from paper_2606_13898_gb300 import inputs as I
     from paper_2606_13898_gb300 import replicas
-    rank, _, _ = replicas.env_rank_world()
+    rank, world, _ = replicas.env_rank_world()
     if rank != 0:
         return
+    # the workload's packed row count (for the config the GPU arm reports)
+    wl = workload(args.ratio)
+    b = I.make_batch(wl)
+    packed_rows = int(O.split(O.score(b.x), b.mask, b.k_keep, b.k_mid, wl.H, wl.W, wl.levels).cu_img[-1])
     budget = 150.0
     per_step = budget / max(1, args.steps + args.warmup)
     # calibrate on an 8x8 crop, then take the largest crop that fits the per-step budget
@@ -235,13 +241,29 @@ def run_reference(args):
             f"tokens, d=3072, keep ratio {args.ratio}) of the 64x64 workload; value = crop tokens / step time")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * el / args.steps,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": workload(args.ratio).name, "B": 1, "H": 64, "W": 64,
-                                            "T": 512, "d": 3072, "heads": 24, "keep_ratio": args.ratio},
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f64 block, fp32 score/split/pack", "data": "synthetic",
+            "config": line_config(wl, args.ratio, packed_rows, world),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
                              "sample": desc},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------ the line's config --
+
+DTYPE_BF16 = "bf16 (MLP GEMM operands fp16)"
+DTYPE_FP8 = "fp8-e4m3 GEMM operands, bf16 attention"
+
+
+def line_config(wl, ratio: str, packed_rows: int, world: int, fp8: bool = False) -> dict:
+    """The ``config`` of the JSON line, identical for both arms: the workload
+    and the packed rows its split produces (a property of the inputs)."""
+    return {"workload": wl.name + ("_fp8" if fp8 else ""), "B": wl.B, "H": wl.H, "W": wl.W, "T": wl.T,
+            "d": wl.d, "heads": wl.heads, "mlp": "4x GELU", "keep_ratio": ratio, "mask": "rect 10-40%",
+            "packed_image_rows": int(packed_rows), "block_rows": int(wl.B * wl.T + packed_rows),
+            "parallelism": f"replicas x{world}",
+            "l2": "no flush: per-step working set > 129 MB L2 (weights: 453 MB bf16, 227 MB e4m3)"}
 
 
 # --------------------------------------------------------------- GPU arm --
@@ -533,16 +555,57 @@ def time_fp8(H, I, torch, stream, wl, hp, inputs, bf16_peak: float, steps: int) 
             "fp8_peak_note": "2 x measured bf16 dense (the nominal fp8 : bf16 ratio)"}
 
 
-def time_configs(H, I, torch, stream, steps: int):
+def oracle_config_baseline(wl, batch, host_weights) -> dict:
+    """The oracle, as it stands, on one workload configuration, timed once on
+    this host's cores: the whole hot path (score -> split -> pack -> block(s)
+    -> unpack) on the same inputs the GPU ran. The weights are widened to fp64
+    outside the timed region (a model load), one layer at a time for the
+    8-block loop, whose 28 steps are extrapolated from one timed step."""
+    from oracle import hilo_oracle as O
+    x, text = batch.x, batch.text
+    T = text.shape[1]
+    if len(host_weights) == 1:
+        w = O.weights_f64(host_weights[0])
+        t0 = time.perf_counter()
+        O.hot_path(x, text, batch.mask, batch.k_keep, batch.k_mid, wl.levels, [w], wl.heads, wl.mlp)
+        el = time.perf_counter() - t0
+        return {"value": wl.B * wl.N / el, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
+                "seconds": el, "sample": f"one full hot-path pass of this configuration ({wl.B} x {wl.H}x{wl.W} "
+                                         f"grid, {T} text, d={wl.d}) in {el:.1f} s"}
+    el = 0.0
+    t0 = time.perf_counter()
+    sp = O.split(O.score(x), batch.mask, batch.k_keep, batch.k_mid, wl.H, wl.W, wl.levels)
+    packed = O.pack(x, sp)
+    el += time.perf_counter() - t0
+    ut, ui = text.reshape(wl.B * T, wl.d), packed
+    for hw in host_weights:
+        w = O.weights_f64(hw)
+        t0 = time.perf_counter()
+        ut, ui = O.block(ut, ui, sp.cu_img, T, w, wl.heads, wl.mlp)
+        el += time.perf_counter() - t0
+        del w
+    t0 = time.perf_counter()
+    O.update(x, O.unpack(ui, sp), 0.035)
+    el += time.perf_counter() - t0
+    return {"value": wl.B * wl.N / el, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
+            "seconds_per_step": el, "seconds_28_steps_extrapolated": 28 * el,
+            "sample": f"one of the 28 steps ({len(host_weights)} blocks, split, pack, unpack and update) "
+                      f"timed in {el:.1f} s; the 28-step time is that x 28 (extrapolated)"}
+
+
+def time_configs(H, I, torch, stream, steps: int, bf16_peak: float, peak_src: str, with_oracle: bool):
     """Hot path, compressed block and dense block of each workload configuration.
 
     Returns a dict keyed by workload name: hot-path ms (score -> split -> pack
     -> block(s) -> unpack), block ms, image-tokens/s over the full grids, block
-    TFLOP/s, and the dense block (every grid token a row, same kernels). The
-    denoising loop runs its 28 steps of 8 blocks once and is compared with a
-    dense 8-block stack per step.
+    TFLOP/s and its fraction of the measured bf16 peak, and the dense block
+    (every grid token a row, same kernels). The denoising loop runs its 28
+    steps of 8 blocks once and is compared with a dense 8-block stack per
+    step. With ``with_oracle`` each configuration also carries the oracle
+    timed on the host cores on the same inputs (``cpu_baseline``).
     """
     res = {}
+    frac_note = f"block FLOPs / block time / {peak_src} bf16 dense peak ({bf16_peak:.0f} TFLOP/s)"
 
     def ev():
         return torch.cuda.Event(enable_timing=True)
@@ -556,7 +619,8 @@ def time_configs(H, I, torch, stream, steps: int):
 
     for wl in (I.tiny_layer(), I.block_64_batch4(), I.block_128_two_level()):
         b = I.make_batch(wl)
-        dw = H.DeviceWeights.from_host(I.make_weights(wl.d, wl.mlp, seed=I.weight_seed(wl)))
+        hw = I.make_weights(wl.d, wl.mlp, seed=I.weight_seed(wl))
+        dw = H.DeviceWeights.from_host(hw)
         sh = shape_of(wl)
         hp = H.HotPath(sh, [dw])
         x, t, m, kk, km = inputs(b)
@@ -592,19 +656,25 @@ def time_configs(H, I, torch, stream, steps: int):
         torch.cuda.synchronize()
         dense = b0.elapsed_time(b1) / steps
         H.hilo_sync_status()
+        blk_tf = block_flops(wl, cu) / (blk * 1e-3) / 1e12
+        dense_tf = block_flops(wl, cu_dense.cpu().numpy()) / (dense * 1e-3) / 1e12
         res[wl.name] = {"hot_path_ms": hot, "block_ms": blk, "image_tokens_per_s": n_img / (hot * 1e-3),
-                        "block_tflops": block_flops(wl, cu) / (blk * 1e-3) / 1e12,
+                        "block_tflops": blk_tf, "frac_bf16": blk_tf / bf16_peak,
                         "packed_image_rows": cu.tolist()[1:] if wl.B > 1 else int(cu[-1]),
-                        "dense_block_ms": dense,
-                        "dense_block_tflops": block_flops(wl, cu_dense.cpu().numpy()) / (dense * 1e-3) / 1e12,
-                        "block_speedup_vs_dense": dense / blk}
+                        "dense_block_ms": dense, "dense_block_tflops": dense_tf,
+                        "dense_frac_bf16": dense_tf / bf16_peak,
+                        "block_speedup_vs_dense": dense / blk, "frac_of": frac_note}
         del hp, dw
         torch.cuda.empty_cache()
+        if with_oracle:
+            res[wl.name]["cpu_baseline"] = oracle_config_baseline(wl, b, [hw])
+        del hw
 
     # denoising loop: 8 blocks x 28 steps, latents updated in place
     wl = I.denoise_loop()
     b = I.make_batch(wl)
-    dws = [H.DeviceWeights.from_host(I.make_weights(wl.d, wl.mlp, seed=I.weight_seed(wl, i))) for i in range(8)]
+    hws = [I.make_weights(wl.d, wl.mlp, seed=I.weight_seed(wl, i)) for i in range(8)]
+    dws = [H.DeviceWeights.from_host(hw) for hw in hws]
     sh = shape_of(wl)
     hp = H.HotPath(sh, dws)
     x, t, m, kk, km = inputs(b)
@@ -646,12 +716,19 @@ def time_configs(H, I, torch, stream, steps: int):
     torch.cuda.synchronize()
     dense_step_ms = a0.elapsed_time(a1) / 5
     H.hilo_sync_status()
+    cu4 = hp.split.cu_img.cpu().numpy()
+    loop_tf = 8 * block_flops(wl, cu4) / (total / 28 * 1e-3) / 1e12
     res[wl.name] = {"total_ms_28_steps": total, "ms_per_step": total / 28,
                     "image_tokens_per_s": wl.N * 28 / (total * 1e-3),
+                    "step_tflops": loop_tf, "frac_bf16": loop_tf / bf16_peak,
+                    "frac_of": f"8 blocks' FLOPs per step / whole step time (score, split, pack, unpack and "
+                               f"update included) / {peak_src} bf16 dense peak ({bf16_peak:.0f} TFLOP/s)",
                     "dense_8_block_ms_per_step": dense_step_ms, "dense_total_ms_28_steps": dense_step_ms * 28,
                     "speedup_vs_dense": dense_step_ms * 28 / total}
     del hp, dws
     torch.cuda.empty_cache()
+    if with_oracle:
+        res[wl.name]["cpu_baseline"] = oracle_config_baseline(wl, b, hws)
     return res
 
 
@@ -807,11 +884,8 @@ def run_hilo(args):
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
         "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "fp8-e4m3 GEMM operands, bf16 attention" if fp8 else "bf16", "data": "synthetic",
-        "config": {"workload": wl.name + ("_fp8" if fp8 else ""), "B": wl.B, "H": wl.H, "W": wl.W, "T": wl.T, "d": wl.d,
-                   "heads": wl.heads, "mlp": "4x GELU", "keep_ratio": args.ratio, "mask": "rect 10-40%",
-                   "packed_image_rows": L, "block_rows": M, "parallelism": f"replicas x{world}",
-                   "l2": "no flush: per-step working set > 129 MB L2 (weights: 453 MB bf16, 227 MB e4m3)"},
+        "dtype": DTYPE_FP8 if fp8 else DTYPE_BF16, "data": "synthetic",
+        "config": line_config(wl, args.ratio, L, world, fp8),
         "block_ms": t_block, "block_tflops": block_tflops,
         "roofline": {"bound": "tensor", "kernel": "gemm2_kernel (tcgen05 cta_group::2" +
                      (", kind::f8f6f4)" if fp8 else ")"), "achieved": gemm_tflops,
@@ -851,7 +925,8 @@ def run_hilo(args):
         extras["low_frequency_set"] = time_lf(H, torch, stream, wl, dw, (x, text, mask, kk, km), Ks)
         extras["fp8"] = time_fp8(H, I, torch, stream, wl, hp, (x, text, mask, kk, km), bf16_peak, Ks)
         if world == 1:
-            extras["configs"] = time_configs(H, I, torch, stream, steps=20)
+            extras["configs"] = time_configs(H, I, torch, stream, steps=20, bf16_peak=bf16_peak, peak_src=peak_src,
+                                             with_oracle=rank == 0)
         # dense block: every grid token is its own row, no score/split/pack/unpack
         cu_dense = torch.arange(wl.B + 1, dtype=torch.int32, device="cuda") * wl.N
         x_rows = x.view(wl.B * wl.N, d)

@@ -56,7 +56,8 @@ enum {
   HILO_ERR_WORKSPACE = -4,   /* workspace missing or smaller than required */
   HILO_ERR_TIMEOUT = -5,     /* a device-side bounded wait ran out (see hilo_sync_status) */
   HILO_ERR_UNSUPPORTED = -6, /* no sm_103a device, or a feature not built */
-  HILO_ERR_CHECK = -7        /* a device-side index check failed (checks build only) */
+  HILO_ERR_CHECK = -7        /* a device-side check failed: an index (checks build), or an
+                                image with more packed rows than the block supports */
 };
 
 /* Per-token labels written by hilo_split (HILO_LF: a non-kept token of the
@@ -310,7 +311,10 @@ size_t hilo_block_workspace_bytes(const hilo_shape* shape, int32_t cap);
  * sequence [its T text rows ; its packed image rows], scale 1/sqrt(head_dim).
  *   in_txt   [B*T, d] text rows,  dtype in_dtype (HILO_BF16 or HILO_F32)
  *   in_img   [cap, d] packed image rows, dtype in_dtype
- *   cu_img   int32 [B+1] device, from hilo_split
+ *   cu_img   int32 [B+1] device, from hilo_split. An image may hold at most
+ *            H*W (+ H*W/lf^2 with the low-frequency set) packed rows, as
+ *            hilo_split produces; an image with more is not attended in
+ *            full, and hilo_sync_status then returns HILO_ERR_CHECK.
  *   out      fp32 [B*T + cap, d]: the residual stream after the block, text
  *            rows first (row space). With in_dtype == HILO_F32, in-place use
  *            (in_txt == out, in_img == out + B*T*d) is allowed.
@@ -435,9 +439,11 @@ int hilo_block_forward_fp8(const hilo_shape* shape, const hilo_block_weights_fp8
  *     HILO_STATIC_SCRATCH_BYTES are rejected with HILO_ERR_WORKSPACE (the
  *     detail in hilo_last_error()); e.g. d=512, T=64, 1024 image rows fits,
  *     the d=3072 blocks do not;
- *   - the first call on a device looks up the array's device address (once
- *     per device, with that device current); make that first call before any
- *     stream capture;
+ *   - every call looks up the array's device address in the current device's
+ *     context (nothing is cached across calls, so a device reset or another
+ *     context is safe); the first call on a device also loads the library's
+ *     device code, so make it before any stream capture;
+ *   - an invalid shape returns HILO_ERR_SHAPE before any size check;
  *   - all calls share the one array: calls that overlap on the GPU (other
  *     streams, other host threads) race and must be serialised by the caller.
  *     No part of the array needs to start at zero.

@@ -205,6 +205,8 @@ bool encode_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t inner, uin
 // (for entry points defined in other files).
 int set_error(int status, const char* msg) { return fail(status, "%s", msg); }
 
+int check_block_shape(const hilo_shape* shape) { return check_shape(shape, true); }
+
 }  // namespace hilo
 
 extern "C" {
@@ -245,11 +247,17 @@ int hilo_sync_status(void* stream) {
   const int a = hilo::attn_take_device_error();
   const int pr = hilo::probe_take_device_error();
   const int dc = hilo::dcheck_take_bw();
-  if (g < 0 || g2 < 0 || a < 0 || pr < 0 || dc < 0)
+  const int ar = hilo::attn_take_rows_error();
+  if (g < 0 || g2 < 0 || a < 0 || pr < 0 || dc < 0 || ar < 0)
     return fail(HILO_ERR_CUDA, "hilo_sync_status: reading the device error word failed");
   if (g || g2 || a || pr)
     return fail(HILO_ERR_TIMEOUT, "device-side wait ran out (gemm=%d, gemm pair=%d, attention=%d, probe=%d)", g,
                 g2, a, pr);
+  if (ar)
+    return fail(HILO_ERR_CHECK,
+                "attention: image %d has more packed rows than H*W (+ H*W/lf^2); its extra rows were not "
+                "computed",
+                ar - 1);
   if (dc) return fail(HILO_ERR_CHECK, "device-side index check %d failed (checks build)", dc);
   return HILO_OK;
 }

@@ -49,6 +49,10 @@
 namespace hilo {
 
 __device__ int g_attn_err;
+// Set when an image has more packed rows than the launch's query tiles cover
+// (cu_img describes more than hilo_shape allows per image); those rows'
+// attention output would be left unwritten, so the call is reported failed.
+__device__ int g_attn_rows_err;
 
 namespace {
 
@@ -170,6 +174,7 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
   // image rows [cu_img[b], cu_img[b+1]) within the capacity
   const int L = min(p.cu_img[b + 1], p.cap) - min(p.cu_img[b], p.cap);
   const int nkv = p.qt_txt + (L + BKV - 1) / BKV;  // also the number of query tiles
+  if (pair == 0 && h == 0 && threadIdx.x == 0 && nkv > 2 * p.pairs_max) atomicExch(&g_attn_rows_err, b + 1);
   if (2 * pair >= nkv) return;                     // beyond this image's compressed length
   const bool has1 = 2 * pair + 1 < nkv;
   // the two query tiles (scalars: a runtime-indexed array would live in
@@ -668,6 +673,13 @@ int attn_take_device_error() {
   int v = 0, z = 0;
   if (cudaMemcpyFromSymbol(&v, g_attn_err, sizeof(int)) != cudaSuccess) return -1;
   if (v) cudaMemcpyToSymbol(g_attn_err, &z, sizeof(int));
+  return v;
+}
+
+int attn_take_rows_error() {
+  int v = 0, z = 0;
+  if (cudaMemcpyFromSymbol(&v, g_attn_rows_err, sizeof(int)) != cudaSuccess) return -1;
+  if (v) cudaMemcpyToSymbol(g_attn_rows_err, &z, sizeof(int));
   return v;
 }
 

@@ -6,6 +6,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include "../../include/hilo.h"
+
 #define HILO_LABEL_KEEP 0
 #define HILO_LABEL_POOL2 1
 #define HILO_LABEL_POOL4 2
@@ -108,6 +110,8 @@ struct AttnArgs {
 };
 cudaError_t launch_attention(const AttnArgs& a, int num_sms, cudaStream_t st);
 int attn_take_device_error();
+// 1 + the first image whose packed rows exceeded max_img_rows (0: none).
+int attn_take_rows_error();
 // The wait-timeout probe: one bounded mbarrier wait that runs out; its code
 // is read (and cleared) like the kernels' device error words.
 cudaError_t launch_wait_probe(cudaStream_t st);
@@ -117,6 +121,9 @@ int dcheck_take_bw();
 
 // ---- error text of the calling thread (api.cu)
 int set_error(int status, const char* msg);
+// The shape check of hilo_block_forward (HILO_OK, or the status it returns
+// with the calling thread's error text set).
+int check_block_shape(const hilo_shape* shape);
 
 // ---- tensor maps (api.cu): 2-D, row-major, 128-byte swizzled boxes
 enum TmapType : int { TMAP_BF16 = 0, TMAP_F16 = 1, TMAP_F32 = 2, TMAP_U8 = 3 };

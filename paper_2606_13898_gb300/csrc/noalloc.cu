@@ -20,10 +20,6 @@ namespace {
 // The shared scratch (one copy per device context).
 static __device__ __align__(256) unsigned char g_static_scratch[HILO_STATIC_SCRATCH_BYTES];
 
-constexpr int kMaxDevices = 64;
-// Device address of g_static_scratch per device ordinal (null until looked up).
-void* g_scratch_addr[kMaxDevices] = {};
-
 }  // namespace
 
 extern "C" int hilo_block_forward_static_ws(const hilo_shape* shape,
@@ -32,6 +28,9 @@ extern "C" int hilo_block_forward_static_ws(const hilo_shape* shape,
                                             const void* in_txt, const void* in_img,
                                             int in_dtype, float* out, void* stream) {
   if (!shape) return hilo::set_error(HILO_ERR_ARG, "hilo_block_forward_static_ws: shape is NULL");
+  // the shape first: the scratch size of an invalid shape means nothing
+  int st = hilo::check_block_shape(shape);
+  if (st) return st;
   if (cap < 0) return hilo::set_error(HILO_ERR_ARG, "hilo_block_forward_static_ws: cap < 0");
   const size_t need = hilo_block_workspace_bytes(shape, cap);
   if (need > HILO_STATIC_SCRATCH_BYTES) {
@@ -42,20 +41,17 @@ extern "C" int hilo_block_forward_static_ws(const hilo_shape* shape,
              need, static_cast<size_t>(HILO_STATIC_SCRATCH_BYTES));
     return hilo::set_error(HILO_ERR_WORKSPACE, msg);
   }
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
-    return hilo::set_error(HILO_ERR_CUDA, "hilo_block_forward_static_ws: no current device");
-  if (!g_scratch_addr[dev]) {
-    // One-time set-up per device, with that device current: the host-side
-    // name g_static_scratch is not a device address; ask the runtime for it.
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || !p)
-      return hilo::set_error(HILO_ERR_CUDA,
-                             "hilo_block_forward_static_ws: cudaGetSymbolAddress of the scratch failed");
-    g_scratch_addr[dev] = p;
-  }
+  // The host-side name g_static_scratch is not a device address: ask the
+  // runtime for the array's address in the current device's context, on
+  // every call, so that nothing cached can outlive that context (a device
+  // reset, another context on the same device). The first call on a device
+  // also loads the module; make it before any stream capture.
+  void* scratch = nullptr;
+  if (cudaGetSymbolAddress(&scratch, g_static_scratch) != cudaSuccess || !scratch)
+    return hilo::set_error(HILO_ERR_CUDA,
+                           "hilo_block_forward_static_ws: cudaGetSymbolAddress of the scratch failed");
   // Nothing in the scratch needs to start at zero: every scratch value the
   // block's kernels read was written earlier in the same call.
   return hilo_block_forward(shape, weights, cu_img, cap, in_txt, in_img, in_dtype, out,
-                            g_scratch_addr[dev], HILO_STATIC_SCRATCH_BYTES, stream);
+                            scratch, HILO_STATIC_SCRATCH_BYTES, stream);
 }

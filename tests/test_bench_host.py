@@ -56,3 +56,23 @@ def test_clock_sampler_without_nvidia_smi(monkeypatch, tmp_path):
     c = bench.ClockSampler(0)
     c.start()
     assert c.stop() is None
+
+
+def test_reference_arm_reports_the_gpu_arms_config(monkeypatch, capsys):
+    # The reference arm (the oracle on the host) must describe the same
+    # workload as the GPU arm: identical config keys and values, including
+    # the packed row count of the workload's split. The oracle's steps are
+    # stubbed out here; only the line is checked.
+    import json
+    monkeypatch.setattr(bench, "oracle_step", lambda sample: None)
+    monkeypatch.setattr(bench, "oracle_sample", lambda ratio, crop, seed_offset=0: (None, I.make_batch(
+        I.tiny_layer()).x, None, None, None, None, None, 8))
+    for v in ("RANK", "WORLD_SIZE", "LOCAL_RANK"):
+        monkeypatch.delenv(v, raising=False)
+    bench.run_reference(bench.parse(["--impl", "reference", "--steps", "1", "--warmup", "0"]))
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["impl"] == "reference"
+    wl = bench.workload("1/4")
+    gpu_cfg = bench.line_config(wl, "1/4", line["config"]["packed_image_rows"], 1)
+    assert line["config"] == gpu_cfg
+    assert line["config"]["packed_image_rows"] == 1877 and line["config"]["block_rows"] == 2389

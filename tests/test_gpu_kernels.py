@@ -313,6 +313,30 @@ def test_block_forward_fp32_in_place_chain(H):
     assert_block_close(got[B * T:], i2, "image rows")
 
 
+def test_block_rejects_image_longer_than_grid(H):
+    # An image may hold at most H*W packed rows (what hilo_split produces).
+    # cu_img is device data, so a longer image is only seen on the device:
+    # the call must report HILO_ERR_CHECK instead of leaving rows unattended.
+    rng = np.random.default_rng(5)
+    d, heads, T = 128, 1, 0
+    lens = [300, 20]                      # image 0: 300 rows on an 8x8 grid (64 tokens)
+    B = len(lens)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    cap = int(cu[-1]) + 16
+    sh = H.Shape(B=B, H=8, W=8, d=d, T=T, heads=heads, mlp=0)
+    ui = bits(rng.standard_normal((cap, d)))
+    out = torch.empty(cap, d, dtype=torch.float32, device="cuda")
+    wsb = H.hilo_block_workspace_bytes(sh, cap)
+    ws = torch.empty(wsb, dtype=torch.uint8, device="cuda")
+    H.hilo_block_forward(sh, H.DeviceWeights.from_host(scaled_weights(rng, d, False, 1.0 / np.sqrt(d))),
+                         to_dev_i32(cu), cap, None, H.bf16_from_bits(ui), H.HILO_BF16, out, ws, wsb)
+    with pytest.raises(H.HiloError) as e:
+        H.hilo_sync_status()
+    assert e.value.status == -7
+    assert "image 0" in H.lib().hilo_last_error().decode()
+    H.hilo_sync_status()                  # read once, then cleared
+
+
 def test_host_argument_errors(H):
     sh = H.Shape(B=1, H=8, W=8, d=128, T=0, heads=1, mlp=0)
     s = torch.empty(64, dtype=torch.float32, device="cuda")

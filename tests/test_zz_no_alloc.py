@@ -36,6 +36,16 @@ def _case(H, seed, lens, d=512, heads=8, T=64, mlp=1):
 def test_static_scratch_matches_workspace_entry_twice():
     H = lib_ready()
     cases = [_case(H, 5, [700]), _case(H, 6, [300, 1000])]
+    # First fill the shared array with NaN: a call whose inputs are all NaN
+    # leaves NaN in every scratch region it writes. A kernel that read a
+    # scratch value before writing it in the same call would then turn the
+    # real cases below non-finite.
+    sh, dw, cu, cap, t_in, i_in = cases[1]
+    poison = torch.empty(sh.B * sh.T + cap, sh.d, dtype=torch.float32, device="cuda")
+    H.hilo_block_forward_static_ws(sh, dw, cu, cap, torch.full_like(t_in, float("nan")),
+                                   torch.full_like(i_in, float("nan")), H.HILO_BF16, poison)
+    H.hilo_sync_status()
+    assert torch.isnan(poison[:sh.B * sh.T + int(cu[-1].item())]).all()
     for sh, dw, cu, cap, t_in, i_in in cases:
         ws_bytes = H.hilo_block_workspace_bytes(sh, cap)
         assert ws_bytes <= 16 << 20
@@ -60,3 +70,8 @@ def test_static_scratch_rejects_oversized_shape():
         H.hilo_block_forward_static_ws(sh, dw, dummy, 4096, dummy, dummy, H.HILO_BF16, dummy)
     assert e.value.status == -4
     assert "scratch bytes" in H.lib().hilo_last_error().decode()
+    # an invalid shape is reported as such, not as a scratch size
+    bad = H.Shape(B=1, H=8, W=8, d=-128, T=8, heads=1, mlp=1)
+    with pytest.raises(H.HiloError) as e:
+        H.hilo_block_forward_static_ws(bad, dw, dummy, 64, dummy, dummy, H.HILO_BF16, dummy)
+    assert e.value.status == -2
