@@ -585,7 +585,7 @@ def oracle_config_baseline(wl, batch, host_weights) -> dict:
         el += time.perf_counter() - t0
         del w
     t0 = time.perf_counter()
-    O.update(x, O.unpack(ui, sp), 0.035)
+    O.update(x, O.unpack(ui, sp).reshape(x.shape), 0.035)
     el += time.perf_counter() - t0
     return {"value": wl.B * wl.N / el, "unit": UNIT, "cores": host_cores(), "kind": "oracle",
             "seconds_per_step": el, "seconds_28_steps_extrapolated": 28 * el,

@@ -76,3 +76,17 @@ def test_reference_arm_reports_the_gpu_arms_config(monkeypatch, capsys):
     gpu_cfg = bench.line_config(wl, "1/4", line["config"]["packed_image_rows"], 1)
     assert line["config"] == gpu_cfg
     assert line["config"]["packed_image_rows"] == 1877 and line["config"]["block_rows"] == 2389
+
+
+def test_oracle_config_baseline_single_and_multi_block():
+    # The per-configuration oracle timing runs the oracle's own hot path: a
+    # single block in one pass, and a stack of blocks one timed step at a
+    # time (extrapolated to 28 steps). Tiny 32x32 layers keep it quick.
+    wl = I.tiny_layer()
+    b = I.make_batch(wl)
+    ws = [I.make_weights(wl.d, wl.mlp, seed=I.weight_seed(wl, i)) for i in range(2)]
+    one = bench.oracle_config_baseline(wl, b, ws[:1])
+    assert one["kind"] == "oracle" and one["value"] > 0 and one["cores"] >= 1
+    two = bench.oracle_config_baseline(wl, b, ws)
+    assert two["value"] > 0
+    assert two["seconds_28_steps_extrapolated"] == 28 * two["seconds_per_step"]
