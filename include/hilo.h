@@ -56,8 +56,7 @@ enum {
   HILO_ERR_WORKSPACE = -4,   /* workspace missing or smaller than required */
   HILO_ERR_TIMEOUT = -5,     /* a device-side bounded wait ran out (see hilo_sync_status) */
   HILO_ERR_UNSUPPORTED = -6, /* no sm_103a device, or a feature not built */
-  HILO_ERR_CHECK = -7        /* a device-side check failed: an index (checks build), or an
-                                image with more packed rows than the block supports */
+  HILO_ERR_CHECK = -7        /* a device-side index check failed (checks build only) */
 };
 
 /* Per-token labels written by hilo_split (HILO_LF: a non-kept token of the
@@ -311,10 +310,8 @@ size_t hilo_block_workspace_bytes(const hilo_shape* shape, int32_t cap);
  * sequence [its T text rows ; its packed image rows], scale 1/sqrt(head_dim).
  *   in_txt   [B*T, d] text rows,  dtype in_dtype (HILO_BF16 or HILO_F32)
  *   in_img   [cap, d] packed image rows, dtype in_dtype
- *   cu_img   int32 [B+1] device, from hilo_split. An image may hold at most
- *            H*W (+ H*W/lf^2 with the low-frequency set) packed rows, as
- *            hilo_split produces; an image with more is not attended in
- *            full, and hilo_sync_status then returns HILO_ERR_CHECK.
+ *   cu_img   int32 [B+1] device, from hilo_split (any non-decreasing
+ *            offsets: rows past cap are not part of the block).
  *   out      fp32 [B*T + cap, d]: the residual stream after the block, text
  *            rows first (row space). With in_dtype == HILO_F32, in-place use
  *            (in_txt == out, in_img == out + B*T*d) is allowed.

@@ -247,17 +247,11 @@ int hilo_sync_status(void* stream) {
   const int a = hilo::attn_take_device_error();
   const int pr = hilo::probe_take_device_error();
   const int dc = hilo::dcheck_take_bw();
-  const int ar = hilo::attn_take_rows_error();
-  if (g < 0 || g2 < 0 || a < 0 || pr < 0 || dc < 0 || ar < 0)
+  if (g < 0 || g2 < 0 || a < 0 || pr < 0 || dc < 0)
     return fail(HILO_ERR_CUDA, "hilo_sync_status: reading the device error word failed");
   if (g || g2 || a || pr)
     return fail(HILO_ERR_TIMEOUT, "device-side wait ran out (gemm=%d, gemm pair=%d, attention=%d, probe=%d)", g,
                 g2, a, pr);
-  if (ar)
-    return fail(HILO_ERR_CHECK,
-                "attention: image %d has more packed rows than H*W (+ H*W/lf^2); its extra rows were not "
-                "computed",
-                ar - 1);
   if (dc) return fail(HILO_ERR_CHECK, "device-side index check %d failed (checks build)", dc);
   return HILO_OK;
 }
@@ -463,7 +457,6 @@ static int block_forward_impl(const hilo_shape* shape, const hilo_block_weights*
   aa.head_dim = d / shape->heads;
   aa.d = d;
   aa.R = R;
-  aa.max_img_rows = static_cast<int>(hilo_row_capacity(shape) / shape->B);
   e = hilo::launch_attention(aa, dev->num_sms, s);
   if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward: attention");
   count(1);
@@ -621,7 +614,6 @@ int hilo_block_forward_fp8(const hilo_shape* shape, const hilo_block_weights_fp8
   aa.head_dim = d / shape->heads;
   aa.d = d;
   aa.R = R;
-  aa.max_img_rows = static_cast<int>(hilo_row_capacity(shape) / shape->B);
   e = hilo::launch_attention(aa, dev->num_sms, s);
   if (e != cudaSuccess) return cuda_fail(e, "hilo_block_forward_fp8: attention");
   count(1);

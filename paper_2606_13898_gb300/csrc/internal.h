@@ -106,12 +106,10 @@ struct AttnArgs {
   void* out;        // bf16 [R, d]
   const int32_t* cu_img;
   const float* n_img = nullptr;  // proportional attention: weight per packed image row
-  int B, T, heads, head_dim, d, R, max_img_rows;
+  int B, T, heads, head_dim, d, R;
 };
 cudaError_t launch_attention(const AttnArgs& a, int num_sms, cudaStream_t st);
 int attn_take_device_error();
-// 1 + the first image whose packed rows exceeded max_img_rows (0: none).
-int attn_take_rows_error();
 // The wait-timeout probe: one bounded mbarrier wait that runs out; its code
 // is read (and cleared) like the kernels' device error words.
 cudaError_t launch_wait_probe(cudaStream_t st);
