@@ -48,8 +48,10 @@ def parse(argv=None):
     ap.add_argument("--impl", choices=["hilo", "reference"], default="hilo")
     ap.add_argument("--ratio", default="1/4", help="keep ratio of the timed workload")
     ap.add_argument("--no-extras", action="store_true", help="skip sweep / dense / e2e / cpu_baseline")
-    ap.add_argument("--variant", choices=["bf16", "fp8"], default="bf16",
-                    help="fp8: the timed step's blocks take e4m3 GEMM operands (no extras)")
+    ap.add_argument("--variant", choices=["bf16", "fp8", "regions", "lf", "prop"], default="bf16",
+                    help="fp8: the timed step's blocks take e4m3 GEMM operands (no extras); regions: the "
+                         "window-granular split and delta unpool; lf: the separate low-frequency set (lf = 4); "
+                         "prop: proportional attention (these three: the step's time only)")
     return ap.parse_args(argv)
 
 
@@ -507,9 +509,9 @@ def time_torch_context(H, torch, stream, wl, hp, dw, inputs, steps: int) -> dict
         torch.cuda.synchronize()
         return a.elapsed_time(b_) / steps
 
-    cu_d = hp.split.cu_img
-    ours = timed(lambda: H.hilo_block_forward(sh, dw, cu_d, hp.cap, text, hp.packed, H.HILO_BF16, hp.out, hp.ws,
-                                              hp.ws_bytes, stream))
+    # this library's block on the same rows, issued exactly as the dense
+    # comparison issues it (HotPath.blocks)
+    ours = timed(lambda: hp.blocks(text, hp.packed, H.HILO_BF16))
     ref = timed(block)
     # agreement of the two on these rows (both against the same bf16 inputs)
     diff = (block() - hp.out[:Rt + L]).abs().max().item()
@@ -751,6 +753,56 @@ def time_configs(H, I, torch, stream, steps: int, bf16_peak: float, peak_src: st
     return res
 
 
+def run_mode_variant(args, H, torch, stream, wl, batch, sh, dw, rank, world, local, barrier, max_over_ranks):
+    """The timed step in one of the optional modes of the path: the
+    window-granular split with the delta unpool (regions), the separate
+    low-frequency token set with lf = 4 (lf), or proportional attention
+    (prop). Reports the step's time; the per-kernel breakdown and the extras
+    belong to the default variant."""
+    import dataclasses
+    from paper_2606_13898_gb300 import replicas
+    mode = args.variant
+    if mode == "lf":
+        sh = dataclasses.replace(sh, lf=4)
+    hp = H.HotPath(sh, [dw])
+    x, text = H.bf16_from_bits(batch.x), H.bf16_from_bits(batch.text)
+    mask, kk, km = (torch.from_numpy(batch.mask).cuda(), torch.from_numpy(batch.k_keep).cuda(),
+                    torch.from_numpy(batch.k_mid).cuda())
+    kw = {"regions": mode == "regions", "prop": mode == "prop"}
+    for _ in range(max(3, args.warmup)):
+        hp.run(x, text, mask, kk, km, **kw)
+    H.hilo_sync_status()
+    rows = int(hp.split.cu_img[-1].item())
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    n0 = H.hilo_launch_count()
+    clocks = ClockSampler(local)
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    time.sleep(0.3)
+    start.record(stream)
+    for _ in range(args.steps):
+        hp.run(x, text, mask, kk, km, **kw)
+    end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    barrier()
+    launches = H.hilo_launch_count() - n0
+    H.hilo_sync_status()
+    ms_total = max_over_ranks(start.elapsed_time(end))
+    N = wl.B * wl.N
+    cfg = line_config(wl, args.ratio, rows, world)
+    cfg["workload"] = f"{wl.name}_{mode}"
+    cfg["mode"] = {"regions": "window-granular split, delta unpool", "lf": "separate low-frequency set, lf = 4",
+                   "prop": "proportional attention"}[mode]
+    line = {"metric": METRIC, "value": replicas.whole_job_throughput(N * args.steps, world, ms_total), "unit": UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_total / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": DTYPE_BF16,
+            "data": "synthetic", "config": cfg, "variant": mode, "gpu_launches": int(launches), "clocks": clk}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
 def run_hilo(args):
     import torch
     import torch.distributed as dist
@@ -792,6 +844,11 @@ def run_hilo(args):
     fp8 = args.variant == "fp8"
     if fp8:
         hp.enable_fp8([H.DeviceWeightsFP8.from_host(w)])
+    if args.variant in ("regions", "lf", "prop"):
+        run_mode_variant(args, H, torch, stream, wl, batch, sh, dw, rank, world, local, barrier, max_over_ranks)
+        if world > 1:
+            dist.destroy_process_group()
+        return
 
     def dev_inputs(b):
         return (H.bf16_from_bits(b.x), H.bf16_from_bits(b.text), torch.from_numpy(b.mask).cuda(),
