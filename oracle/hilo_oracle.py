@@ -610,7 +610,7 @@ def f32_to_f16_sat(a) -> np.ndarray:
     return a.astype(np.float32).astype(np.float16).astype(np.float64)
 
 
-def block_fp8(u_txt, u_img, cu_img, T: int, weights_q, heads: int, mlp: bool):
+def block_fp8(u_txt, u_img, cu_img, T: int, weights_q, heads: int, mlp: bool, n_img=None):
     """The MMDiT block of ``block`` with e4m3 GEMM operands, in the order the
     kernels take: LayerNorm -> fp32 -> per-row e4m3; QKV = (codes_A codes_W^T)
     * scale_A[r] * scale_W[o] + b, rounded to bf16; attention (fp64) rounded
@@ -618,7 +618,8 @@ def block_fp8(u_txt, u_img, cu_img, T: int, weights_q, heads: int, mlp: bool):
     MLP1 -> GELU rounded to fp16 -> per-row e4m3 -> MLP2. The residual stream
     stays fp64 here (fp32 in the kernels). ``weights_q`` per stream holds
     (codes, scale) for w_qkv, w_o, w_1, w_2 (see quantize_weights) and the
-    bf16 biases. Returns fp64 (txt, img).
+    bf16 biases. n_img (optional): proportional attention, as in ``block``.
+    Returns fp64 (txt, img).
 
     Paper: Sec. 3.3 (FP8 on top of HiLo-Token) applied to the Sec. 2.1 block."""
     ut = _as_f64(u_txt)
@@ -636,10 +637,11 @@ def block_fp8(u_txt, u_img, cu_img, T: int, weights_q, heads: int, mlp: bool):
         t0, t1 = b * T, (b + 1) * T
         i0, i1 = int(cu_img[b]), int(cu_img[b + 1])
         joint = np.concatenate([qkv[0][t0:t1], qkv[1][i0:i1]], axis=0)
+        kn = None if n_img is None else np.concatenate([np.ones(T), np.asarray(n_img[i0:i1], np.float64)])
         o = np.empty((joint.shape[0], d))
         for h in range(heads):
             c = slice(h * hd, (h + 1) * hd)
-            o[:, c] = softmax_attention(joint[:, c], joint[:, d:][:, c], joint[:, 2 * d:][:, c])
+            o[:, c] = softmax_attention(joint[:, c], joint[:, d:][:, c], joint[:, 2 * d:][:, c], kn)
         att[0][t0:t1] = o[:T]
         att[1][i0:i1] = o[T:]
     out = []
@@ -657,11 +659,12 @@ def block_fp8(u_txt, u_img, cu_img, T: int, weights_q, heads: int, mlp: bool):
 
 
 def block_rows_fp8(u_txt, u_img, cu_img, T: int, weights_q, heads: int, mlp: bool, b: int, txt_rows,
-                   img_rows):
+                   img_rows, n_img=None):
     """block_fp8's outputs for selected rows of image ``b`` only: keys and
     values of the whole joint sequence of image b (each row's quantisation
     depends on that row alone), queries, attention, out-projection and MLP
-    for the given rows (absolute row ids in u_txt / u_img). fp64 (txt, img).
+    for the given rows (absolute row ids in u_txt / u_img). n_img as in
+    block_fp8. fp64 (txt, img).
 
     Paper: Sec. 3.3, as block_fp8."""
     ut = _as_f64(u_txt)
@@ -682,6 +685,7 @@ def block_rows_fp8(u_txt, u_img, cu_img, T: int, weights_q, heads: int, mlp: boo
 
     kv = np.concatenate([qkv_part(ut[t0:t1], wt, d, 3 * d) if t1 > t0 else np.zeros((0, 2 * d)),
                          qkv_part(ui[i0:i1], wi, d, 3 * d) if i1 > i0 else np.zeros((0, 2 * d))], axis=0)
+    kn = None if n_img is None else np.concatenate([np.ones(t1 - t0), np.asarray(n_img[i0:i1], np.float64)])
     res = []
     for rows, u_all, w in ((np.asarray(txt_rows, int), ut, wt), (np.asarray(img_rows, int), ui, wi)):
         if rows.size == 0:
@@ -692,7 +696,7 @@ def block_rows_fp8(u_txt, u_img, cu_img, T: int, weights_q, heads: int, mlp: boo
         o = np.empty((len(rows), d))
         for h in range(heads):
             c = slice(h * hd, (h + 1) * hd)
-            o[:, c] = softmax_attention(q[:, c], kv[:, :d][:, c], kv[:, d:][:, c])
+            o[:, c] = softmax_attention(q[:, c], kv[:, :d][:, c], kv[:, d:][:, c], kn)
         a16 = bf16_to_f32(f32_to_bf16(o)).astype(np.float64)
         u = u + gemm_e4m3(a16, w.w_o, w.b_o)
         if mlp:

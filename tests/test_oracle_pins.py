@@ -847,6 +847,59 @@ def test_block_rows_fp8_matches_block_fp8():
     assert np.allclose(ri, fi[[9, 15, 22]], rtol=0, atol=1e-12)
 
 
+def _fp8_weights(rng, d):
+    std = 1 / np.sqrt(d)
+
+    def one():
+        s = I.StreamWeights(w_qkv=bits(rng.normal(0, std, (3 * d, d))), b_qkv=bits(rng.normal(0, std, 3 * d)),
+                            w_o=bits(rng.normal(0, std, (d, d))), b_o=bits(rng.normal(0, std, d)))
+        s.w_1, s.b_1 = bits(rng.normal(0, std, (4 * d, d))), bits(rng.normal(0, std, 4 * d))
+        s.w_2, s.b_2 = bits(rng.normal(0, std / 2, (d, 4 * d))), bits(rng.normal(0, std, d))
+        return s
+    return O.quantize_weights(I.BlockWeights(txt=one(), img=one()))
+
+
+def test_block_fp8_proportional_ones_is_plain_fp8_block():
+    """Row weights of one add ln 1 = 0 to every logit: the FP8 block with
+    proportional attention is then the plain FP8 block, bit for bit."""
+    rng = np.random.default_rng(34)
+    d, heads, T = 64, 2, 4
+    wq = _fp8_weights(rng, d)
+    ut = bits(rng.standard_normal((2 * T, d)))
+    ui = bits(rng.standard_normal((13, d)))
+    cu = [0, 6, 13]
+    a = O.block_fp8(ut, ui, cu, T, wq, heads, True)
+    b = O.block_fp8(ut, ui, cu, T, wq, heads, True, n_img=np.ones(13, np.float32))
+    assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
+
+
+def test_block_fp8_proportional_equals_fp8_block_on_duplicated_rows():
+    """The FP8 block with row weights n equals the plain FP8 block on the
+    sequence where image row r appears n_r times: every row's quantisation
+    depends on that row alone, so the copies carry the same codes and the
+    softmax over n copies of a key is the weighted one. Checked on the text
+    rows and the first copy of each image row, and through block_rows_fp8."""
+    rng = np.random.default_rng(35)
+    d, heads, T = 64, 2, 3
+    wq = _fp8_weights(rng, d)
+    ut = bits(rng.standard_normal((2 * T, d)))
+    ui = bits(rng.standard_normal((9, d)))
+    cu = [0, 5, 9]
+    n = np.array([1, 3, 1, 2, 4, 2, 1, 1, 3], dtype=np.float32)
+    pt, pi = O.block_fp8(ut, ui, cu, T, wq, heads, True, n_img=n)
+    rep = np.repeat(np.arange(9), n.astype(int))
+    cu_dup = [0, int(n[:5].sum()), int(n.sum())]
+    dt, di = O.block_fp8(ut, ui[rep], cu_dup, T, wq, heads, True)
+    first = np.searchsorted(rep, np.arange(9))
+    assert np.allclose(pt, dt, rtol=0, atol=1e-9)
+    assert np.allclose(pi, di[first], rtol=0, atol=1e-9)
+    # the weights matter: the plain FP8 block differs
+    qt, qi = O.block_fp8(ut, ui, cu, T, wq, heads, True)
+    assert np.abs(qi - pi).max() > 1e-3
+    rt, ri = O.block_rows_fp8(ut, ui, cu, T, wq, heads, True, 1, [3, 5], [6, 8], n_img=n)
+    assert np.allclose(rt, pt[[3, 5]], rtol=0, atol=1e-12) and np.allclose(ri, pi[[6, 8]], rtol=0, atol=1e-12)
+
+
 def test_keep_ratio_one_is_dense_block():
     wl = I.tiny_layer(keep_ratio=1024, H=16, W=16, d=64, heads=2, T=8)
     b = I.make_batch(wl)
