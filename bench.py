@@ -548,6 +548,10 @@ def time_fp8(H, I, torch, stream, wl, hp, inputs, bf16_peak: float, steps: int) 
                                                 hp.ws_bytes, stream))
     b16 = timed(lambda: H.hilo_block_forward(sh, hp.weights[0], cu, hp.cap, text, hp.packed, H.HILO_BF16, hp.out,
                                              hp.ws, hp.ws_bytes, stream))
+    # proportional attention inside the FP8 block (row sizes from the split)
+    path_prop_ms = timed(lambda: hp.run(x, text, mask, kk, km, fp8=True, prop=True))
+    b8p = timed(lambda: H.hilo_block_forward_fp8_prop(sh, w8, cu, hp.cap, text, hp.packed, H.HILO_BF16, hp.n_img,
+                                                      hp.out, hp.ws, hp.ws_bytes, stream))
     # per-stage times of the FP8 block (the bf16 block's stage marks)
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(8)]
     for e in ev:
@@ -568,6 +572,8 @@ def time_fp8(H, I, torch, stream, wl, hp, inputs, bf16_peak: float, steps: int) 
     tflops = 24.0 * M * d * d / (gemm_ms * 1e-3) / 1e12
     return {"block_ms_fp8": b8, "block_ms_bf16_same_rows": b16, "block_speedup": b16 / b8,
             "hot_path_ms": path_ms, "image_tokens_per_s": wl.B * wl.N / (path_ms * 1e-3),
+            "proportional_attention": {"block_ms_fp8_prop": b8p, "hot_path_ms": path_prop_ms,
+                                       "block_overhead_vs_fp8": b8p / b8 - 1.0},
             "stage_ms": {"ln1": st[0], "qkv": st[1], "attention_and_quant": st[2], "out_proj": st[3],
                          "ln2": st[4], "mlp1_and_quant": st[5], "mlp2": st[6]},
             "gemm_TFLOP/s_incl_hidden_quant": tflops,

@@ -422,6 +422,21 @@ int hilo_block_forward_fp8(const hilo_shape* shape, const hilo_block_weights_fp8
                            int in_dtype, float* out, void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * hilo_block_forward_fp8_prop -- hilo_block_forward_fp8 with the proportional
+ * attention of hilo_block_forward_prop: as a key, packed image row r adds
+ * ln(n_img[r]) to its logits (text keys add 0), the kernel multiplying each
+ * probability by n_img[r] before the row sum and the bf16 rounding of P.
+ * The paper gives neither FP8 scheme nor pooled-token attention (Sec. 3.3,
+ * Sec. 2.3); both are this library's readings. n_img: fp32 [cap] device,
+ * 4-byte aligned, from hilo_row_sizes. Other arguments, layouts and errors
+ * as hilo_block_forward_fp8.
+ */
+int hilo_block_forward_fp8_prop(const hilo_shape* shape, const hilo_block_weights_fp8* weights,
+                                const int32_t* cu_img, int32_t cap, const void* in_txt, const void* in_img,
+                                int in_dtype, const float* n_img, float* out, void* ws, size_t ws_bytes,
+                                void* stream);
+
+/*
  * hilo_block_forward_static_ws -- hilo_block_forward without a workspace
  * argument, for callers that cannot allocate device memory at call time (code
  * inside a host framework whose allocator the call site cannot reach, or a

@@ -524,9 +524,12 @@ size_t hilo_block_fp8_workspace_bytes(const hilo_shape* shape, int32_t cap) {
   return block_fp8_ws_layout(shape, cap).total;
 }
 
-int hilo_block_forward_fp8(const hilo_shape* shape, const hilo_block_weights_fp8* w, const int32_t* cu_img,
-                           int32_t cap, const void* in_txt, const void* in_img, int in_dtype, float* out,
-                           void* ws, size_t ws_bytes, void* stream) {
+// The block of hilo_block_forward_fp8; n_img != NULL selects proportional
+// attention (hilo_block_forward_fp8_prop).
+static int block_forward_fp8_impl(const hilo_shape* shape, const hilo_block_weights_fp8* w,
+                                  const int32_t* cu_img, int32_t cap, const void* in_txt, const void* in_img,
+                                  int in_dtype, const float* n_img, float* out, void* ws, size_t ws_bytes,
+                                  void* stream) {
   int st = check_shape(shape, true);
   if (st) return st;
   if (shape->d < 1024 || shape->d % 256)
@@ -608,6 +611,7 @@ int hilo_block_forward_fp8(const hilo_shape* shape, const hilo_block_weights_fp8
   aa.qkv = qkv;
   aa.out = attn;
   aa.cu_img = cu_img;
+  aa.n_img = n_img;
   aa.B = B;
   aa.T = T;
   aa.heads = shape->heads;
@@ -642,6 +646,23 @@ int hilo_block_forward_fp8(const hilo_shape* shape, const hilo_block_weights_fp8
     stage_mark(7, s);
   }
   return HILO_OK;
+}
+
+int hilo_block_forward_fp8(const hilo_shape* shape, const hilo_block_weights_fp8* w, const int32_t* cu_img,
+                           int32_t cap, const void* in_txt, const void* in_img, int in_dtype, float* out,
+                           void* ws, size_t ws_bytes, void* stream) {
+  return block_forward_fp8_impl(shape, w, cu_img, cap, in_txt, in_img, in_dtype, nullptr, out, ws, ws_bytes,
+                                stream);
+}
+
+int hilo_block_forward_fp8_prop(const hilo_shape* shape, const hilo_block_weights_fp8* w, const int32_t* cu_img,
+                                int32_t cap, const void* in_txt, const void* in_img, int in_dtype,
+                                const float* n_img, float* out, void* ws, size_t ws_bytes, void* stream) {
+  if (!n_img) return fail(HILO_ERR_ARG, "hilo_block_forward_fp8_prop: n_img is NULL");
+  if (reinterpret_cast<uintptr_t>(n_img) & 3)
+    return fail(HILO_ERR_ARG, "hilo_block_forward_fp8_prop: n_img must be 4-byte aligned");
+  return block_forward_fp8_impl(shape, w, cu_img, cap, in_txt, in_img, in_dtype, n_img, out, ws, ws_bytes,
+                                stream);
 }
 
 int hilo_row_sizes(const hilo_shape* shape, const hilo_split_out* split, float* n_img, int32_t cap,

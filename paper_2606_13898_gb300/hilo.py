@@ -68,7 +68,7 @@ EXPORTS = ("hilo_status_string", "hilo_last_error", "hilo_sync_status", "hilo_de
            "hilo_block_forward_static_ws", "hilo_sobel_workspace_bytes", "hilo_sobel_select",
            "hilo_split_regions", "hilo_unpack_delta", "hilo_row_sizes", "hilo_block_forward_prop",
            "hilo_row_capacity", "hilo_quantize_rows_e4m3", "hilo_block_fp8_workspace_bytes",
-           "hilo_block_forward_fp8", "hilo_debug_wait_timeout")
+           "hilo_block_forward_fp8", "hilo_block_forward_fp8_prop", "hilo_debug_wait_timeout")
 
 _lib = None
 
@@ -120,6 +120,8 @@ def lib() -> ctypes.CDLL:
         "hilo_block_fp8_workspace_bytes": (S, [shp, ctypes.c_int32]),
         "hilo_block_forward_fp8": (I, [shp, ctypes.POINTER(hilo_block_weights_fp8), P, ctypes.c_int32, P, P, I,
                                        P, P, S, P]),
+        "hilo_block_forward_fp8_prop": (I, [shp, ctypes.POINTER(hilo_block_weights_fp8), P, ctypes.c_int32, P, P,
+                                            I, P, P, P, S, P]),
         "hilo_block_forward_prop": (I, [shp, ctypes.POINTER(hilo_block_weights), P, ctypes.c_int32, P, P, I,
                                         P, P, P, S, P]),
     }
@@ -391,6 +393,15 @@ def hilo_block_forward_fp8(shape: Shape, weights: DeviceWeightsFP8, cu_img, cap:
         _ptr(ws), ws_bytes, _stream(stream)))
 
 
+def hilo_block_forward_fp8_prop(shape: Shape, weights: DeviceWeightsFP8, cu_img, cap: int, in_txt, in_img,
+                                in_dtype: int, n_img, out, ws, ws_bytes: int, stream=None) -> None:
+    s = shape.c()
+    w = weights.c()
+    _check("hilo_block_forward_fp8_prop", lib().hilo_block_forward_fp8_prop(
+        ctypes.byref(s), ctypes.byref(w), _ptr(cu_img), cap, _ptr(in_txt), _ptr(in_img), in_dtype, _ptr(n_img),
+        _ptr(out), _ptr(ws), ws_bytes, _stream(stream)))
+
+
 def hilo_row_sizes(shape: Shape, split: SplitBuffers, n_img, cap: int, stream=None) -> None:
     s = shape.c()
     o = split.c()
@@ -501,9 +512,7 @@ class HotPath:
         if prop:
             hilo_row_sizes(sh, self.split, self.n_img, self.cap, stream)
         if fp8:
-            if prop:
-                raise ValueError("proportional attention has no FP8 block")
-            self.blocks_fp8(text, self.packed, HILO_BF16, stream)
+            self.blocks_fp8(text, self.packed, HILO_BF16, stream, self.n_img if prop else None)
         else:
             self.blocks(text, self.packed, HILO_BF16, stream, self.n_img if prop else None)
         if unpack:
@@ -514,12 +523,16 @@ class HotPath:
             else:
                 hilo_unpack(sh, self.out_img, self.split, self.y, stream)
 
-    def blocks_fp8(self, in_txt, in_img, in_dtype, stream=None) -> None:
+    def blocks_fp8(self, in_txt, in_img, in_dtype, stream=None, n_img=None) -> None:
         sh = self.shape
         for i, w in enumerate(self.weights_fp8):
             args = (in_txt, in_img, in_dtype) if i == 0 else (self.out, self.out_img, HILO_F32)
-            hilo_block_forward_fp8(sh, w, self.split.cu_img, self.cap, *args, self.out, self.ws, self.ws_bytes,
-                                   stream)
+            if n_img is None:
+                hilo_block_forward_fp8(sh, w, self.split.cu_img, self.cap, *args, self.out, self.ws, self.ws_bytes,
+                                       stream)
+            else:
+                hilo_block_forward_fp8_prop(sh, w, self.split.cu_img, self.cap, *args, n_img, self.out, self.ws,
+                                            self.ws_bytes, stream)
 
     def blocks(self, in_txt, in_img, in_dtype, stream=None, n_img=None) -> None:
         sh = self.shape

@@ -153,3 +153,50 @@ def test_block_forward_fp8_against_oracle(H, d, heads, T, lens):
         e_ex = np.linalg.norm(got - ex) / delta
         assert e_emu < 0.03, e_emu
         assert 0.005 < e_ex < 0.1, e_ex
+
+
+@pytest.mark.parametrize("d,heads,T,lens", [
+    (1024, 8, 64, [300, 77]),
+    (2048, 16, 128, [400]),
+])
+def test_block_forward_fp8_prop_against_oracle(H, d, heads, T, lens):
+    """Proportional attention in the FP8 block: each packed row weighted by a
+    row size (1..16, as pooled windows give), against the oracle's FP8
+    emulation with the same weights and the exact proportional block."""
+    rng = np.random.default_rng(d + 7)
+    B = len(lens)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    rows = int(cu[-1])
+    cap = rows + 29
+    ut = bits(rng.standard_normal((B * T, d)))
+    ui = bits(rng.standard_normal((rows, d)))
+    n = rng.choice([1.0, 1.0, 2.0, 3.0, 4.0, 16.0], size=rows).astype(np.float32)
+    w = scaled_weights(rng, d, 1, std=1.0 / np.sqrt(d))
+    grid = int(np.ceil(np.sqrt(cap)))
+    sh = H.Shape(B=B, H=2 * grid, W=2 * grid, d=d, T=T, heads=heads, mlp=1)
+    w8 = H.DeviceWeightsFP8.from_host(w)
+    in_img = torch.full((cap, d), float("nan"), dtype=torch.bfloat16, device="cuda")
+    in_img[:rows] = H.bf16_from_bits(ui)
+    n_dev = torch.ones(cap, dtype=torch.float32, device="cuda")
+    n_dev[:rows] = torch.from_numpy(n).cuda()
+    out = torch.empty(B * T + cap, d, dtype=torch.float32, device="cuda")
+    wsb = H.hilo_block_fp8_workspace_bytes(sh, cap)
+    ws = torch.full((wsb,), 0xFF, dtype=torch.uint8, device="cuda")
+    H.hilo_block_forward_fp8_prop(sh, w8, to_dev_i32(cu), cap, H.bf16_from_bits(ut) if T else None, in_img,
+                                  H.HILO_BF16, n_dev, out, ws, wsb)
+    H.hilo_sync_status()
+    o = out.cpu().numpy()
+    BT = B * T
+    wq = O.quantize_weights(w)
+    qt, qi = O.block_fp8(ut, ui, cu, T, wq, heads, True, n_img=n)
+    et, ei = O.block(ut, ui, cu, T, w, heads, True, n_img=n)
+    pt, pi = O.block_fp8(ut, ui, cu, T, wq, heads, True)
+    for got, emu, ex, plain, u in ((o[BT:BT + rows], qi, ei, pi, ui), (o[:BT], qt, et, pt, ut)):
+        assert np.all(np.isfinite(got))
+        delta = np.linalg.norm(ex - O.bf16_to_f32(u).astype(np.float64))
+        e_emu = np.linalg.norm(got - emu) / delta
+        e_ex = np.linalg.norm(got - ex) / delta
+        assert e_emu < 0.03, e_emu
+        assert 0.005 < e_ex < 0.1, e_ex
+        # the weights are applied: the unweighted FP8 block is much further away
+        assert np.linalg.norm(got - plain) / delta > 3 * e_emu

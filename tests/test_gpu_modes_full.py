@@ -129,3 +129,37 @@ def test_fp8_block_full_size(H, setup):
     e_ex = np.linalg.norm(g - ex) / delta
     assert e_emu < 0.03, e_emu
     assert 0.005 < e_ex < 0.1, e_ex
+
+
+def test_fp8_block_proportional_attention_full_size(H, setup):
+    """The FP8 block with proportional attention (row sizes from the GPU's
+    own split, bit-exact against the oracle's) at the timed workload's size:
+    sampled rows against the oracle's FP8 emulation with the same weights,
+    and against the exact proportional block within the e4m3 model."""
+    wl, batch, w = setup
+    hp, sh = run(H, wl, batch, [H.DeviceWeights.from_host(w)])
+    hp.enable_fp8([H.DeviceWeightsFP8.from_host(w)])
+    hp.run(*inputs(H, batch), fp8=True, prop=True)
+    H.hilo_sync_status()
+    sp = O.split(O.score(batch.x), batch.mask, batch.k_keep, batch.k_mid, wl.H, wl.W, wl.levels)
+    check_split(hp, sp, wl)
+    n = O.row_sizes(sp)
+    rows = int(sp.cu_img[-1])
+    assert np.array_equal(hp.n_img[:rows].cpu().numpy(), n.astype(np.float32))
+    packed = O.pack(batch.x, sp)
+    got = hp.out.cpu().numpy()
+    tr, ir = sampled(wl, sp.cu_img, 53, n=30)
+    txt = batch.text.reshape(-1, wl.d)
+    qt, qi = O.block_rows_fp8(txt, packed, sp.cu_img, wl.T, O.quantize_weights(w), wl.heads, wl.mlp, 0, tr, ir,
+                              n_img=n)
+    et, ei = O.block_rows(txt, packed, sp.cu_img, wl.T, O.weights_f64(w), wl.heads, wl.mlp, 0, tr, ir, n_img=n)
+    u = np.concatenate([O.bf16_to_f32(txt[tr]), O.bf16_to_f32(packed[ir])]).astype(np.float64)
+    g = np.concatenate([got[tr], got[wl.T + ir]])
+    emu = np.concatenate([qt, qi])
+    ex = np.concatenate([et, ei])
+    assert np.all(np.isfinite(g))
+    delta = np.linalg.norm(ex - u)
+    e_emu = np.linalg.norm(g - emu) / delta
+    e_ex = np.linalg.norm(g - ex) / delta
+    assert e_emu < 0.03, e_emu
+    assert 0.005 < e_ex < 0.1, e_ex
