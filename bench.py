@@ -870,9 +870,10 @@ def run_hilo(args):
 
     # ---- timed region: K steps. Every INSTR-th step carries per-kernel CUDA
     # events on the launching stream (an event between two kernels ends the
-    # programmatic overlap of their launches, so only those steps pay for it).
+    # programmatic overlap of their launches, so only those steps pay for it;
+    # one step in 32 in long runs, at least 3 instrumented steps in short ones).
     K = args.steps
-    INSTR = 8
+    INSTR = 32 if K >= 96 else max(1, K // 3)
     inst = list(range(0, K, INSTR))
     ev = {i: [torch.cuda.Event(enable_timing=True) for _ in range(13)] for i in inst}
     for row in ev.values():
