@@ -43,7 +43,9 @@ constexpr int STAGE_BYTES = 2 * HALF_BYTES; // A + W slices of this CTA
 constexpr int THREADS = 192;
 constexpr uint32_t TMEM_COLS = 512;         // two 128 x 256 fp32 accumulators
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + EPI_SMEM_BYTES + 1024 + 256;
-constexpr int SPLIT_MIN_KB = 16;            // shortest K piece of a tile cut along K
+constexpr int SPLIT_MIN_KB = 32;            // shortest piece of a tile cut into equal K pieces
+constexpr int SPLIT_MAX = 8;                // most equal pieces per tile
+constexpr int STREAM_MIN_KB = 16;           // shortest stream-K range
 
 struct Params {
   int N, K;
@@ -95,33 +97,61 @@ struct Work {
   int t, k0, k1;
 };
 
+// Pieces per tile of the partial round: the count that makes the longest
+// pair's share of the round (rounds of pieces x piece length, in k-blocks)
+// shortest, with pieces of at least SPLIT_MIN_KB k-blocks, so that a piece's
+// main loop still hides the reduce-add epilogue of the piece before it. Ties
+// go to fewer pieces.
+__device__ __forceinline__ int tail_splits(int rem, int ncl, int kb) {
+  if (rem == 0) return 1;
+  int best = 1, cost = kb;  // rem < ncl: one round of whole tiles
+  for (int s = 2; s <= SPLIT_MAX && kb / s >= SPLIT_MIN_KB; ++s) {
+    const int c = ((rem * s + ncl - 1) / ncl) * ((kb + s - 1) / s);
+    if (c < cost) {
+      best = s;
+      cost = c;
+    }
+  }
+  return best;
+}
+
 // The work of pair `cid` of `ncl`. Tiles are dealt round-robin, whole, while
 // a full round remains. When the output is accumulated in place (fp32 +=,
-// written by TMA reduce-add) the tiles of the last, partial round are instead
-// cut along K so that every pair gets the same number of k-blocks
-// (stream-K): each piece adds its partial sum to the output, and only the
-// piece that starts at k = 0 adds the bias. Other epilogues deal every tile
-// whole. All roles of the pair walk the same sequence.
+// written by TMA reduce-add) the tiles of the last, partial round are cut
+// along K instead; each piece adds its partial sum to the output, and only
+// the piece that starts at k = 0 adds the bias. Two cuts:
+//  * equal pieces (tail_splits of them per tile, when that shortens the
+//    round), dealt round-robin piece-major: the pieces that run at the same
+//    time cover one or two K ranges, so the pairs share those slices of A
+//    and W in L2 even when A and W together exceed it;
+//  * otherwise stream-K: the round's k-blocks in equal contiguous ranges of
+//    at least STREAM_MIN_KB, one per pair, each spanning one or two tiles
+//    (shorter than whole pieces, but every pair at its own K offset).
+// Other epilogues deal every tile whole. All roles of the pair walk the same
+// sequence.
 struct WorkIter {
-  int t, t_end, ncl, kb;
-  long long lo, hi;  // this pair's k-block range in the partial round
+  int t, t_end, ncl, kb, rem, nsplit, u, u_end;
+  long long lo, hi;  // stream-K: this pair's k-block range, over the whole tile sequence
   __device__ WorkIter(const Sched& sc, int cid, int ncl_, int kblocks, bool split) {
     ncl = ncl_;
     kb = kblocks;
-    const int rem = split && sc.total > ncl ? sc.total % ncl : 0;
+    rem = split && sc.total > ncl ? sc.total % ncl : 0;
     t_end = sc.total - rem;
     t = cid;
-    // pieces of at least SPLIT_MIN_KB k-blocks: the partial round goes to
-    // fewer pairs when it is short
-    const long long w = static_cast<long long>(rem) * kblocks;
-    const int np = static_cast<int>(max(1LL, min(static_cast<long long>(ncl), w / SPLIT_MIN_KB)));
+    nsplit = tail_splits(rem, ncl, kblocks);
+    u = cid;
+    u_end = nsplit > 1 ? rem * nsplit : 0;
     lo = hi = 0;
-    if (cid < np) {
-      lo = w * cid / np;
-      hi = w * (cid + 1) / np;
+    if (rem > 0 && nsplit == 1) {
+      const long long w = static_cast<long long>(rem) * kblocks;
+      const int np = static_cast<int>(max(1LL, min(static_cast<long long>(ncl), w / STREAM_MIN_KB)));
+      if (cid < np) {
+        lo = w * cid / np;
+        hi = w * (cid + 1) / np;
+      }
+      lo += static_cast<long long>(t_end) * kblocks;
+      hi += static_cast<long long>(t_end) * kblocks;
     }
-    lo += static_cast<long long>(t_end) * kblocks;  // in k-blocks of the whole tile sequence
-    hi += static_cast<long long>(t_end) * kblocks;
   }
   __device__ bool next(Work& w) {
     if (t < t_end) {
@@ -129,6 +159,14 @@ struct WorkIter {
       w.k0 = 0;
       w.k1 = kb;
       t += ncl;
+      return true;
+    }
+    if (u < u_end) {
+      const int s = u / rem;  // piece index: u_end > 0 implies rem > 0
+      w.t = t_end + (u - s * rem);
+      w.k0 = s * kb / nsplit;
+      w.k1 = (s + 1) * kb / nsplit;
+      u += ncl;
       return true;
     }
     if (lo >= hi) return false;
