@@ -410,8 +410,9 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
         umma_commit(&s_full[i]);
       };
       // O_i (+)= P_i V: P_i from the first 64 TMEM columns of S_i (8 columns =
-      // 16 keys per MMA), V from stage vst
-      auto issue_pv = [&](int i, int vst, bool acc) {
+      // 16 keys per MMA), V from stage vst. The last PV_i of a job commits
+      // o_done[i] (one phase per job with steps for warpgroup i)
+      auto issue_pv = [&](int i, int vst, bool acc, bool last) {
         const uint32_t v_base = smem_u32(sV(vst));
 #pragma unroll
         for (int k = 0; k < BKV / 16; ++k) {
@@ -419,7 +420,7 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
           umma_bf16_tmem_a(tmem + 256u + 128u * i, tmem + 128u * i + 8u * k, bd, idesc_o,
                            (acc || k > 0) ? 1u : 0u);
         }
-        umma_commit(&o_done[i]);
+        if (last) umma_commit(&o_done[i]);
       };
       bool ok = true;
       uint32_t kt = 0, sc0 = 0, sc1 = 0;
@@ -468,7 +469,7 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
               break;
             }
             tc_fence_after();
-            issue_pv(0, kv_stage(kt, t), s > 0);
+            issue_pv(0, kv_stage(kt, t), s > 0, s + 1 == n0);
             if (!jb.pair) umma_commit(&v_empty[kv_stage(kt, t)]);
             if (s + 1 < n0) {
               const int t2 = job_tile(jb, 0, s + 1);
@@ -482,17 +483,20 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
             }
           }
           if (s < n1) {
+            // in a pair job, V tile t and K tile t2 are the ones warpgroup 0's
+            // products above already waited for
             const int t = job_tile(jb, 1, s);
-            if (!mbar_wait(&p_full[1], (sc1 + s) & 1u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 8) || !wait_v(t)) {
+            if (!mbar_wait(&p_full[1], (sc1 + s) & 1u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 8) ||
+                (!jb.pair && !wait_v(t))) {
               ok = false;
               break;
             }
             tc_fence_after();
-            issue_pv(1, kv_stage(kt, t), s > 0);
+            issue_pv(1, kv_stage(kt, t), s > 0, s + 1 == n1);
             umma_commit(&v_empty[kv_stage(kt, t)]);
             if (s + 1 < n1) {
               const int t2 = job_tile(jb, 1, s + 1);
-              if (!wait_k(t2)) {
+              if (!jb.pair && !wait_k(t2)) {
                 ok = false;
                 break;
               }
@@ -550,13 +554,16 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
       cp_async_commit();
     };
     bool ok = true;
-    uint32_t kt = 0, sc0 = 0, sc1 = 0;
+    // sc*: S phases so far (one per step); oc*: o_done phases so far (one
+    // per job in which the warpgroup has steps)
+    uint32_t kt = 0, sc0 = 0, sc1 = 0, oc0 = 0, oc1 = 0;
     long long g = g_begin;
     Job jb;
     for (uint32_t jn = 0; ok && next_job(p, g, g_end, jb); ++jn) {
       const int n0 = job_steps(jb, 0), n1 = job_steps(jb, 1);
       const int n = i ? n1 : n0;
       const uint32_t sc = i ? sc1 : sc0;
+      const uint32_t oc = i ? oc1 : oc0;
       float m = -INFINITY, l = 0.f;
       // ragged key tile: rows past `valid` hold other tokens (or stale data);
       // the warpgroup that owns V tile t (the first one in a pair) zeroes
@@ -734,10 +741,9 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
       }
       float a0 = 1.f, a1 = 0.f, inv = 1.f;
       if (ok && writer) {
-        bool done = mbar_wait_warp(&o_done[i], (sc + n - 1) & 1u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 14);
+        bool done = mbar_wait_warp(&o_done[i], oc & 1u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 14);
         if (!jb.pair && n1 > 0)
-          done = done && mbar_wait_warp(&o_done[1], (sc1 + n1 - 1) & 1u, abort_flag, err,
-                                        DEV_TIMEOUT_ATTN + 256 * 15);
+          done = done && mbar_wait_warp(&o_done[1], oc1 & 1u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 15);
         ok = done;
         if (ok) {
           tc_fence_after();
@@ -810,6 +816,8 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
       if (threadIdx.x == 0) mbar_arrive(epi_done);
       sc0 += static_cast<uint32_t>(n0);
       sc1 += static_cast<uint32_t>(n1);
+      oc0 += n0 > 0 ? 1u : 0u;
+      oc1 += n1 > 0 ? 1u : 0u;
       kt += static_cast<uint32_t>(jb.nkv);
     }
     if (PROP) cp_async_wait<0>();
