@@ -170,6 +170,47 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// One lane of the warp, the same one for every call with all lanes active.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t r;
+  asm volatile("{\n\t.reg .pred p;\n\telect.sync _|p, 0xffffffff;\n\tselp.u32 %0, 1, 0, p;\n\t}" : "=r"(r));
+  return r != 0;
+}
+
+// The two 32-bit words of a 128-byte-swizzle shared-memory descriptor: the
+// low word holds start address >> 4 (bits 0..13) and LBO >> 4 (bits
+// 16..29), the high word SBO >> 4, the descriptor version (bit 46) and the
+// swizzle mode (bits 61..63). Shared addresses stay below 2^18 bytes, so
+// adding an offset >> 4 to a low word never carries into the LBO field.
+__host__ __device__ constexpr uint32_t sw128_lo_lbo(uint32_t lbo) { return ((lbo >> 4) & 0x3FFFu) << 16; }
+__host__ __device__ constexpr uint32_t sw128_hi(uint32_t sbo) {
+  return ((sbo >> 4) & 0x3FFFu) | (1u << 14) | (2u << 29);
+}
+
+// tcgen05.mma kind::f16, A and B from shared memory, descriptors given as words
+__device__ __forceinline__ void umma_bf16_w(uint32_t d_tmem, uint32_t a_lo, uint32_t b_lo, uint32_t hi,
+                                            uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t.reg .b64 da, db;\n\t"
+      "setp.ne.b32 p, %5, 0;\n\t"
+      "mov.b64 da, {%1, %3};\n\t"
+      "mov.b64 db, {%2, %3};\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], da, db, %4, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_lo), "r"(b_lo), "r"(hi), "r"(idesc), "r"(acc)
+      : "memory");
+}
+// the same with A from tensor memory
+__device__ __forceinline__ void umma_bf16_tmem_a_w(uint32_t d_tmem, uint32_t a_tmem, uint32_t b_lo, uint32_t hi,
+                                                   uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t.reg .b64 db;\n\t"
+      "setp.ne.b32 p, %5, 0;\n\t"
+      "mov.b64 db, {%2, %3};\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], db, %4, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "r"(b_lo), "r"(hi), "r"(idesc), "r"(acc)
+      : "memory");
+}
+
 // The largest of three floats in one instruction (three-input max.f32). A
 // maximum is exact, so grouping the row's values by threes gives the same
 // result as any other order.
@@ -393,134 +434,154 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
       }
     }
   } else if (warp == MMA_WARP) {
-    if (lane == 0) {
-      // ---------------- MMA issuer
-      const uint32_t idesc_s = idesc_bf16(BQ, BKV, 0, 0);
-      const uint32_t idesc_o = idesc_bf16(BQ, HD, 0, 1);
-      // S_i = Q_qb K^T (K from stage kst)
-      auto issue_s = [&](int i, int qb, int kst) {
-        const uint32_t q_base = smem_u32(sQ(qb));
-        const uint32_t k_base = smem_u32(sK(kst));
+    // ---------------- MMA issuer. The whole warp walks the schedule and
+    // waits, so that the stage indices and descriptor words stay
+    // warp-uniform (no per-MMA moves into the uniform datapath); one elected
+    // lane issues the MMAs and commits. Each MMA's shared-memory descriptor
+    // is a precomputed high word and a low word that is one add away from
+    // its operand's base (start address >> 4 in the low 14 bits, LBO above).
+    const bool leader = elect_one();
+    constexpr uint32_t idesc_s = idesc_bf16(BQ, BKV, 0, 0);
+    constexpr uint32_t idesc_o = idesc_bf16(BQ, HD, 0, 1);
+    constexpr uint32_t TILE16 = C::TILE_BYTES >> 4;
+    const uint32_t base16 = smem_u32(smem) >> 4;
+    const uint32_t q_lo = base16 + (C::OFF_Q >> 4) + sw128_lo_lbo(16);
+    const uint32_t k_lo = base16 + (C::OFF_K >> 4) + sw128_lo_lbo(16);
+    const uint32_t v_lo = base16 + (C::OFF_V >> 4) + sw128_lo_lbo(BOX_BYTES);
+    constexpr uint32_t hi = sw128_hi(1024);
+    // S_i = Q_qb K^T (K from stage kst)
+    auto issue_s = [&](int i, int qb, int kst) {
+      if (leader) {
+        const uint32_t a = q_lo + static_cast<uint32_t>(qb) * TILE16, b = k_lo + static_cast<uint32_t>(kst) * TILE16;
 #pragma unroll
         for (int k = 0; k < HD / 16; ++k) {
-          const uint32_t off = (k >> 2) * BOX_BYTES + (k & 3) * 32;
-          umma_bf16(tmem + 128u * i, sw128_desc(q_base + off, 16, 1024),
-                    sw128_desc(k_base + off, 16, 1024), idesc_s, k > 0 ? 1u : 0u);
+          const uint32_t off = static_cast<uint32_t>((k >> 2) * BOX_BYTES + (k & 3) * 32) >> 4;
+          umma_bf16_w(tmem + 128u * i, a + off, b + off, hi, idesc_s, k > 0 ? 1u : 0u);
         }
         umma_commit(&s_full[i]);
-      };
-      // O_i (+)= P_i V: P_i from the first 64 TMEM columns of S_i (8 columns =
-      // 16 keys per MMA), V from stage vst. The last PV_i of a job commits
-      // o_done[i] (one phase per job with steps for warpgroup i)
-      auto issue_pv = [&](int i, int vst, bool acc, bool last) {
-        const uint32_t v_base = smem_u32(sV(vst));
-#pragma unroll
-        for (int k = 0; k < BKV / 16; ++k) {
-          const uint64_t bd = sw128_desc(v_base + k * 2048, BOX_BYTES, 1024);
-          umma_bf16_tmem_a(tmem + 256u + 128u * i, tmem + 128u * i + 8u * k, bd, idesc_o,
-                           (acc || k > 0) ? 1u : 0u);
-        }
-        if (last) umma_commit(&o_done[i]);
-      };
-      bool ok = true;
-      uint32_t kt = 0, sc0 = 0, sc1 = 0;
-      long long g = g_begin;
-      Job jb;
-      for (uint32_t jn = 0; ok && next_job(p, g, g_end, jb); ++jn) {
-        const int n0 = job_steps(jb, 0), n1 = job_steps(jb, 1);
-        const int qb1 = jb.pair ? 1 : 0;  // the Q buffer of warpgroup 1
-        auto wait_k = [&](int t) {
-          return mbar_wait(&k_full[kv_stage(kt, t)], kv_phase(kt, t), abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 4);
-        };
-        auto wait_v = [&](int t) {
-          return mbar_wait(&v_full[kv_stage(kt, t)], kv_phase(kt, t), abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 6);
-        };
-        if (!mbar_wait(q_full, jn & 1u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 3) || !wait_k(0)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        // the first S of each warpgroup; a pair shares key tile 0, a split
-        // job gives warpgroup 1 key tile 1
-        issue_s(0, 0, kv_stage(kt, 0));
-        if (jb.pair) {
-          issue_s(1, 1, kv_stage(kt, 0));
-          umma_commit(&k_empty[kv_stage(kt, 0)]);
-        } else {
-          umma_commit(&k_empty[kv_stage(kt, 0)]);
-          if (n1 > 0) {
-            if (!wait_k(1)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
-            issue_s(1, 0, kv_stage(kt, 1));
-            umma_commit(&k_empty[kv_stage(kt, 1)]);
-          }
-        }
-        // ping-pong: PV_0(s), S_0(s+1), PV_1(s), S_1(s+1); S_i(s+1)
-        // overwrites P_i(s) only after PV_i(s), in issue order
-        const int nmax = n0 > n1 ? n0 : n1;
-        for (int s = 0; s < nmax && ok; ++s) {
-          if (s < n0) {
-            const int t = job_tile(jb, 0, s);
-            if (!mbar_wait(&p_full[0], (sc0 + s) & 1u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 5) || !wait_v(t)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
-            issue_pv(0, kv_stage(kt, t), s > 0, s + 1 == n0);
-            if (!jb.pair) umma_commit(&v_empty[kv_stage(kt, t)]);
-            if (s + 1 < n0) {
-              const int t2 = job_tile(jb, 0, s + 1);
-              if (!wait_k(t2)) {
-                ok = false;
-                break;
-              }
-              tc_fence_after();
-              issue_s(0, 0, kv_stage(kt, t2));
-              if (!jb.pair) umma_commit(&k_empty[kv_stage(kt, t2)]);
-            }
-          }
-          if (s < n1) {
-            // in a pair job, V tile t and K tile t2 are the ones warpgroup 0's
-            // products above already waited for
-            const int t = job_tile(jb, 1, s);
-            if (!mbar_wait(&p_full[1], (sc1 + s) & 1u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 8) ||
-                (!jb.pair && !wait_v(t))) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
-            issue_pv(1, kv_stage(kt, t), s > 0, s + 1 == n1);
-            umma_commit(&v_empty[kv_stage(kt, t)]);
-            if (s + 1 < n1) {
-              const int t2 = job_tile(jb, 1, s + 1);
-              if (!jb.pair && !wait_k(t2)) {
-                ok = false;
-                break;
-              }
-              tc_fence_after();
-              issue_s(1, qb1, kv_stage(kt, t2));
-              umma_commit(&k_empty[kv_stage(kt, t2)]);
-            }
-          }
-        }
-        // every MMA of this job issued: once they complete, Q may be reloaded
-        umma_commit(q_empty);
-        sc0 += static_cast<uint32_t>(n0);
-        sc1 += static_cast<uint32_t>(n1);
-        kt += static_cast<uint32_t>(jb.nkv);
       }
-      umma_commit(drain);
-      const uint64_t t0 = globaltimer_ns();
-      while (!mbar_try_wait(smem_u32(drain), 0u)) {
-        if (globaltimer_ns() - t0 > HILO_WAIT_LIMIT_NS) {
-          atomicExch(err, DEV_TIMEOUT_ATTN + 256 * 9);
-          break;
+      __syncwarp();
+    };
+    // O_i (+)= P_i V: P_i from the first 64 TMEM columns of S_i (8 columns =
+    // 16 keys per MMA), V from stage vst. The last PV_i of a job commits
+    // o_done[i] (one phase per job with steps for warpgroup i)
+    auto issue_pv = [&](int i, int vst, bool acc, bool last) {
+      if (leader) {
+        const uint32_t b = v_lo + static_cast<uint32_t>(vst) * TILE16;
+#pragma unroll
+        for (int k = 0; k < BKV / 16; ++k)
+          umma_bf16_tmem_a_w(tmem + 256u + 128u * i, tmem + 128u * i + 8u * k, b + ((k * 2048) >> 4), hi, idesc_o,
+                             (acc || k > 0) ? 1u : 0u);
+        if (last) umma_commit(&o_done[i]);
+      }
+      __syncwarp();
+    };
+    auto commit = [&](uint64_t* bar) {
+      if (leader) umma_commit(bar);
+      __syncwarp();
+    };
+    bool ok = true;
+    uint32_t kt = 0, sc0 = 0, sc1 = 0;
+    long long g = g_begin;
+    Job jb;
+    for (uint32_t jn = 0; ok && next_job(p, g, g_end, jb); ++jn) {
+      const int n0 = job_steps(jb, 0), n1 = job_steps(jb, 1);
+      const int qb1 = jb.pair ? 1 : 0;  // the Q buffer of warpgroup 1
+      auto wait_k = [&](int t) {
+        return mbar_wait_warp(&k_full[kv_stage(kt, t)], kv_phase(kt, t), abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 4);
+      };
+      auto wait_v = [&](int t) {
+        return mbar_wait_warp(&v_full[kv_stage(kt, t)], kv_phase(kt, t), abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 6);
+      };
+      if (!mbar_wait_warp(q_full, jn & 1u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 3) || !wait_k(0)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      // the first S of each warpgroup; a pair shares key tile 0, a split
+      // job gives warpgroup 1 key tile 1
+      issue_s(0, 0, kv_stage(kt, 0));
+      if (jb.pair) {
+        issue_s(1, 1, kv_stage(kt, 0));
+        commit(&k_empty[kv_stage(kt, 0)]);
+      } else {
+        commit(&k_empty[kv_stage(kt, 0)]);
+        if (n1 > 0) {
+          if (!wait_k(1)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          issue_s(1, 0, kv_stage(kt, 1));
+          commit(&k_empty[kv_stage(kt, 1)]);
         }
+      }
+      // ping-pong: PV_0(s), S_0(s+1), PV_1(s), S_1(s+1); S_i(s+1)
+      // overwrites P_i(s) only after PV_i(s), in issue order
+      const int nmax = n0 > n1 ? n0 : n1;
+      for (int s = 0; s < nmax && ok; ++s) {
+        if (s < n0) {
+          const int t = job_tile(jb, 0, s);
+          if (!mbar_wait_warp(&p_full[0], (sc0 + s) & 1u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 5) ||
+              !wait_v(t)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          issue_pv(0, kv_stage(kt, t), s > 0, s + 1 == n0);
+          if (!jb.pair) commit(&v_empty[kv_stage(kt, t)]);
+          if (s + 1 < n0) {
+            const int t2 = job_tile(jb, 0, s + 1);
+            if (!wait_k(t2)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            issue_s(0, 0, kv_stage(kt, t2));
+            if (!jb.pair) commit(&k_empty[kv_stage(kt, t2)]);
+          }
+        }
+        if (s < n1) {
+          // in a pair job, V tile t and K tile t2 are the ones warpgroup 0's
+          // products above already waited for
+          const int t = job_tile(jb, 1, s);
+          if (!mbar_wait_warp(&p_full[1], (sc1 + s) & 1u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 8) ||
+              (!jb.pair && !wait_v(t))) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          issue_pv(1, kv_stage(kt, t), s > 0, s + 1 == n1);
+          commit(&v_empty[kv_stage(kt, t)]);
+          if (s + 1 < n1) {
+            const int t2 = job_tile(jb, 1, s + 1);
+            if (!jb.pair && !wait_k(t2)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            issue_s(1, qb1, kv_stage(kt, t2));
+            commit(&k_empty[kv_stage(kt, t2)]);
+          }
+        }
+      }
+      // every MMA of this job issued: once they complete, Q may be reloaded
+      commit(q_empty);
+      sc0 += static_cast<uint32_t>(n0);
+      sc1 += static_cast<uint32_t>(n1);
+      kt += static_cast<uint32_t>(jb.nkv);
+    }
+    // every issued MMA has completed before TMEM is freed, also after an
+    // abort (so this wait ignores the abort flag; it is bounded by time)
+    commit(drain);
+    const uint64_t t0 = globaltimer_ns();
+    while (!mbar_try_wait(smem_u32(drain), 0u)) {
+      if (globaltimer_ns() - t0 > HILO_WAIT_LIMIT_NS) {
+        if (leader) atomicExch(err, DEV_TIMEOUT_ATTN + 256 * 9);
+        break;
       }
     }
+    __syncwarp();
     }
   } else {
     setmaxnreg_inc<SOFTMAX_REGS>();
@@ -722,7 +783,10 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
           tmem_st32(tS + 32 * h2, pk);
         }
         tmem_st_wait();
-        fence_proxy_async_smem();  // the zeroed V rows, if any, are read by the tensor core
+        // V rows zeroed above (ragged tile, owning warpgroup) are read by the
+        // tensor core: make them visible to the async proxy before P_i is
+        // handed over; other steps wrote no shared memory
+        if ((jb.pair ? i == 0 : true) && valid < BKV) fence_proxy_async_smem();
         tc_fence_before();
         mbar_arrive(&p_full[i]);
       }
