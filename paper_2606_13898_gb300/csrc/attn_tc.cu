@@ -835,18 +835,7 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
           constexpr int RPI = 32 / UNITS;  // rows per store instruction
           uint4* stage = reinterpret_cast<uint4*>(smem + C::OFF_K) + warp * 32 * UNITS;
           const bool merge = !jb.pair && n1 > 0;
-#pragma unroll 1
-          for (int c = 0; c < HD / 32; ++c) {
-            float o[32];
-            tmem_ld32(tO + c * 32, o);
-            tmem_ld_wait();
-            if (merge) {
-              float o1[32];
-              tmem_ld32(tO1 + c * 32, o1);
-              tmem_ld_wait();
-#pragma unroll
-              for (int j = 0; j < 32; ++j) o[j] = o[j] * a0 + o1[j] * a1;
-            }
+          auto stage_chunk = [&](int c, const float* o) {
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
               uint4 v;
@@ -855,6 +844,29 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
               v.z = pack_bf16x2(o[8 * j + 4] * inv, o[8 * j + 5] * inv);
               v.w = pack_bf16x2(o[8 * j + 6] * inv, o[8 * j + 7] * inv);
               stage[lane * UNITS + ((4 * c + j) ^ (lane & (UNITS - 1)))] = v;
+            }
+          };
+          if (!merge) {
+            // all of O's columns in flight before one wait (the softmax's
+            // registers are free here)
+            float o[HD];
+#pragma unroll
+            for (int c = 0; c < HD / 32; ++c) tmem_ld32(tO + c * 32, o + c * 32);
+#pragma unroll
+            for (int c = 0; c < HD / 32; ++c) tmem_ld_wait_regs(o + c * 32);
+#pragma unroll
+            for (int c = 0; c < HD / 32; ++c) stage_chunk(c, o + c * 32);
+          } else {
+#pragma unroll 1
+            for (int c = 0; c < HD / 32; ++c) {
+              float o[32], o1[32];
+              tmem_ld32(tO + c * 32, o);
+              tmem_ld32(tO1 + c * 32, o1);
+              tmem_ld_wait_regs(o);
+              tmem_ld_wait_regs(o1);
+#pragma unroll
+              for (int j = 0; j < 32; ++j) o[j] = o[j] * a0 + o1[j] * a1;
+              stage_chunk(c, o);
             }
           }
           __syncwarp();
