@@ -29,7 +29,12 @@
 //   warp 8       TMA: Q tiles, then K tiles (two stages), 128-byte
 //                swizzled boxes of 64 columns
 //   warp 10      TMA: V tiles (two stages)
-//   warp 9       MMA: S_i = Q_i K^T into TMEM, O_i += P_i V into TMEM
+//   warp 9       MMA: S_i = Q_i K^T into TMEM, O_i += P_i V into TMEM. The
+//                whole warp walks the schedule and waits, so that stage
+//                indices and descriptor words stay warp-uniform; one elected
+//                lane issues. (With one lane alone, each MMA's descriptor
+//                arithmetic sat on that lane's dependent chain and the issue
+//                fell behind the tensor pipe.)
 //   warp 11      idle (the third warpgroup gives its registers away)
 // Tensor memory holds S_0 | S_1 | O_0 | O_1 (128 columns each). A softmax
 // warpgroup reads S_i once into registers and writes the probabilities P_i
