@@ -126,6 +126,12 @@ class ClockSampler:
 
 # -------------------------------------------------------------- workloads --
 
+def ordinal(n: int) -> str:
+    """1st, 2nd, 3rd, 4th, ..., 11th, 12th, 13th, ..., 21st, 32nd."""
+    suffix = "th" if 10 <= n % 100 <= 20 else {1: "st", 2: "nd", 3: "rd"}.get(n % 10, "th")
+    return f"{n}{suffix}"
+
+
 def workload(ratio: str):
     from paper_2606_13898_gb300 import inputs as I
     return I.block_64(keep_ratio=ratio)
@@ -984,7 +990,7 @@ def run_hilo(args):
                      "traffic": traffic, "peak_source": f"{peak_src} bf16 dense (burst)" +
                      (" x 2 (nominal fp8 : bf16)" if fp8 else ""),
                      "algorithmic": f"24*M*d^2 FLOP per step over 4 launches, M={M} rows",
-                     "timed_launches": f"events on every {INSTR}th step of the timed region ({len(inst)} steps)"},
+                     "timed_launches": f"events on every {ordinal(INSTR)} step of the timed region ({len(inst)} steps)"},
         "kernels": kernels,
         "gpu_launches": int(launches),
         "clocks": clk,
