@@ -537,11 +537,13 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
           if (!jb.pair) commit(&v_empty[kv_stage(kt, t)]);
           if (s + 1 < n0) {
             const int t2 = job_tile(jb, 0, s + 1);
+            // no tcgen05 fence here: S reads only TMA-written Q and K (ordered
+            // by their mbarrier), and it follows the PV block above, whose
+            // fence already ordered the softmax's TMEM accesses, in issue order
             if (!wait_k(t2)) {
               ok = false;
               break;
             }
-            tc_fence_after();
             issue_s(0, 0, kv_stage(kt, t2));
             if (!jb.pair) commit(&k_empty[kv_stage(kt, t2)]);
           }
@@ -564,7 +566,6 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
               ok = false;
               break;
             }
-            tc_fence_after();
             issue_s(1, qb1, kv_stage(kt, t2));
             commit(&k_empty[kv_stage(kt, t2)]);
           }
