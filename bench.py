@@ -649,6 +649,30 @@ def time_configs(H, I, torch, stream, steps: int, bf16_peak: float, peak_src: st
         return (H.bf16_from_bits(b.x), H.bf16_from_bits(b.text), torch.from_numpy(b.mask).cuda(),
                 torch.from_numpy(b.k_keep).cuda(), torch.from_numpy(b.k_mid).cuda())
 
+    def graph_ms(fn) -> float:
+        """fn(stream) captured once in a CUDA graph, then replayed `steps`
+        times back to back on the timing stream: the same launches without
+        the Python host loop between them (at small sizes that loop, not the
+        GPU, sets the eager pace)."""
+        cs = torch.cuda.Stream()
+        cs.wait_stream(stream)
+        fn(cs)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=cs):
+            fn(cs)
+        for _ in range(3):
+            g.replay()
+        torch.cuda.synchronize()
+        e0, e1 = ev(), ev()
+        e0.record(stream)
+        for _ in range(steps):
+            g.replay()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        del g
+        return e0.elapsed_time(e1) / steps
+
     for wl in (I.tiny_layer(), I.block_64_batch4(), I.block_128_two_level()):
         b = I.make_batch(wl)
         hw = I.make_weights(wl.d, wl.mlp, seed=I.weight_seed(wl))
@@ -688,6 +712,11 @@ def time_configs(H, I, torch, stream, steps: int, bf16_peak: float, peak_src: st
         b1.record(stream)
         torch.cuda.synchronize()
         dense = b0.elapsed_time(b1) / steps
+        # the same three, replayed from CUDA graphs
+        hot_g = graph_ms(lambda cs: hp.run(x, t, m, kk, km, stream=cs))
+        blk_g = graph_ms(lambda cs: hp.blocks(t, hp.packed, H.HILO_BF16, stream=cs))
+        dense_g = graph_ms(lambda cs: H.hilo_block_forward(sh, dw, cu_dense, hp.cap, t, xr, H.HILO_BF16, hp.out,
+                                                            hp.ws, hp.ws_bytes, cs))
         H.hilo_sync_status()
         blk_tf = block_flops(wl, cu) / (blk * 1e-3) / 1e12
         dense_tf = block_flops(wl, cu_dense.cpu().numpy()) / (dense * 1e-3) / 1e12
@@ -696,7 +725,11 @@ def time_configs(H, I, torch, stream, steps: int, bf16_peak: float, peak_src: st
                         "packed_image_rows": cu.tolist()[1:] if wl.B > 1 else int(cu[-1]),
                         "dense_block_ms": dense, "dense_block_tflops": dense_tf,
                         "dense_frac_bf16": dense_tf / bf16_peak,
-                        "block_speedup_vs_dense": dense / blk, "frac_of": frac_note}
+                        "block_speedup_vs_dense": dense / blk, "frac_of": frac_note,
+                        "cuda_graph": {"hot_path_ms": hot_g, "image_tokens_per_s": n_img / (hot_g * 1e-3),
+                                       "block_ms": blk_g, "dense_block_ms": dense_g,
+                                       "block_speedup_vs_dense": dense_g / blk_g,
+                                       "how": "each replayed back to back from one captured CUDA graph"}}
         del hp, dw
         torch.cuda.empty_cache()
         if with_oracle:
