@@ -172,7 +172,13 @@ class Shape:
         return self.H * self.W
 
     def c(self) -> hilo_shape:
-        return hilo_shape(self.B, self.H, self.W, self.d, self.T, self.heads, int(self.mlp), self.levels, self.lf)
+        """The C struct, built once per (frozen) shape; the C entry points
+        only read it (const hilo_shape*)."""
+        st = self.__dict__.get("_c")
+        if st is None:
+            st = hilo_shape(self.B, self.H, self.W, self.d, self.T, self.heads, int(self.mlp), self.levels, self.lf)
+            self.__dict__["_c"] = st
+        return st
 
 
 @dataclasses.dataclass
@@ -196,8 +202,15 @@ class SplitBuffers:
             tok_row=torch.empty(n, dtype=torch.int32, device=device))
 
     def c(self) -> hilo_split_out:
-        return hilo_split_out(*(t.data_ptr() for t in (self.labels, self.row_src, self.counts, self.cu_img,
-                                                      self.tok_row)))
+        """The C struct of the five device pointers, rebuilt only when one of
+        the tensors is replaced."""
+        ts = (self.labels, self.row_src, self.counts, self.cu_img, self.tok_row)
+        key = tuple(id(t) for t in ts)
+        cached = self.__dict__.get("_c")
+        if cached is None or cached[0] != key:
+            cached = (key, hilo_split_out(*(t.data_ptr() for t in ts)), ts)
+            self.__dict__["_c"] = cached
+        return cached[1]
 
 
 def bf16_from_bits(a: np.ndarray, device="cuda") -> torch.Tensor:
@@ -237,10 +250,16 @@ class DeviceWeights:
         return DeviceWeights(t)
 
     def c(self) -> hilo_block_weights:
-        def sw(s):
-            return hilo_stream_weights(*(_ptr(self.tensors[(s, f)]) for f in
-                                         ("w_qkv", "b_qkv", "w_o", "b_o", "w_1", "b_1", "w_2", "b_2")))
-        return hilo_block_weights(sw("txt"), sw("img"))
+        """The C struct of the block's device pointers, built once: the
+        tensors of a DeviceWeights are fixed after construction."""
+        st = self.__dict__.get("_c")
+        if st is None:
+            def sw(s):
+                return hilo_stream_weights(*(_ptr(self.tensors[(s, f)]) for f in
+                                             ("w_qkv", "b_qkv", "w_o", "b_o", "w_1", "b_1", "w_2", "b_2")))
+            st = hilo_block_weights(sw("txt"), sw("img"))
+            self.__dict__["_c"] = st
+        return st
 
 
 @dataclasses.dataclass
@@ -271,9 +290,15 @@ class DeviceWeightsFP8:
         return DeviceWeightsFP8(t)
 
     def c(self) -> hilo_block_weights_fp8:
-        def sw(s):
-            return hilo_stream_weights_fp8(*(_ptr(self.tensors[(s, f)]) for f in _FP8_FIELDS))
-        return hilo_block_weights_fp8(sw("txt"), sw("img"))
+        """The C struct of the block's device pointers, built once (as for
+        DeviceWeights)."""
+        st = self.__dict__.get("_c")
+        if st is None:
+            def sw(s):
+                return hilo_stream_weights_fp8(*(_ptr(self.tensors[(s, f)]) for f in _FP8_FIELDS))
+            st = hilo_block_weights_fp8(sw("txt"), sw("img"))
+            self.__dict__["_c"] = st
+        return st
 
 
 # ---------------------------------------------------------------------------
