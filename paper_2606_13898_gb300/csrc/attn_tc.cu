@@ -175,6 +175,15 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// mbar_wait_warp on two barriers: both phases must complete. The common case
+// (both already complete) costs two try_waits and one warp vote.
+__device__ __forceinline__ bool mbar_wait2_warp(uint64_t* a, uint32_t pa, uint64_t* b, uint32_t pb,
+                                                volatile int* abort, int* err, int code_a, int code_b) {
+  bool ok = mbar_try_wait(smem_u32(a), pa) && mbar_try_wait(smem_u32(b), pb);
+  if (!ok) ok = mbar_wait(a, pa, abort, err, code_a) && mbar_wait(b, pb, abort, err, code_b);
+  return __all_sync(0xffffffffu, ok);
+}
+
 // One lane of the warp, the same one for every call with all lanes active.
 __device__ __forceinline__ bool elect_one() {
   uint32_t r;
@@ -527,8 +536,8 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
       for (int s = 0; s < nmax && ok; ++s) {
         if (s < n0) {
           const int t = job_tile(jb, 0, s);
-          if (!mbar_wait_warp(&p_full[0], (sc0 + s) & 1u, abort_flag, err, DEV_TIMEOUT_ATTN + 256 * 5) ||
-              !wait_v(t)) {
+          if (!mbar_wait2_warp(&p_full[0], (sc0 + s) & 1u, &v_full[kv_stage(kt, t)], kv_phase(kt, t), abort_flag,
+                               err, DEV_TIMEOUT_ATTN + 256 * 5, DEV_TIMEOUT_ATTN + 256 * 6)) {
             ok = false;
             break;
           }
