@@ -763,12 +763,26 @@ __global__ void __launch_bounds__(ATTN_THREADS, 1)
 #pragma unroll
           for (int u = 0; u < 8; ++u) ls8[u] = 0.f;
           if (full_tile) {
+            // by key pairs: the exponent arguments as one paired fma, the
+            // row-sum partials (2u, 2u+1) of pair c (u = c mod 4) as one
+            // paired add; the same per-lane operations, partition and order
+            // as key j into partial j mod 8 (one issue slot per pair)
+            const uint64_t sc2 = f2(p.scale_log2, p.scale_log2), nm2 = f2(-m_use, -m_use);
+            uint64_t ls4[4];
 #pragma unroll
-            for (int j = 0; j < BKV; ++j) {
-              const float pj = ex2(fmaf(sv[j], p.scale_log2, -m_use));
-              sv[j] = pj;
-              ls8[j & 7] += pj;
+            for (int u = 0; u < 4; ++u) ls4[u] = 0ull;
+#pragma unroll
+            for (int c = 0; c < BKV / 2; ++c) {
+              float a, a1;
+              f2_split(f2_fma(f2(sv[2 * c], sv[2 * c + 1]), sc2, nm2), a, a1);
+              a = ex2(a);
+              a1 = ex2(a1);
+              sv[2 * c] = a;
+              sv[2 * c + 1] = a1;
+              ls4[c & 3] = f2_add(ls4[c & 3], f2(a, a1));
             }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) f2_split(ls4[u], ls8[2 * u], ls8[2 * u + 1]);
           } else {
 #pragma unroll
             for (int j = 0; j < BKV; ++j) {
